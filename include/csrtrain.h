@@ -1,0 +1,240 @@
+/*
+ * csrtrain.h -- C ABI of the GB300 (sm_103a) CSR-weight training step.
+ *
+ * Method: Lee & Lee, "Compressed Learning of Deep Neural Networks for
+ * OpenCL-Capable Embedded Systems", arXiv 1905.07931. A training step over
+ * layers whose weight matrices are held in compressed sparse row form
+ * (Section 3.1): forward product Y = W X (Section 3.2.1), backward product
+ * dX = W^T dY (Section 3.2.2), the dense weight gradient for the l1-proximal
+ * phase and the gradient sampled at the stored entries for the debias phase
+ * (Section 2.4), the soft-threshold proximal update (Section 2.2, Eq. prox,
+ * Section 3.3) followed by re-compaction of the CSR arrays after every update.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Layout. W is M x K (M = outputs, K = inputs). Dense activations are
+ *    feature-major, row-major with the sample index contiguous: X is K x n,
+ *    Y and dY are M x n. (The paper's Caffe orientation X_T = X_B W' holds
+ *    samples in rows; this is its transpose.) All floating-point data is
+ *    IEEE float32; indices are int32; M * K must be below 2^31.
+ *  - Memory. Every pointer inside a csrt_csr and every array argument is a
+ *    DEVICE pointer unless stated otherwise; the csrt_csr struct itself and
+ *    the small out-parameters are HOST memory. The caller owns and allocates
+ *    every buffer. The library allocates no memory of its own.
+ *  - Streams. `stream` is a cudaStream_t passed as void* (NULL = the legacy
+ *    default stream). Every call only enqueues work on that stream; none
+ *    synchronises except csrt_get_status. No call reads nnz on the host:
+ *    nnz lives on the device in row_ptr[M].
+ *  - Workspace. Calls that take `ws` need a device scratch buffer of at least
+ *    csrt_workspace_bytes(...) bytes, initialised once with
+ *    csrt_workspace_init. Its first 256 bytes hold a device status word that
+ *    accumulates data-dependent errors (see CSRT_DEV_*). A workspace serves
+ *    one stream at a time: calls on two streams need two workspaces.
+ *  - Errors. Each call returns CSRT_OK or a CSRT_ERR_* code at once for bad
+ *    arguments or a failed launch; no work is enqueued in that case.
+ *    Data-dependent errors (capacity overflow, a bounded wait that ran out,
+ *    non-finite values) cannot be known on the host without a sync; kernels
+ *    OR them into the device status word, read by csrt_get_status.
+ *    csrt_last_error() returns a message for the last failing call on the
+ *    calling host thread.
+ */
+#ifndef CSRTRAIN_H
+#define CSRTRAIN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Return codes. */
+#define CSRT_OK 0
+#define CSRT_ERR_ARG 1        /* invalid argument: nothing enqueued */
+#define CSRT_ERR_CUDA 2       /* a CUDA runtime call or launch failed */
+#define CSRT_ERR_WORKSPACE 3  /* workspace smaller than required */
+
+/* Device status bits (OR-ed by kernels into the workspace status word). */
+#define CSRT_DEV_CAPACITY 1   /* an output CSR needed more entries than its capacity;
+                                 the CSR written is truncated but structurally valid
+                                 (row_ptr clamped to capacity). required_nnz reports
+                                 the count that was needed. */
+#define CSRT_DEV_TIMEOUT 2    /* a bounded inter-block wait gave up; results invalid */
+#define CSRT_DEV_NONFINITE 4  /* the prox step met a NaN in w - eta*G (dropped) */
+
+/* weight_grad_dense precision. */
+#define CSRT_PREC_FP32 0      /* float32 FMA on the CUDA cores */
+#define CSRT_PREC_TF32 1      /* tcgen05 tensor cores, kind::tf32, float32 accumulate */
+
+/*
+ * A CSR matrix (Section 3.1, Figure "spformats" (iii): row_ptrs, col_indices,
+ * elements), plus an optional transposed copy of the same pattern.
+ *
+ * Section 3.2.2 notes that the backward product reads W column by column,
+ * which row-wise CSR storage cannot serve with coalesced loads, and that a
+ * second, column-ordered copy of the nonzeros would remove the problem. The
+ * t_* arrays are that copy:
+ * W^T in CSR form (entries sorted by column, then row) and, for each CSR
+ * entry k, its position t_pos[k] in the transposed arrays. They are needed by
+ * spmm_bwd_t only; layers whose input gradient is never needed can leave
+ * them NULL.
+ */
+typedef struct csrt_csr {
+    int32_t rows;        /* M */
+    int32_t cols;        /* K */
+    int64_t capacity;    /* allocated entries of col_idx/val (and t_col_idx/t_val/t_pos) */
+    int32_t *row_ptr;    /* [rows+1]; row_ptr[0] = 0, row_ptr[rows] = nnz */
+    int32_t *col_idx;    /* [capacity]; ascending and unique within a row */
+    float *val;          /* [capacity] */
+    int32_t *t_row_ptr;  /* [cols+1] or NULL */
+    int32_t *t_col_idx;  /* [capacity] or NULL: row index of each transposed entry */
+    float *t_val;        /* [capacity] or NULL */
+    int32_t *t_pos;      /* [capacity] or NULL: CSR entry k sits at t_*[t_pos[k]] */
+} csrt_csr;
+
+/* ------------------------------------------------------------------------ */
+/* Workspace and status                                                      */
+/* ------------------------------------------------------------------------ */
+
+/* Bytes of workspace needed by every call below for matrices of at most
+ * `rows` x `cols` and products with at most `max_n` columns. Host only. */
+int csrt_workspace_bytes(int32_t rows, int32_t cols, int32_t max_n, size_t *bytes);
+
+/* Zero the whole workspace (status word included) on `stream`. */
+int csrt_workspace_init(void *ws, size_t ws_bytes, void *stream);
+
+/* Synchronise `stream`, then copy the status bits and the largest required
+ * nnz reported by a capacity overflow to the host. Either out-pointer may be
+ * NULL. Does not clear the status (see csrt_clear_status). */
+int csrt_get_status(const void *ws, int32_t *flags, int64_t *required_nnz, void *stream);
+
+/* Clear the status word on `stream`. */
+int csrt_clear_status(void *ws, void *stream);
+
+/* Message for the last failing call on this host thread ("" if none). */
+const char *csrt_last_error(void);
+
+/* Number of kernels the library launched on the calling host thread since
+ * the last reset (an instrument for counting launches inside a timed region). */
+int64_t csrt_launch_count(int reset);
+
+/* ------------------------------------------------------------------------ */
+/* The training-step calls                                                   */
+/* ------------------------------------------------------------------------ */
+
+/* csr_from_dense -- Section 3.1. Compress a dense row-major rows x cols
+ * matrix, keeping every entry with value != 0 (+0.0 and -0.0 dropped, NaN
+ * and Inf kept) in row-major order. Writes out->row_ptr, col_idx, val; if
+ * out->t_row_ptr is not NULL also builds the transposed arrays
+ * (csr_transpose). out->rows/cols must equal rows/cols. An output needing
+ * more than out->capacity entries sets CSRT_DEV_CAPACITY. */
+int csr_from_dense(const float *dense, int32_t rows, int32_t cols, csrt_csr *out,
+                   void *ws, size_t ws_bytes, void *stream);
+
+/* csr_transpose -- the column-wise copy of Section 3.2.2. Rebuilds
+ * w->t_row_ptr, t_col_idx, t_val and t_pos from w's CSR arrays
+ * (deterministic: entries of a column are ordered by row). All four t_*
+ * pointers must be set. */
+int csr_transpose(csrt_csr *w, void *ws, size_t ws_bytes, void *stream);
+
+/* spmm_fwd -- Section 3.2.1 (dense x compressed', the forward pass).
+ * Y[M x n] = W X[K x n]: Y[i, c] = sum over stored k of row i of
+ * val[k] * X[col_idx[k], c], float32 accumulation. Y is overwritten. */
+int spmm_fwd(const csrt_csr *w, const float *x, int32_t n, float *y,
+             void *ws, size_t ws_bytes, void *stream);
+
+/* spmm_bwd_t -- Section 3.2.2 (dense x compressed, the backward pass).
+ * dX[K x n] = W^T dY[M x n], through the transposed arrays (which must be
+ * current: built by csr_from_dense / csr_transpose / prox_update_compact and
+ * kept in step by debias_update). dX is overwritten. */
+int spmm_bwd_t(const csrt_csr *w, const float *dy, int32_t n, float *dx,
+               void *ws, size_t ws_bytes, void *stream);
+
+/* weight_grad_dense -- gradient of every weight for the prox phase (the
+ * matrix w - eta*G of Section 3.3 needs G at all M x K entries).
+ * G[i, j] = sum_c dY[i, c] X[j, c]; dY is m x n, X is k x n, G is m x k,
+ * all row-major. No 1/n factor is applied. precision: CSRT_PREC_FP32 or
+ * CSRT_PREC_TF32 (operands rounded to TF32, float32 accumulation). */
+int weight_grad_dense(const float *dy, const float *x, int32_t m, int32_t k, int32_t n,
+                      float *g, int32_t precision, void *ws, size_t ws_bytes, void *stream);
+
+/* weight_grad_sddmm -- gradient at the stored entries only, for the debias
+ * phase (Section 2.4: zero weights are not trained).
+ * g_nnz[k] = sum_c dY[i_k, c] X[j_k, c] for every stored entry k = (i_k, j_k).
+ * g_nnz has at least nnz entries. */
+int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_t n,
+                      float *g_nnz, void *ws, size_t ws_bytes, void *stream);
+
+/* prox_update_compact -- Eq. prox with the soft threshold of Section 2.2,
+ * applied to the dense matrix w - eta*G as in Section 3.3, then compacted
+ * back to CSR (Section 4.4: compression after every update).
+ * For every (i, j), row-major, with w = the stored value or +0:
+ *   thr = fl32(eta*lambda), t = fl32(eta*G[i,j]), z = fl32(w - t) (no FMA),
+ *   keep iff |z| > thr, kept value = z - thr (z > 0) or z + thr (z < 0).
+ * G is a dense row-major M x K float32 matrix. w_out must be a different CSR
+ * with the same shape; capacity M*K can never overflow (zero weights may
+ * re-enter). If w_out->t_row_ptr is not NULL the transposed arrays of w_out
+ * are rebuilt too. eta and lambda must be finite and >= 0. */
+int prox_update_compact(const csrt_csr *w_in, const float *g, float eta, float lambda,
+                        csrt_csr *w_out, void *ws, size_t ws_bytes, void *stream);
+
+/* debias_update -- the retraining step of Section 2.4 / Section 4.3 (zero
+ * weights fixed and not updated): val[k] <- fl32(val[k] - fl32(eta*g_nnz[k]))
+ * for every stored entry; row_ptr and col_idx are untouched, and a value
+ * reaching 0.0 stays stored. If w->t_val is not NULL the transposed values
+ * are updated through t_pos. */
+int debias_update(csrt_csr *w, const float *g_nnz, float eta, void *stream);
+
+/* ------------------------------------------------------------------------ */
+/* Network glue (Caffe layers the paper uses but does not describe).         */
+/* Convolution activations are C x (B*H*W) matrices: channel, then sample,   */
+/* then row, then column.                                                    */
+/* ------------------------------------------------------------------------ */
+
+/* y[i, c] += bias[i]; then y = max(y, 0) if relu != 0. In place, m x n. */
+int csrt_bias_act_fwd(float *y, const float *bias, int32_t m, int32_t n, int32_t relu, void *stream);
+
+/* dy[e] = y[e] > 0 ? dy[e] : 0 for e < count (ReLU backward through its output). */
+int csrt_relu_bwd(float *dy, const float *y, int64_t count, void *stream);
+
+/* gb[i] = sum_c dy[i, c]; bias[i] <- fl32(bias[i] - fl32(eta*gb[i])).
+ * gb_out (m floats) may be NULL. Plain SGD, no regulariser. */
+int csrt_bias_grad_sgd(const float *dy, int32_t m, int32_t n, float *bias, float eta,
+                       float *gb_out, void *stream);
+
+/* Mean softmax cross-entropy over the n columns of z (classes x n).
+ * `loss` holds n + 1 floats: loss[1 + c] = -log softmax(z[:, c])[labels[c]]
+ * and loss[0] = their mean (summed in a fixed order).
+ * dz = (softmax(z) - onehot(labels)) / n (the 1/|B| of the minibatch
+ * gradient, Section 2.2). labels are int32 in [0, classes). */
+int csrt_softmax_xent(const float *z, const int32_t *labels, int32_t classes, int32_t n,
+                      float *dz, float *loss, void *stream);
+
+/* Unfold x (c x (b*h*w)) into cols ((c*k*k) x (b*ho*wo)), stride 1, no
+ * padding: cols[c*k*k + ky*k + kx][s*ho*wo + oy*wo + ox] = x[c][s][oy+ky][ox+kx]. */
+int csrt_im2col(const float *x, int32_t c, int32_t b, int32_t h, int32_t w, int32_t k,
+                float *cols, void *stream);
+
+/* Adjoint of csrt_im2col: dx = sum of every column entry onto its pixel. */
+int csrt_col2im(const float *dcols, int32_t c, int32_t b, int32_t h, int32_t w, int32_t k,
+                float *dx, void *stream);
+
+/* 2x2 max pooling, stride 2 (h, w even): y is c x (b*(h/2)*(w/2)); idx (int8)
+ * records the winning window position dy*2+dx, first maximum in scan order. */
+int csrt_maxpool2_fwd(const float *x, int32_t c, int32_t b, int32_t h, int32_t w,
+                      float *y, int8_t *idx, void *stream);
+
+/* Route pooled gradients back: dx (c x (b*h*w)) is overwritten. */
+int csrt_maxpool2_bwd(const float *dy, const int8_t *idx, int32_t c, int32_t b, int32_t h,
+                      int32_t w, float *dx, void *stream);
+
+/* (c x (b*hw)) -> ((c*hw) x b): xf[ci*hw + s][bi] = x[ci][bi*hw + s] (Caffe
+ * flatten order), and its inverse. */
+int csrt_flatten(const float *x, int32_t c, int32_t b, int32_t hw, float *xf, void *stream);
+int csrt_unflatten(const float *xf, int32_t c, int32_t b, int32_t hw, float *x, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CSRTRAIN_H */

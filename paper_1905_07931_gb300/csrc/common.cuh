@@ -1,0 +1,137 @@
+// Internal helpers shared by the CUDA translation units of libcsrtrain.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "csrtrain.h"
+
+namespace csrt {
+
+// ---------------------------------------------------------------------------
+// Workspace header: the first 256 bytes of every workspace.
+// ---------------------------------------------------------------------------
+struct WsHeader {
+    unsigned int flags;             // CSRT_DEV_* bits, OR-ed by kernels
+    unsigned int pad0;
+    unsigned long long required;    // largest nnz an overflowing output needed
+    unsigned int ticket;            // tile ticket of the running compaction
+    unsigned int timeout_site;      // last wait that gave up (diagnostics)
+    unsigned int pad1[58];
+};
+static_assert(sizeof(WsHeader) == 256, "workspace header is 256 bytes");
+constexpr size_t kWsHeaderBytes = 256;
+
+inline char *ws_scratch(void *ws) { return static_cast<char *>(ws) + kWsHeaderBytes; }
+
+// Bounded spin: a wait on another block's flag gives up after this many
+// polls (with nanosleep back-off it is far above any legitimate wait) and
+// reports CSRT_DEV_TIMEOUT instead of hanging.
+constexpr unsigned int kSpinLimit = 1u << 22;
+
+__device__ __forceinline__ void dev_flag(WsHeader *h, unsigned int bits) {
+    atomicOr(&h->flags, bits);
+}
+
+// ---------------------------------------------------------------------------
+// Host-side error reporting
+// ---------------------------------------------------------------------------
+int fail(int code, const char *fmt, ...);
+int check_launch(const char *what);
+void count_launch(int n = 1);
+int num_sms();   // SMs of the current device (cached per device)
+
+#define CSRT_CHECK_CUDA(call)                                                   \
+    do {                                                                        \
+        cudaError_t e_ = (call);                                                \
+        if (e_ != cudaSuccess)                                                  \
+            return ::csrt::fail(CSRT_ERR_CUDA, "%s: %s", #call,                 \
+                                cudaGetErrorString(e_));                        \
+    } while (0)
+
+#define CSRT_ARG(cond, ...)                                                     \
+    do {                                                                        \
+        if (!(cond)) return ::csrt::fail(CSRT_ERR_ARG, __VA_ARGS__);            \
+    } while (0)
+
+inline cudaStream_t as_stream(void *s) { return static_cast<cudaStream_t>(s); }
+
+// ---------------------------------------------------------------------------
+// Workspace sizes of the individual operations (bytes after the header).
+// ---------------------------------------------------------------------------
+size_t compact_scratch_bytes(int64_t elems);
+size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
+size_t spmm_scratch_bytes(int32_t max_n);
+size_t sddmm_scratch_bytes(int64_t capacity, int32_t max_n);
+size_t gemm_scratch_bytes(int32_t m, int32_t k, int32_t max_n);
+
+// Internal entry used by csr_from_dense / prox_update_compact.
+int transpose_impl(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// Device helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long *p) {
+    unsigned long long v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void st_release_u64(unsigned long long *p, unsigned long long v) {
+    asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+__device__ __forceinline__ float4 ldg_f4(const float *p) {
+    return __ldg(reinterpret_cast<const float4 *>(p));
+}
+
+__device__ __forceinline__ float4 ld_stream_f4(const float *p) {
+    float4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0,%1,%2,%3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "l"(p));
+    return v;
+}
+
+template <typename T>
+__host__ __device__ __forceinline__ T imin(T a, T b) {
+    return a < b ? a : b;
+}
+template <typename T>
+__host__ __device__ __forceinline__ T imax(T a, T b) {
+    return a < b ? b : a;
+}
+
+template <typename T>
+__host__ __device__ __forceinline__ T ceil_div(T a, T b) {
+    return (a + b - 1) / b;
+}
+
+// First index in [lo, hi) where the monotone predicate (true ... true,
+// false ... false) is false, or hi. All 32 lanes of a warp call it and get the
+// same answer after about log32(hi - lo) rounds of one probe per lane.
+template <typename Pred>
+__device__ __forceinline__ int64_t warp_first_false(int64_t lo, int64_t hi, Pred pred) {
+    const int lane = threadIdx.x & 31;
+    int64_t len = hi - lo;
+    while (len > 32) {
+        const int64_t idx = lo + ((int64_t)(lane + 1) * len) / 32 - 1;  // last of chunk `lane`
+        const int l = __popc(__ballot_sync(0xffffffffu, pred(idx)));
+        if (l == 32) return hi;
+        const int64_t nlo = lo + ((int64_t)l * len) / 32;
+        hi = lo + ((int64_t)(l + 1) * len) / 32;
+        lo = nlo;
+        len = hi - lo;
+    }
+    const int64_t idx = lo + lane;
+    const bool p = idx < hi && pred(idx);
+    return lo + __popc(__ballot_sync(0xffffffffu, p));
+}
+
+// First position p in [s, e) with col[p] >= target (col ascending in [s, e)).
+__device__ __forceinline__ int64_t warp_lower_bound(const int32_t *__restrict__ col, int64_t s, int64_t e,
+                                                    int32_t target) {
+    return warp_first_false(s, e, [&](int64_t p) { return __ldg(col + p) < target; });
+}
+
+}  // namespace csrt

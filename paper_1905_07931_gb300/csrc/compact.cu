@@ -1,0 +1,516 @@
+// CSR construction and the fused proximal update + re-compaction.
+//
+// csr_from_dense (Section 3.1) and prox_update_compact (Eq. prox with the
+// soft threshold of Section 2.2, applied to the dense w - eta*G as in
+// Section 3.3, compacted after every update as in Section 4.4) are the same
+// stream compaction over the M*K entries in row-major order; they differ only
+// in the predicate and the kept value.
+//
+// Design (GB300): the M*K matrix is viewed as one flat array cut into tiles
+// of 4096 entries. One 256-thread block per tile streams its 16 KB of the
+// dense input with 16-byte loads that bypass L1, evaluates the predicate,
+// ranks the kept entries with a block scan, and learns the number of entries
+// kept by all earlier tiles with a single-pass decoupled look-back
+// (Merrill & Garland) over a per-tile status word. Tiles are numbered by an
+// atomic ticket, so a block only ever waits on blocks that are already
+// running; every wait is bounded and reports CSRT_DEV_TIMEOUT instead of
+// hanging. The dense input is read once and the CSR written once, coalesced.
+// For the prox step, the old CSR entries of the tile's flat range are
+// contiguous in the old arrays; they are scattered into a shared-memory copy
+// of the tile so that w is read once as well.
+//
+// csr_transpose builds the column-wise copy of the pattern that Section 3.2.2
+// asks for (entries ordered by column, then row) in four deterministic
+// kernels: per 32-row block and column a bitmask of the rows present, a scan
+// of the per-block counts down each column, a scan over the columns, and a
+// scatter whose rank inside a block is a popcount of the bitmask.
+#include "common.cuh"
+
+namespace csrt {
+
+constexpr int kCThreads = 256;
+constexpr int kCQuads = 4;                           // float4 per thread
+constexpr int kTile = kCThreads * kCQuads * 4;       // 4096 entries per tile
+constexpr unsigned long long kFlagAgg = 1ull << 32;  // tile aggregate published
+constexpr unsigned long long kFlagInc = 2ull << 32;  // inclusive prefix published
+
+size_t compact_scratch_bytes(int64_t elems) {
+    return (size_t)ceil_div<int64_t>(elems, kTile) * sizeof(unsigned long long);
+}
+
+struct CompactArgs {
+    const float *src;          // dense matrix (from-dense) or G (prox)
+    int32_t rows, cols;
+    int64_t elems;
+    const int32_t *in_row_ptr;  // prox: old CSR
+    const int32_t *in_col;
+    const float *in_val;
+    float eta, thr;
+    int32_t *out_row_ptr;
+    int32_t *out_col;
+    float *out_val;
+    int64_t capacity;
+    WsHeader *hdr;
+    unsigned long long *status;  // one word per tile
+    int64_t num_tiles;
+};
+
+template <bool kProx, bool kVec>
+__global__ void __launch_bounds__(kCThreads) compact_kernel(CompactArgs a) {
+    __shared__ __align__(16) float w_tile[kProx ? kTile : 4];
+    __shared__ int32_t s_rowptr[kProx ? kTile + 2 : 2];
+    __shared__ unsigned long long s_warp[kCThreads / 32];
+    __shared__ unsigned long long s_excl;
+    __shared__ int64_t s_range[2];
+    __shared__ unsigned int s_tile;
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (tid == 0) s_tile = atomicAdd(&a.hdr->ticket, 1u);
+    __syncthreads();
+    const int64_t tile = s_tile;
+    if (tile >= a.num_tiles) return;  // cannot happen: one block per tile
+    const int64_t e0 = tile * kTile;
+    const int64_t e1 = min(e0 + (int64_t)kTile, a.elems);
+    const int64_t K = a.cols;
+
+    // 1. Stream this thread's 16 entries: quad q covers e0 + 4*(q*256 + tid).
+    float v[kCQuads][4];
+#pragma unroll
+    for (int q = 0; q < kCQuads; ++q) {
+        const int64_t e = e0 + 4 * (int64_t)(q * kCThreads + tid);
+        if (kVec && e + 3 < e1) {
+            float4 f = ld_stream_f4(a.src + e);
+            v[q][0] = f.x; v[q][1] = f.y; v[q][2] = f.z; v[q][3] = f.w;
+        } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c) v[q][c] = (e + c < e1) ? a.src[e + c] : 0.f;
+        }
+    }
+
+    // 2. Prox: the old weights of this flat range, scattered into w_tile.
+    if (kProx) {
+        for (int i = tid; i < kTile; i += kCThreads) w_tile[i] = 0.f;
+        const int64_t r0 = e0 / K, r1 = (e1 - 1) / K;  // rows touched, inclusive
+        const int nr = (int)(r1 - r0 + 2);              // row_ptr entries r0..r1+1
+        for (int i = tid; i < nr; i += kCThreads) s_rowptr[i] = a.in_row_ptr[r0 + i];
+        __syncthreads();
+        if (warp == 0) {
+            int64_t s0 = warp_lower_bound(a.in_col, s_rowptr[0], s_rowptr[1], (int32_t)(e0 - r0 * K));
+            if (lane == 0) s_range[0] = s0;
+        } else if (warp == 1) {
+            int64_t s1;
+            if (e1 == (r1 + 1) * K) s1 = s_rowptr[nr - 1];
+            else s1 = warp_lower_bound(a.in_col, s_rowptr[nr - 2], s_rowptr[nr - 1], (int32_t)(e1 - r1 * K));
+            if (lane == 0) s_range[1] = s1;
+        }
+        __syncthreads();
+        const int64_t s0 = s_range[0], s1 = s_range[1];
+        for (int64_t k = s0 + tid; k < s1; k += kCThreads) {
+            int lo = 0, hi = nr - 2;  // last row whose start is <= k
+            while (lo < hi) {
+                int mid = (lo + hi + 1) >> 1;
+                if (s_rowptr[mid] <= k) lo = mid; else hi = mid - 1;
+            }
+            const int64_t f = (r0 + lo) * K + __ldg(a.in_col + k);
+            w_tile[f - e0] = __ldg(a.in_val + k);
+        }
+        __syncthreads();
+    }
+
+    // 3. Predicate and kept value per entry.
+    unsigned int keep = 0;  // bit q*4+c
+    bool nonfinite = false;
+#pragma unroll
+    for (int q = 0; q < kCQuads; ++q) {
+        const int64_t e = e0 + 4 * (int64_t)(q * kCThreads + tid);
+        float4 w4 = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (kProx) w4 = reinterpret_cast<const float4 *>(w_tile)[q * kCThreads + tid];
+        const float wv[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const bool valid = e + c < e1;
+            bool k;
+            if (kProx) {
+                const float t = __fmul_rn(a.eta, v[q][c]);
+                const float z = __fsub_rn(wv[c], t);
+                k = valid && fabsf(z) > a.thr;
+                nonfinite |= valid && isnan(z);
+                v[q][c] = z > 0.f ? __fsub_rn(z, a.thr) : __fadd_rn(z, a.thr);
+            } else {
+                k = valid && v[q][c] != 0.f;
+            }
+            keep |= (unsigned)k << (q * 4 + c);
+        }
+    }
+    if (kProx) {
+        if (__syncthreads_or(nonfinite) && tid == 0) dev_flag(a.hdr, CSRT_DEV_NONFINITE);
+    }
+
+    // 4. Block scan of the four per-quad counts, packed in 16-bit fields.
+    unsigned long long packed = 0;
+#pragma unroll
+    for (int q = 0; q < kCQuads; ++q)
+        packed |= (unsigned long long)__popc((keep >> (q * 4)) & 0xFu) << (16 * q);
+    unsigned long long incl = packed;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        unsigned long long y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    unsigned long long warp_prefix = 0, block_total = 0;
+#pragma unroll
+    for (int w = 0; w < kCThreads / 32; ++w) {
+        const unsigned long long t = s_warp[w];
+        if (w < warp) warp_prefix += t;
+        block_total += t;
+    }
+    const unsigned long long excl = incl - packed + warp_prefix;
+    uint32_t quad_total[kCQuads];
+    uint32_t tile_count = 0;
+#pragma unroll
+    for (int q = 0; q < kCQuads; ++q) {
+        quad_total[q] = (uint32_t)((block_total >> (16 * q)) & 0xFFFFu);
+        tile_count += quad_total[q];
+    }
+
+    // 5. Decoupled look-back for the number of entries kept before this tile.
+    if (warp == 0) {
+        unsigned long long prefix = 0;
+        if (tile == 0) {
+            if (lane == 0) st_release_u64(a.status, kFlagInc | tile_count);
+        } else {
+            if (lane == 0) st_release_u64(a.status + tile, kFlagAgg | tile_count);
+            int64_t pred = tile - 1;
+            unsigned int spins = 0;
+            bool timed_out = false;
+            while (true) {
+                const int64_t idx = pred - lane;
+                unsigned long long st = idx >= 0 ? ld_acquire_u64(a.status + idx) : kFlagInc;
+                while (__any_sync(0xffffffffu, (st >> 32) == 0)) {
+                    if (++spins > kSpinLimit) { timed_out = true; break; }
+                    __nanosleep(64);
+                    if ((st >> 32) == 0) st = ld_acquire_u64(a.status + idx);
+                }
+                if (timed_out) break;
+                const unsigned inc_mask = __ballot_sync(0xffffffffu, (st >> 32) == 2);
+                unsigned long long part = st & 0xffffffffull;
+                if (inc_mask) {
+                    const int first = __ffs(inc_mask) - 1;  // nearest inclusive predecessor
+                    if (lane > first) part = 0;
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
+                prefix += part;
+                if (inc_mask) break;
+                pred -= 32;
+            }
+            if (lane == 0) {
+                if (timed_out) {
+                    dev_flag(a.hdr, CSRT_DEV_TIMEOUT);
+                    a.hdr->timeout_site = 1;
+                }
+                st_release_u64(a.status + tile, kFlagInc | (prefix + tile_count));
+            }
+        }
+        if (lane == 0) s_excl = prefix;
+    }
+    __syncthreads();
+    const int64_t tile_base = (int64_t)s_excl;
+    const int64_t cap = a.capacity;
+
+    // 6. Write kept entries and the row starts that fall in this tile.
+    int64_t quad_base = tile_base;
+#pragma unroll
+    for (int q = 0; q < kCQuads; ++q) {
+        int64_t pos = quad_base + (int64_t)((excl >> (16 * q)) & 0xFFFFu);
+        const int64_t e = e0 + 4 * (int64_t)(q * kCThreads + tid);
+        if (e < e1) {
+            int64_t r = e / K;
+            int64_t col = e - r * K;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                if (e + c < e1) {
+                    if (col == 0) a.out_row_ptr[r] = (int32_t)min(pos, cap);
+                    if ((keep >> (q * 4 + c)) & 1u) {
+                        if (pos < cap) {
+                            a.out_col[pos] = (int32_t)col;
+                            a.out_val[pos] = v[q][c];
+                        }
+                        ++pos;
+                    }
+                    if (++col == K) { col = 0; ++r; }
+                }
+            }
+        }
+        quad_base += quad_total[q];
+    }
+    if (tile == a.num_tiles - 1 && tid == 0) {
+        const int64_t total = tile_base + tile_count;
+        a.out_row_ptr[a.rows] = (int32_t)min(total, cap);
+        if (total > cap) {
+            dev_flag(a.hdr, CSRT_DEV_CAPACITY);
+            atomicMax(&a.hdr->required, (unsigned long long)total);
+        }
+    }
+}
+
+static int compact_launch(bool prox, const float *src, int32_t rows, int32_t cols, const csrt_csr *in,
+                          float eta, float thr, csrt_csr *out, void *ws, size_t ws_bytes,
+                          cudaStream_t s) {
+    const int64_t elems = (int64_t)rows * cols;
+    if (elems == 0) {
+        CSRT_CHECK_CUDA(cudaMemsetAsync(out->row_ptr, 0, sizeof(int32_t) * ((size_t)rows + 1), s));
+        return CSRT_OK;
+    }
+    const int64_t tiles = ceil_div<int64_t>(elems, kTile);
+    CSRT_ARG(ws_bytes >= kWsHeaderBytes + compact_scratch_bytes(elems), "workspace too small for compaction");
+    WsHeader *hdr = static_cast<WsHeader *>(ws);
+    unsigned long long *status = reinterpret_cast<unsigned long long *>(ws_scratch(ws));
+    CSRT_CHECK_CUDA(cudaMemsetAsync(&hdr->ticket, 0, sizeof(unsigned int), s));
+    CSRT_CHECK_CUDA(cudaMemsetAsync(status, 0, sizeof(unsigned long long) * tiles, s));
+    CompactArgs a;
+    a.src = src;
+    a.rows = rows;
+    a.cols = cols;
+    a.elems = elems;
+    a.in_row_ptr = in ? in->row_ptr : nullptr;
+    a.in_col = in ? in->col_idx : nullptr;
+    a.in_val = in ? in->val : nullptr;
+    a.eta = eta;
+    a.thr = thr;
+    a.out_row_ptr = out->row_ptr;
+    a.out_col = out->col_idx;
+    a.out_val = out->val;
+    a.capacity = out->capacity;
+    a.hdr = hdr;
+    a.status = status;
+    a.num_tiles = tiles;
+    const bool vec = (reinterpret_cast<uintptr_t>(src) & 15) == 0;
+    dim3 grid((unsigned)tiles), block(kCThreads);
+    if (prox) {
+        if (vec) compact_kernel<true, true><<<grid, block, 0, s>>>(a);
+        else compact_kernel<true, false><<<grid, block, 0, s>>>(a);
+    } else {
+        if (vec) compact_kernel<false, true><<<grid, block, 0, s>>>(a);
+        else compact_kernel<false, false><<<grid, block, 0, s>>>(a);
+    }
+    count_launch();
+    return check_launch("compact_kernel");
+}
+
+// ---------------------------------------------------------------------------
+// Transposed pattern (column-wise copy), deterministic.
+// ---------------------------------------------------------------------------
+constexpr int kTrRows = 32;      // rows per block: one bit each in a 32-bit word
+constexpr int kTrChunk = 8192;   // columns per block (32 KB of bitmask words)
+
+size_t transpose_scratch_bytes(int32_t rows, int32_t cols) {
+    const int64_t nb = ceil_div<int64_t>(rows, kTrRows);
+    return (size_t)(nb * cols + cols + 64) * sizeof(int32_t);
+}
+
+// Bitmask of the rows of block b present in each column of chunk [c0, c0+cw).
+__device__ __forceinline__ void tr_build_bits(unsigned int *bits, const int32_t *__restrict__ row_ptr,
+                                              const int32_t *__restrict__ col, int32_t rows, int b,
+                                              int c0, int cw, bool chunked) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int j = threadIdx.x; j < cw; j += blockDim.x) bits[j] = 0u;
+    __syncthreads();
+    for (int rr = warp; rr < kTrRows; rr += blockDim.x / 32) {
+        const int r = b * kTrRows + rr;
+        if (r >= rows) break;
+        int64_t s = row_ptr[r], e = row_ptr[r + 1];
+        if (chunked) {
+            s = warp_lower_bound(col, s, e, c0);
+            e = warp_lower_bound(col, s, e, c0 + cw);
+        }
+        for (int64_t k = s + lane; k < e; k += 32) atomicOr(&bits[__ldg(col + k) - c0], 1u << rr);
+    }
+    __syncthreads();
+}
+
+__global__ void __launch_bounds__(256) tr_count_kernel(const int32_t *__restrict__ row_ptr,
+                                                       const int32_t *__restrict__ col, int32_t rows,
+                                                       int32_t cols, int32_t *__restrict__ cnt) {
+    __shared__ unsigned int bits[kTrChunk];
+    const int b = blockIdx.x, c0 = blockIdx.y * kTrChunk;
+    const int cw = min(kTrChunk, cols - c0);
+    tr_build_bits(bits, row_ptr, col, rows, b, c0, cw, gridDim.y > 1);
+    int32_t *out = cnt + (int64_t)b * cols + c0;
+    for (int j = threadIdx.x; j < cw; j += blockDim.x) out[j] = __popc(bits[j]);
+}
+
+// Exclusive scan of cnt[b][j] over b for 32 columns per block; column totals.
+__global__ void __launch_bounds__(256) tr_colscan_kernel(int32_t *__restrict__ cnt, int32_t nb,
+                                                         int32_t cols, int32_t *__restrict__ coltot) {
+    __shared__ int32_t seg[8][32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int j = blockIdx.x * 32 + lane;
+    const int b0 = (int)(((int64_t)nb * warp) / 8), b1 = (int)(((int64_t)nb * (warp + 1)) / 8);
+    int32_t sum = 0;
+    if (j < cols)
+        for (int b = b0; b < b1; ++b) sum += cnt[(int64_t)b * cols + j];
+    seg[warp][lane] = sum;
+    __syncthreads();
+    int32_t run = 0;
+    for (int w = 0; w < warp; ++w) run += seg[w][lane];
+    if (j < cols) {
+        for (int b = b0; b < b1; ++b) {
+            int32_t *p = cnt + (int64_t)b * cols + j;
+            const int32_t v = *p;
+            *p = run;
+            run += v;
+        }
+        if (warp == 7) coltot[j] = run;
+    }
+}
+
+// Exclusive scan of n values into out[0..n] (out[n] = total); one block.
+__global__ void __launch_bounds__(1024) scan_single_block_kernel(const int32_t *__restrict__ in, int32_t n,
+                                                                 int32_t *__restrict__ out) {
+    __shared__ int32_t s_warp[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int per = (n + 1023) / 1024;
+    const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+    int32_t local = 0;
+    for (int i = i0; i < i1; ++i) local += in[i];
+    int32_t incl = local;
+    for (int off = 1; off < 32; off <<= 1) {
+        int32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    int32_t wp = 0, total = 0;
+    for (int w = 0; w < 32; ++w) {
+        if (w < warp) wp += s_warp[w];
+        total += s_warp[w];
+    }
+    int32_t run = incl - local + wp;
+    for (int i = i0; i < i1; ++i) {
+        out[i] = run;
+        run += in[i];
+    }
+    if (tid == 0) out[n] = total;
+}
+
+__global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict__ row_ptr,
+                                                       const int32_t *__restrict__ col,
+                                                       const float *__restrict__ val, int32_t rows,
+                                                       int32_t cols, const int32_t *__restrict__ off,
+                                                       const int32_t *__restrict__ t_row_ptr,
+                                                       int32_t *__restrict__ t_col, float *__restrict__ t_val,
+                                                       int32_t *__restrict__ t_pos, int64_t capacity) {
+    __shared__ unsigned int bits[kTrChunk];
+    const int b = blockIdx.x, c0 = blockIdx.y * kTrChunk;
+    const int cw = min(kTrChunk, cols - c0);
+    const bool chunked = gridDim.y > 1;
+    tr_build_bits(bits, row_ptr, col, rows, b, c0, cw, chunked);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int32_t *boff = off + (int64_t)b * cols;
+    for (int rr = warp; rr < kTrRows; rr += blockDim.x / 32) {
+        const int r = b * kTrRows + rr;
+        if (r >= rows) break;
+        int64_t s = row_ptr[r], e = row_ptr[r + 1];
+        if (chunked) {
+            s = warp_lower_bound(col, s, e, c0);
+            e = warp_lower_bound(col, s, e, c0 + cw);
+        }
+        const unsigned int below = (1u << rr) - 1u;
+        for (int64_t k = s + lane; k < e; k += 32) {
+            const int j = __ldg(col + k);
+            const int64_t p = (int64_t)t_row_ptr[j] + boff[j] + __popc(bits[j - c0] & below);
+            if (p < capacity) {
+                t_col[p] = r;
+                t_val[p] = __ldg(val + k);
+                t_pos[k] = (int32_t)p;
+            }
+        }
+    }
+}
+
+int transpose_impl(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s) {
+    CSRT_ARG(w->t_row_ptr && w->t_col_idx && w->t_val && w->t_pos, "transposed arrays not set");
+    const int32_t rows = w->rows, cols = w->cols;
+    if (cols == 0) return CSRT_OK;
+    if (rows == 0) {
+        CSRT_CHECK_CUDA(cudaMemsetAsync(w->t_row_ptr, 0, sizeof(int32_t) * ((size_t)cols + 1), s));
+        return CSRT_OK;
+    }
+    CSRT_ARG(ws_bytes >= kWsHeaderBytes + transpose_scratch_bytes(rows, cols), "workspace too small for transpose");
+    const int nb = (int)ceil_div<int64_t>(rows, kTrRows);
+    const int nc = (int)ceil_div<int64_t>(cols, kTrChunk);
+    int32_t *cnt = reinterpret_cast<int32_t *>(ws_scratch(ws));
+    int32_t *coltot = cnt + (int64_t)nb * cols;
+    tr_count_kernel<<<dim3(nb, nc), 256, 0, s>>>(w->row_ptr, w->col_idx, rows, cols, cnt);
+    tr_colscan_kernel<<<ceil_div(cols, 32), 256, 0, s>>>(cnt, nb, cols, coltot);
+    scan_single_block_kernel<<<1, 1024, 0, s>>>(coltot, cols, w->t_row_ptr);
+    tr_write_kernel<<<dim3(nb, nc), 256, 0, s>>>(w->row_ptr, w->col_idx, w->val, rows, cols, cnt,
+                                                 w->t_row_ptr, w->t_col_idx, w->t_val, w->t_pos,
+                                                 w->capacity);
+    count_launch(4);
+    return check_launch("csr_transpose kernels");
+}
+
+}  // namespace csrt
+
+using namespace csrt;
+
+static int check_csr(const csrt_csr *w, bool need_t) {
+    CSRT_ARG(w != nullptr, "csr is NULL");
+    CSRT_ARG(w->rows >= 0 && w->cols >= 0, "negative shape");
+    CSRT_ARG((int64_t)w->rows * w->cols < ((int64_t)1 << 31), "rows*cols must be below 2^31");
+    CSRT_ARG(w->row_ptr != nullptr, "row_ptr is NULL");
+    CSRT_ARG(w->capacity >= 0 && w->capacity < ((int64_t)1 << 31), "capacity out of range");
+    CSRT_ARG(w->capacity == 0 || (w->col_idx && w->val), "col_idx/val NULL");
+    if (need_t) CSRT_ARG(w->t_row_ptr && w->t_col_idx && w->t_val && w->t_pos, "transposed arrays not set");
+    return CSRT_OK;
+}
+
+extern "C" {
+
+int csr_from_dense(const float *dense, int32_t rows, int32_t cols, csrt_csr *out, void *ws, size_t ws_bytes,
+                   void *stream) {
+    int rc = check_csr(out, false);
+    if (rc) return rc;
+    CSRT_ARG(out->rows == rows && out->cols == cols, "out shape differs from rows/cols");
+    CSRT_ARG(dense != nullptr || (int64_t)rows * cols == 0, "dense is NULL");
+    CSRT_ARG(ws != nullptr, "workspace is NULL");
+    cudaStream_t s = as_stream(stream);
+    rc = compact_launch(false, dense, rows, cols, nullptr, 0.f, 0.f, out, ws, ws_bytes, s);
+    if (rc) return rc;
+    if (out->t_row_ptr) rc = transpose_impl(out, ws, ws_bytes, s);
+    return rc;
+}
+
+int csr_transpose(csrt_csr *w, void *ws, size_t ws_bytes, void *stream) {
+    int rc = check_csr(w, true);
+    if (rc) return rc;
+    CSRT_ARG(ws != nullptr, "workspace is NULL");
+    return transpose_impl(w, ws, ws_bytes, as_stream(stream));
+}
+
+int prox_update_compact(const csrt_csr *w_in, const float *g, float eta, float lambda, csrt_csr *w_out,
+                        void *ws, size_t ws_bytes, void *stream) {
+    int rc = check_csr(w_in, false);
+    if (rc) return rc;
+    rc = check_csr(w_out, false);
+    if (rc) return rc;
+    CSRT_ARG(w_in->rows == w_out->rows && w_in->cols == w_out->cols, "w_in and w_out shapes differ");
+    CSRT_ARG(w_in->row_ptr != w_out->row_ptr && w_in->col_idx != w_out->col_idx && w_in->val != w_out->val,
+             "w_out must not alias w_in");
+    CSRT_ARG(g != nullptr || (int64_t)w_in->rows * w_in->cols == 0, "G is NULL");
+    CSRT_ARG(eta >= 0.f && lambda >= 0.f && eta <= 3.0e38f && lambda <= 3.0e38f,
+             "eta and lambda must be finite and >= 0");
+    CSRT_ARG(ws != nullptr, "workspace is NULL");
+    const float thr = eta * lambda;  // fl32(eta*lambda), the threshold of Eq. prox
+    cudaStream_t s = as_stream(stream);
+    rc = compact_launch(true, g, w_in->rows, w_in->cols, w_in, eta, thr, w_out, ws, ws_bytes, s);
+    if (rc) return rc;
+    if (w_out->t_row_ptr) rc = transpose_impl(w_out, ws, ws_bytes, s);
+    return rc;
+}
+
+}  // extern "C"

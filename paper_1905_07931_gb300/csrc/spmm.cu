@@ -1,0 +1,482 @@
+// Sparse x dense products of the training step.
+//
+// spmm_fwd   Y = W X         Section 3.2.1 (dense x compressed', forward)
+// spmm_bwd_t dX = W^T dY     Section 3.2.2 (dense x compressed, backward),
+//                            run as the same kernel over the transposed arrays
+// weight_grad_sddmm          gradient at the stored entries (Section 2.4)
+// debias_update              SGD on the stored entries (Section 2.4, 4.3)
+//
+// Design (GB300): one warp per work unit. The rows and nonzeros of the CSR
+// are split evenly with a merge-path partition (row ends merged with nonzero
+// indices, Merrill & Garland), so a unit owns the same amount of work whether
+// rows are uniform or power-law. The n columns of the dense operand are cut
+// into tiles of 32*VW*NV floats; each lane holds NV vectors of VW floats, so
+// one nonzero costs every lane NV 16-byte loads of X and 4*NV FMAs, and a
+// warp moves 512*NV contiguous bytes per nonzero. Column indices and values
+// are loaded 32 at a time, coalesced, and broadcast with shuffles; four
+// nonzeros are in flight per lane. A row cut by a unit boundary leaves a
+// partial sum ("carry") in the workspace; a fix-up kernel adds the carries of
+// each cut row in unit order, so the result is deterministic and no float
+// atomics are used.
+#include "common.cuh"
+
+namespace csrt {
+
+constexpr int kSpThreads = 256;
+constexpr int kWarpsPerSM = 32;   // units requested per SM
+
+template <int VW> struct Vec;
+template <> struct Vec<1> { using T = float; };
+template <> struct Vec<2> { using T = float2; };
+template <> struct Vec<4> { using T = float4; };
+
+template <int VW>
+__device__ __forceinline__ typename Vec<VW>::T ldv(const float *p) {
+    return __ldg(reinterpret_cast<const typename Vec<VW>::T *>(p));
+}
+template <int VW>
+__device__ __forceinline__ void stv(float *p, const float (&a)[VW]) {
+    if constexpr (VW == 4) *reinterpret_cast<float4 *>(p) = make_float4(a[0], a[1], a[2], a[3]);
+    else if constexpr (VW == 2) *reinterpret_cast<float2 *>(p) = make_float2(a[0], a[1]);
+    else *p = a[0];
+}
+template <int VW>
+__device__ __forceinline__ void unpack(const typename Vec<VW>::T &v, float (&a)[VW]) {
+    if constexpr (VW == 4) { a[0] = v.x; a[1] = v.y; a[2] = v.z; a[3] = v.w; }
+    else if constexpr (VW == 2) { a[0] = v.x; a[1] = v.y; }
+    else a[0] = v;
+}
+
+// Number of row ends the merge path has consumed at diagonal d: the smallest
+// i in [lo, hi) with row_ptr[i+1] + i >= d, else hi (Merrill & Garland's
+// merge-path search with row ends as one list and nonzero indices as the
+// other).
+__device__ __forceinline__ int merge_rows_before(const int32_t *__restrict__ row_ptr, int64_t d, int64_t lo,
+                                                 int64_t hi) {
+    return (int)warp_first_false(lo, hi, [&](int64_t i) { return (int64_t)__ldg(row_ptr + i + 1) + i < d; });
+}
+
+struct SpmmArgs {
+    const int32_t *row_ptr;
+    const int32_t *col;
+    const float *val;
+    int32_t rows;
+    const float *x;
+    int32_t n;
+    float *y;
+    int32_t units;    // merge-path units per n-tile
+    int32_t n_tiles;
+    float *carry;     // [n_tiles][units][TN]
+    int32_t *carry_row;  // [units]
+};
+
+template <int VW, int NV>
+__device__ __forceinline__ void spmm_consume(const SpmmArgs &a, int64_t k, int64_t kend, int n0,
+                                             float (&acc)[NV][VW]) {
+    const int lane = threadIdx.x & 31;
+    constexpr int kStride = 32 * VW;
+    bool in_n[NV];
+#pragma unroll
+    for (int v = 0; v < NV; ++v) in_n[v] = n0 + v * kStride < a.n;
+    for (int64_t kb = k; kb < kend; kb += 32) {
+        const int cnt = (int)imin<int64_t>(32, kend - kb);
+        int my_c = 0;
+        float my_w = 0.f;
+        if (lane < cnt) {
+            my_c = __ldg(a.col + kb + lane);
+            my_w = __ldg(a.val + kb + lane);
+        }
+        int q = 0;
+        for (; q + 4 <= cnt; q += 4) {
+            int c[4];
+            float w[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                c[u] = __shfl_sync(0xffffffffu, my_c, q + u);
+                w[u] = __shfl_sync(0xffffffffu, my_w, q + u);
+            }
+            typename Vec<VW>::T xv[4][NV];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v = 0; v < NV; ++v)
+                    if (in_n[v]) xv[u][v] = ldv<VW>(a.x + (int64_t)c[u] * a.n + n0 + v * kStride);
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v = 0; v < NV; ++v)
+                    if (in_n[v]) {
+                        float f[VW];
+                        unpack<VW>(xv[u][v], f);
+#pragma unroll
+                        for (int e = 0; e < VW; ++e) acc[v][e] = fmaf(w[u], f[e], acc[v][e]);
+                    }
+        }
+        for (; q < cnt; ++q) {
+            const int c = __shfl_sync(0xffffffffu, my_c, q);
+            const float w = __shfl_sync(0xffffffffu, my_w, q);
+#pragma unroll
+            for (int v = 0; v < NV; ++v)
+                if (in_n[v]) {
+                    float f[VW];
+                    unpack<VW>(ldv<VW>(a.x + (int64_t)c * a.n + n0 + v * kStride), f);
+#pragma unroll
+                    for (int e = 0; e < VW; ++e) acc[v][e] = fmaf(w, f[e], acc[v][e]);
+                }
+        }
+    }
+}
+
+template <int VW, int NV>
+__global__ void __launch_bounds__(kSpThreads) spmm_merge_kernel(SpmmArgs a) {
+    constexpr int TN = 32 * VW * NV;
+    constexpr int kStride = 32 * VW;
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * kSpThreads + threadIdx.x) >> 5;
+    if (gw >= (int64_t)a.units * a.n_tiles) return;
+    const int u = (int)(gw % a.units);
+    const int t = (int)(gw / a.units);
+    const int64_t nnz = __ldg(a.row_ptr + a.rows);
+    const int64_t items = (int64_t)a.rows + nnz;
+    const int64_t per = ceil_div<int64_t>(items, a.units);
+    const int64_t d0 = min((int64_t)u * per, items), d1 = min(d0 + per, items);
+    const int i0 = merge_rows_before(a.row_ptr, d0, imax<int64_t>(0, d0 - nnz), imin<int64_t>(d0, a.rows));
+    const int i1 = merge_rows_before(a.row_ptr, d1, imax<int64_t>(0, d1 - nnz), imin<int64_t>(d1, a.rows));
+    const int64_t k0 = d0 - i0, k1 = d1 - i1;
+    const int n0 = t * TN + lane * VW;
+
+    float acc[NV][VW];
+#pragma unroll
+    for (int v = 0; v < NV; ++v)
+#pragma unroll
+        for (int e = 0; e < VW; ++e) acc[v][e] = 0.f;
+
+    int64_t k = k0;
+    for (int i = i0; i < i1; ++i) {
+        const int64_t kend = __ldg(a.row_ptr + i + 1);
+        spmm_consume<VW, NV>(a, k, kend, n0, acc);
+        k = kend;
+        float *yrow = a.y + (int64_t)i * a.n + n0;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            if (n0 + v * kStride < a.n) stv<VW>(yrow + v * kStride, acc[v]);
+#pragma unroll
+            for (int e = 0; e < VW; ++e) acc[v][e] = 0.f;
+        }
+    }
+    spmm_consume<VW, NV>(a, k, k1, n0, acc);
+    const bool has_carry = k1 > k;
+    if (a.units > 1) {
+        if (t == 0 && lane == 0) a.carry_row[u] = has_carry ? i1 : -1;
+        if (has_carry) {
+            float *cp = a.carry + ((int64_t)t * a.units + u) * TN + lane * VW;
+#pragma unroll
+            for (int v = 0; v < NV; ++v) stv<VW>(cp + v * kStride, acc[v]);
+        }
+    }
+}
+
+// Adds the carries of every cut row, in unit order, to that row of Y.
+template <int TN>
+__global__ void __launch_bounds__(256) spmm_fixup_kernel(SpmmArgs a) {
+    const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t per_tile = (int64_t)a.units * TN;
+    if (tid >= per_tile * a.n_tiles) return;
+    const int t = (int)(tid / per_tile);
+    const int u = (int)((tid % per_tile) / TN);
+    const int j = (int)(tid % TN);
+    const int r = a.carry_row[u];
+    if (r < 0 || (u > 0 && a.carry_row[u - 1] == r)) return;  // not the first carry of its row
+    const int col = t * TN + j;
+    if (col >= a.n) return;
+    float sum = 0.f;
+    for (int v = u; v < a.units && a.carry_row[v] == r; ++v)
+        sum += a.carry[((int64_t)t * a.units + v) * TN + j];
+    float *yp = a.y + (int64_t)r * a.n + col;
+    *yp = *yp + sum;
+}
+
+struct SpmmShape {
+    int vw, nv, tn, n_tiles, units;
+};
+
+static SpmmShape spmm_shape(int32_t n, int64_t max_items, bool vec4_ok, bool vec2_ok) {
+    SpmmShape s;
+    if (vec4_ok && n >= 128) { s.vw = 4; s.nv = n >= 256 ? 2 : 1; }
+    else if (vec2_ok && n >= 64) { s.vw = 2; s.nv = 1; }
+    else { s.vw = 1; s.nv = 1; }
+    s.tn = 32 * s.vw * s.nv;
+    s.n_tiles = (int)ceil_div<int64_t>(n, s.tn);
+    const int64_t target = (int64_t)num_sms() * kWarpsPerSM;
+    int64_t units = ceil_div<int64_t>(target, s.n_tiles);
+    units = imax<int64_t>(1, imin<int64_t>(units, max_items));
+    s.units = (int)units;
+    return s;
+}
+
+size_t spmm_scratch_bytes(int32_t max_n) {
+    // units * n_tiles <= target + n_tiles, TN <= 256: carries plus carry rows.
+    const int64_t target = (int64_t)num_sms() * kWarpsPerSM;
+    const int64_t floats = (target + 1) * 256 + (int64_t)max_n + 256;
+    return (size_t)floats * sizeof(float) + (size_t)(target + 1) * sizeof(int32_t) + 512;
+}
+
+static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *val, int32_t rows,
+                       int64_t capacity, const float *x, int32_t n, float *y, void *ws, size_t ws_bytes,
+                       cudaStream_t s) {
+    if (rows == 0 || n == 0) return CSRT_OK;
+    const bool v4 = (n % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15) == 0;
+    const bool v2 = (n % 2 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 7) == 0;
+    const SpmmShape sh = spmm_shape(n, (int64_t)rows + capacity, v4, v2);
+    SpmmArgs a;
+    a.row_ptr = row_ptr;
+    a.col = col;
+    a.val = val;
+    a.rows = rows;
+    a.x = x;
+    a.n = n;
+    a.y = y;
+    a.units = sh.units;
+    a.n_tiles = sh.n_tiles;
+    const size_t carry_floats = (size_t)sh.units * sh.n_tiles * sh.tn;
+    a.carry = reinterpret_cast<float *>(ws_scratch(ws));
+    a.carry_row = reinterpret_cast<int32_t *>(a.carry + ((carry_floats + 63) / 64) * 64);
+    if (sh.units > 1) {
+        const size_t need = kWsHeaderBytes + ((carry_floats + 63) / 64) * 64 * sizeof(float) +
+                            (size_t)sh.units * sizeof(int32_t);
+        CSRT_ARG(ws != nullptr && ws_bytes >= need, "workspace too small for spmm (%zu < %zu)", ws_bytes, need);
+    }
+    const int64_t threads = (int64_t)sh.units * sh.n_tiles * 32;
+    const unsigned grid = (unsigned)ceil_div<int64_t>(threads, kSpThreads);
+#define CSRT_SPMM_CASE(VW, NV)                                                               \
+    if (sh.vw == VW && sh.nv == NV) {                                                        \
+        spmm_merge_kernel<VW, NV><<<grid, kSpThreads, 0, s>>>(a);                            \
+        count_launch();                                                                      \
+        if (sh.units > 1) {                                                                  \
+            const int64_t ft = (int64_t)sh.units * sh.n_tiles * (32 * VW * NV);              \
+            spmm_fixup_kernel<32 * VW * NV><<<(unsigned)ceil_div<int64_t>(ft, 256), 256, 0, s>>>(a); \
+            count_launch();                                                                  \
+        }                                                                                    \
+    }
+    CSRT_SPMM_CASE(4, 2)
+    else CSRT_SPMM_CASE(4, 1)
+    else CSRT_SPMM_CASE(2, 1)
+    else CSRT_SPMM_CASE(1, 1)
+#undef CSRT_SPMM_CASE
+    return check_launch("spmm_merge_kernel");
+}
+
+// ---------------------------------------------------------------------------
+// SDDMM: g[k] = <dY[i_k, :], X[j_k, :]>
+// ---------------------------------------------------------------------------
+constexpr int kSdChunk = 2048;   // columns of the n range per partial sum
+
+struct SddmmArgs {
+    const int32_t *row_ptr;
+    const int32_t *col;
+    int32_t rows;
+    const float *dy;
+    const float *x;
+    int32_t n;
+    float *out;       // g (one chunk) or partial[chunk][capacity]
+    int64_t out_stride;
+    int32_t units;
+    int32_t chunks;
+    int32_t chunk_len;
+};
+
+// The row holding entry k: the largest i in [0, rows) with row_ptr[i] <= k.
+__device__ __forceinline__ int row_of_entry(const int32_t *__restrict__ row_ptr, int32_t rows, int64_t k) {
+    return (int)warp_first_false(1, rows, [&](int64_t i) { return (int64_t)__ldg(row_ptr + i) <= k; }) - 1;
+}
+
+template <int VW>
+__global__ void __launch_bounds__(kSpThreads) sddmm_kernel(SddmmArgs a) {
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * kSpThreads + threadIdx.x) >> 5;
+    if (gw >= (int64_t)a.units * a.chunks) return;
+    const int u = (int)(gw % a.units);
+    const int ch = (int)(gw / a.units);
+    const int64_t nnz = __ldg(a.row_ptr + a.rows);
+    const int64_t per = ceil_div<int64_t>(nnz, a.units);
+    const int64_t k0 = min((int64_t)u * per, nnz), k1 = min(k0 + per, nnz);
+    if (k0 >= k1) return;
+    const int nb = ch * a.chunk_len, ne = min(a.n, nb + a.chunk_len);
+    int row = row_of_entry(a.row_ptr, a.rows, k0);
+    int64_t next = __ldg(a.row_ptr + row + 1);
+    float *out = a.out + (int64_t)ch * a.out_stride;
+    for (int64_t kb = k0; kb < k1; kb += 32) {
+        const int cnt = (int)imin<int64_t>(32, k1 - kb);
+        const int my_c = lane < cnt ? __ldg(a.col + kb + lane) : 0;
+        for (int q = 0; q < cnt; q += 4) {
+            int c[4], r[4];
+            bool ok[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int64_t k = kb + q + e;
+                ok[e] = q + e < cnt;
+                c[e] = __shfl_sync(0xffffffffu, my_c, min(q + e, cnt - 1));
+                if (ok[e]) {
+                    while (next <= k) { ++row; next = __ldg(a.row_ptr + row + 1); }
+                }
+                r[e] = row;
+            }
+            float part[4] = {0.f, 0.f, 0.f, 0.f};
+            for (int nc = nb + lane * VW; nc < ne; nc += 32 * VW) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    if (!ok[e]) continue;
+                    float xf[VW], df[VW];
+                    unpack<VW>(ldv<VW>(a.x + (int64_t)c[e] * a.n + nc), xf);
+                    unpack<VW>(ldv<VW>(a.dy + (int64_t)r[e] * a.n + nc), df);
+#pragma unroll
+                    for (int j = 0; j < VW; ++j) part[e] = fmaf(df[j], xf[j], part[e]);
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) part[e] += __shfl_xor_sync(0xffffffffu, part[e], off);
+            }
+            if (lane < 4 && ok[lane]) {
+                float pv = lane == 0 ? part[0] : lane == 1 ? part[1] : lane == 2 ? part[2] : part[3];
+                out[kb + q + lane] = pv;
+            }
+        }
+    }
+}
+
+__global__ void sddmm_reduce_kernel(const int32_t *__restrict__ row_ptr, int32_t rows,
+                                    const float *__restrict__ partial, int64_t stride, int32_t chunks,
+                                    float *__restrict__ g) {
+    const int64_t nnz = __ldg(row_ptr + rows);
+    for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < nnz; k += (int64_t)gridDim.x * blockDim.x) {
+        float s = 0.f;
+        for (int c = 0; c < chunks; ++c) s += partial[(int64_t)c * stride + k];
+        g[k] = s;
+    }
+}
+
+static int sddmm_chunks(int64_t capacity, int32_t n) {
+    if (n <= kSdChunk) return 1;
+    const int64_t want = ceil_div<int64_t>(n, kSdChunk);
+    const int64_t room = imax<int64_t>(1, ((int64_t)1 << 22) / imax<int64_t>(1, capacity));
+    return (int)min(want, room);
+}
+
+size_t sddmm_scratch_bytes(int64_t capacity, int32_t max_n) {
+    const int chunks = sddmm_chunks(capacity, max_n);
+    if (chunks <= 1) return 0;
+    return (size_t)chunks * (size_t)capacity * sizeof(float) + 256;
+}
+
+}  // namespace csrt
+
+using namespace csrt;
+
+static int check_csr_basic(const csrt_csr *w) {
+    CSRT_ARG(w != nullptr && w->row_ptr != nullptr, "csr or row_ptr is NULL");
+    CSRT_ARG(w->rows >= 0 && w->cols >= 0, "negative shape");
+    CSRT_ARG((int64_t)w->rows * w->cols < ((int64_t)1 << 31), "rows*cols must be below 2^31");
+    CSRT_ARG(w->capacity >= 0 && w->capacity < ((int64_t)1 << 31), "capacity out of range");
+    CSRT_ARG(w->capacity == 0 || (w->col_idx && w->val), "col_idx/val NULL");
+    return CSRT_OK;
+}
+
+extern "C" {
+
+int spmm_fwd(const csrt_csr *w, const float *x, int32_t n, float *y, void *ws, size_t ws_bytes, void *stream) {
+    int rc = check_csr_basic(w);
+    if (rc) return rc;
+    CSRT_ARG(n >= 0, "n < 0");
+    CSRT_ARG((x && y) || n == 0 || w->rows == 0, "X or Y is NULL");
+    return spmm_launch(w->row_ptr, w->col_idx, w->val, w->rows, w->capacity, x, n, y, ws, ws_bytes,
+                       as_stream(stream));
+}
+
+int spmm_bwd_t(const csrt_csr *w, const float *dy, int32_t n, float *dx, void *ws, size_t ws_bytes,
+               void *stream) {
+    int rc = check_csr_basic(w);
+    if (rc) return rc;
+    CSRT_ARG(w->t_row_ptr && w->t_col_idx && w->t_val, "transposed arrays not set");
+    CSRT_ARG(n >= 0, "n < 0");
+    CSRT_ARG((dy && dx) || n == 0 || w->cols == 0, "dY or dX is NULL");
+    return spmm_launch(w->t_row_ptr, w->t_col_idx, w->t_val, w->cols, w->capacity, dy, n, dx, ws, ws_bytes,
+                       as_stream(stream));
+}
+
+int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_t n, float *g_nnz, void *ws,
+                      size_t ws_bytes, void *stream) {
+    int rc = check_csr_basic(w);
+    if (rc) return rc;
+    CSRT_ARG(n >= 0, "n < 0");
+    if (w->rows == 0 || w->capacity == 0) return CSRT_OK;
+    CSRT_ARG(g_nnz != nullptr, "g_nnz is NULL");
+    cudaStream_t s = as_stream(stream);
+    if (n == 0) {
+        CSRT_CHECK_CUDA(cudaMemsetAsync(g_nnz, 0, sizeof(float) * (size_t)w->capacity, s));
+        return CSRT_OK;
+    }
+    CSRT_ARG(dy && x, "dY or X is NULL");
+    const bool v4 = (n % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(dy)) & 15) == 0;
+    const int chunks = sddmm_chunks(w->capacity, n);
+    SddmmArgs a;
+    a.row_ptr = w->row_ptr;
+    a.col = w->col_idx;
+    a.rows = w->rows;
+    a.dy = dy;
+    a.x = x;
+    a.n = n;
+    a.chunks = chunks;
+    a.chunk_len = chunks > 1 ? (int)ceil_div<int64_t>(n, chunks) : n;
+    if (v4 && chunks > 1) a.chunk_len = (a.chunk_len + 3) / 4 * 4;
+    const int64_t target = (int64_t)num_sms() * kWarpsPerSM;
+    a.units = (int)imax<int64_t>(1, imin<int64_t>(ceil_div<int64_t>(target, chunks), w->capacity));
+    if (chunks > 1) {
+        CSRT_ARG(ws != nullptr && ws_bytes >= kWsHeaderBytes + sddmm_scratch_bytes(w->capacity, n),
+                 "workspace too small for sddmm");
+        a.out = reinterpret_cast<float *>(ws_scratch(ws));
+        a.out_stride = w->capacity;
+    } else {
+        a.out = g_nnz;
+        a.out_stride = 0;
+    }
+    const unsigned grid = (unsigned)ceil_div<int64_t>((int64_t)a.units * chunks * 32, kSpThreads);
+    if (v4) sddmm_kernel<4><<<grid, kSpThreads, 0, s>>>(a);
+    else sddmm_kernel<1><<<grid, kSpThreads, 0, s>>>(a);
+    count_launch();
+    if (chunks > 1) {
+        const unsigned rg = (unsigned)imin<int64_t>(ceil_div<int64_t>(w->capacity, 256), (int64_t)num_sms() * 8);
+        sddmm_reduce_kernel<<<rg, 256, 0, s>>>(w->row_ptr, w->rows, a.out, a.out_stride, chunks, g_nnz);
+        count_launch();
+    }
+    return check_launch("sddmm_kernel");
+}
+
+}  // extern "C"
+
+namespace csrt {
+__global__ void debias_kernel(const int32_t *__restrict__ row_ptr, int32_t rows, float *__restrict__ val,
+                              const float *__restrict__ g, float eta, float *__restrict__ t_val,
+                              const int32_t *__restrict__ t_pos) {
+    const int64_t nnz = __ldg(row_ptr + rows);
+    for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < nnz; k += (int64_t)gridDim.x * blockDim.x) {
+        const float nv = __fsub_rn(val[k], __fmul_rn(eta, __ldg(g + k)));
+        val[k] = nv;
+        if (t_val) t_val[__ldg(t_pos + k)] = nv;
+    }
+}
+}  // namespace csrt
+
+extern "C" int debias_update(csrt_csr *w, const float *g_nnz, float eta, void *stream) {
+    int rc = check_csr_basic(w);
+    if (rc) return rc;
+    CSRT_ARG(!(eta < 0.f) && eta <= 3.0e38f, "eta must be finite and >= 0");
+    if (w->rows == 0 || w->capacity == 0) return CSRT_OK;
+    CSRT_ARG(g_nnz != nullptr, "g_nnz is NULL");
+    CSRT_ARG(w->t_val == nullptr || w->t_pos != nullptr, "t_val set without t_pos");
+    const unsigned grid = (unsigned)imax<int64_t>(1, imin<int64_t>(ceil_div<int64_t>(w->capacity, 256), (int64_t)num_sms() * 8));
+    debias_kernel<<<grid, 256, 0, as_stream(stream)>>>(w->row_ptr, w->rows, w->val, g_nnz, eta, w->t_val, w->t_pos);
+    count_launch();
+    return check_launch("debias_kernel");
+}

@@ -1,0 +1,254 @@
+"""The CSR-weight training step over a network of sparse layers.
+
+A network is a list of layers, each a dict with ``kind`` in
+{"fc", "conv", "pool2", "flatten"} (fc: {"relu"}, conv: {"k", "in_shape",
+"relu"}). Weights of fc and conv layers are CSR matrices (Section 3.1);
+convolutions are lowered to a matrix product with im2col. One step
+(Section 2.3 with a minibatch gradient):
+
+  forward   per layer: [im2col] -> spmm_fwd -> bias (+ ReLU) -> [pool/flatten]
+  loss      softmax cross-entropy; dL/dlogits = (softmax - onehot) / B
+  backward  per layer, last to first: [ReLU backward] -> weight gradient
+            (prox phase: dense G = dY X^T; debias phase: SDDMM at the stored
+            entries) -> bias SGD -> spmm_bwd_t (not for the first layer)
+            [-> col2im] -> weight update right away, while G is hot in L2:
+            prox phase: prox_update_compact into the other CSR buffer
+            (Eq. prox, compaction after every update, Section 4.4);
+            debias phase: debias_update in place (Section 2.4).
+
+Every buffer is allocated up front, every call is enqueued on one stream and
+nothing synchronises, so a step can be captured in a CUDA graph. This module
+only sequences calls into the CUDA library.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import csrtrain as C
+
+
+class SparseNet:
+    def __init__(self, layers, dense_weights, biases, batch: int, in_shape, *, device="cuda",
+                 precision: int = C.CSRT_PREC_TF32, stream=None, grad_per_layer: bool = False):
+        """layers: layer dicts; dense_weights/biases: numpy arrays, one per fc/conv
+        layer (weights M x K, zero off the initial pattern); in_shape: (K,) for an
+        fc-first net or (C, H, W) for a conv-first net. The dense gradients of
+        all layers share one buffer unless grad_per_layer is set (then each
+        layer's G stays readable after the step)."""
+        self.grad_per_layer = grad_per_layer
+        self.layers = [dict(l) for l in layers]
+        self.batch = int(batch)
+        self.device = device
+        self.precision = precision
+        self.stream = stream
+        B = self.batch
+        dev = dict(device=device, dtype=torch.float32)
+        if len(in_shape) == 1:
+            self.x_in = torch.zeros(in_shape[0], B, **dev)
+        else:
+            c, h, w = in_shape
+            self.x_in = torch.zeros(c, B * h * w, **dev)
+        self.labels = torch.zeros(B, dtype=torch.int32, device=device)
+        shape = tuple(in_shape)           # (K,) or (C, H, W) per sample
+        cur = self.x_in
+        wi = 0
+        max_rows = max_cols = max_n = 1
+        max_mk = 1
+        first_param = True
+        self.params = []
+        for L in self.layers:
+            kind = L["kind"]
+            L["x"] = cur
+            if kind in ("fc", "conv"):
+                W0 = np.ascontiguousarray(dense_weights[wi], dtype=np.float32)
+                M, K = W0.shape
+                L["needs_dx"] = not first_param
+                first_param = False
+                L["W"] = [C.CSR(M, K, transposed=L["needs_dx"], device=device),
+                          C.CSR(M, K, transposed=L["needs_dx"], device=device)]
+                L["cur"] = 0
+                L["b"] = torch.tensor(np.asarray(biases[wi], dtype=np.float32), device=device)
+                L["W0"] = torch.from_numpy(W0).to(device)
+                if kind == "fc":
+                    if shape != (K,):
+                        raise ValueError(f"fc layer expects {K} inputs, got {shape}")
+                    n = B
+                    L["xmat"] = cur
+                    shape = (M,)
+                else:
+                    ci, h, w = L["in_shape"]
+                    k = L["k"]
+                    if shape != (ci, h, w) or K != ci * k * k:
+                        raise ValueError(f"conv layer shape mismatch: {shape} vs {(ci, h, w)}")
+                    ho, wo = h - k + 1, w - k + 1
+                    n = B * ho * wo
+                    L["cols"] = torch.zeros(K, n, **dev)
+                    L["xmat"] = L["cols"]
+                    if L["needs_dx"]:
+                        L["dcols"] = torch.zeros(K, n, **dev)
+                    shape = (M, ho, wo)
+                L["y"] = torch.zeros(M, n, **dev)
+                L["dy"] = torch.zeros(M, n, **dev)
+                if L["needs_dx"]:
+                    L["dx"] = torch.zeros_like(cur)
+                L["g"] = torch.zeros(M * K, **dev)
+                if grad_per_layer:
+                    L["G"] = torch.zeros(M, K, **dev)
+                max_rows, max_cols, max_n = max(max_rows, M, K), max(max_cols, K, M), max(max_n, n)
+                max_mk = max(max_mk, M * K)
+                cur = L["y"]
+                self.params.append(L)
+                wi += 1
+            elif kind == "pool2":
+                c, h, w = shape
+                L["shape"] = shape
+                L["y"] = torch.zeros(c, B * (h // 2) * (w // 2), **dev)
+                L["idx"] = torch.zeros(c * B * (h // 2) * (w // 2), dtype=torch.int8, device=device)
+                L["dy"] = torch.zeros_like(L["y"])
+                L["dx"] = torch.zeros_like(cur)
+                shape = (c, h // 2, w // 2)
+                cur = L["y"]
+            elif kind == "flatten":
+                c, h, w = shape
+                L["shape"] = shape
+                L["y"] = torch.zeros(c * h * w, B, **dev)
+                L["dy"] = torch.zeros_like(L["y"])
+                L["dx"] = torch.zeros_like(cur)
+                shape = (c * h * w,)
+                cur = L["y"]
+            else:
+                raise ValueError(kind)
+        self.logits = cur
+        self.classes = shape[0]
+        self.dlogits = torch.zeros_like(cur)
+        self.loss = torch.zeros(B + 1, **dev)
+        self.G = torch.zeros(max_mk, **dev)
+        self.ws = C.Workspace(max(max_rows, max_cols), max(max_rows, max_cols), max_n, device=device, stream=stream)
+        for L in self.params:
+            C.csr_from_dense(L["W0"], L["W"][0], self.ws, stream)
+
+    # ------------------------------------------------------------------
+    def weights(self, li: int) -> C.CSR:
+        L = self.params[li]
+        return L["W"][L["cur"]]
+
+    def forward(self):
+        s = self.stream
+        for L in self.layers:
+            kind = L["kind"]
+            if kind == "fc":
+                W = L["W"][L["cur"]]
+                C.spmm_fwd(W, L["x"], L["y"], self.ws, s)
+                C.bias_act_fwd(L["y"], L["b"], L["relu"], s)
+            elif kind == "conv":
+                ci, h, w = L["in_shape"]
+                C.im2col(L["x"], ci, self.batch, h, w, L["k"], L["cols"], s)
+                W = L["W"][L["cur"]]
+                C.spmm_fwd(W, L["cols"], L["y"], self.ws, s)
+                C.bias_act_fwd(L["y"], L["b"], L["relu"], s)
+            elif kind == "pool2":
+                c, h, w = L["shape"]
+                C.maxpool2_fwd(L["x"], c, self.batch, h, w, L["y"], L["idx"], s)
+            elif kind == "flatten":
+                c, h, w = L["shape"]
+                C.flatten(L["x"], c, self.batch, h * w, L["y"], s)
+        return self.logits
+
+    def step(self, phase: str, eta: float, lam: float):
+        """One training step on the data in ``x_in`` / ``labels``. Returns the
+        device tensor whose element 0 is the mean loss (not synchronised)."""
+        s = self.stream
+        self.forward()
+        C.softmax_xent(self.logits, self.labels, self.dlogits, self.loss, s)
+        d = self.dlogits
+        for L in reversed(self.layers):
+            kind = L["kind"]
+            if kind in ("fc", "conv"):
+                W = L["W"][L["cur"]]
+                dpre = d
+                if L["relu"]:
+                    C.relu_bwd(dpre, L["y"], s)
+                M, K = W.rows, W.cols
+                if phase == "prox":
+                    G = L["G"] if self.grad_per_layer else self.G[: M * K].view(M, K)
+                    C.weight_grad_dense(dpre, L["xmat"], G, self.ws, self.precision, s)
+                else:
+                    C.weight_grad_sddmm(W, dpre, L["xmat"], L["g"], self.ws, s)
+                C.bias_grad_sgd(dpre, L["b"], eta, None, s)
+                if L["needs_dx"]:
+                    if kind == "fc":
+                        C.spmm_bwd_t(W, dpre, L["dx"], self.ws, s)
+                    else:
+                        ci, h, w = L["in_shape"]
+                        C.spmm_bwd_t(W, dpre, L["dcols"], self.ws, s)
+                        C.col2im(L["dcols"], ci, self.batch, h, w, L["k"], L["dx"], s)
+                if phase == "prox":
+                    Wn = L["W"][1 - L["cur"]]
+                    C.prox_update_compact(W, G, eta, lam, Wn, self.ws, s)
+                    L["cur"] = 1 - L["cur"]
+                else:
+                    C.debias_update(W, L["g"], eta, s)
+                if not L["needs_dx"]:
+                    break
+                d = L["dx"]
+            elif kind == "pool2":
+                c, h, w = L["shape"]
+                C.maxpool2_bwd(d, L["idx"], c, self.batch, h, w, L["dx"], s)
+                d = L["dx"]
+            elif kind == "flatten":
+                c, h, w = L["shape"]
+                C.unflatten(d, c, self.batch, h * w, L["dx"], s)
+                d = L["dx"]
+        return self.loss
+
+    def reset_weights(self):
+        """Rebuild every layer's CSR (buffer 0) from its initial dense weights."""
+        for L in self.params:
+            L["cur"] = 0
+            C.csr_from_dense(L["W0"], L["W"][0], self.ws, self.stream)
+
+
+def mlp_layers(n_layers: int):
+    return [{"kind": "fc", "relu": i < n_layers - 1} for i in range(n_layers)]
+
+
+def lenet_layers():
+    return [{"kind": "conv", "k": 5, "in_shape": (1, 28, 28), "relu": False},
+            {"kind": "pool2"},
+            {"kind": "conv", "k": 5, "in_shape": (20, 12, 12), "relu": False},
+            {"kind": "pool2"},
+            {"kind": "flatten"},
+            {"kind": "fc", "relu": True},
+            {"kind": "fc", "relu": False}]
+
+
+class SingleLayer:
+    """The single-layer step (one CSR layer, upstream gradient given):
+    forward SpMM, backward SpMM^T, dense weight gradient, prox + compaction."""
+
+    def __init__(self, w_dense: np.ndarray, n: int, device="cuda", precision: int = C.CSRT_PREC_TF32,
+                 stream=None):
+        M, K = w_dense.shape
+        self.stream = stream
+        self.precision = precision
+        self.W = [C.CSR(M, K, device=device), C.CSR(M, K, device=device)]
+        self.cur = 0
+        self.W0 = torch.from_numpy(np.ascontiguousarray(w_dense, dtype=np.float32)).to(device)
+        self.x = torch.zeros(K, n, device=device)
+        self.dy = torch.zeros(M, n, device=device)
+        self.y = torch.zeros(M, n, device=device)
+        self.dx = torch.zeros(K, n, device=device)
+        self.G = torch.zeros(M, K, device=device)
+        self.ws = C.Workspace(max(M, K), max(M, K), n, device=device, stream=stream)
+        C.csr_from_dense(self.W0, self.W[0], self.ws, stream)
+
+    def step(self, eta: float, lam: float):
+        s = self.stream
+        W = self.W[self.cur]
+        C.spmm_fwd(W, self.x, self.y, self.ws, s)
+        C.spmm_bwd_t(W, self.dy, self.dx, self.ws, s)
+        C.weight_grad_dense(self.dy, self.x, self.G, self.ws, self.precision, s)
+        C.prox_update_compact(W, self.G, eta, lam, self.W[1 - self.cur], self.ws, s)
+        self.cur = 1 - self.cur

@@ -1,0 +1,390 @@
+"""Parity of every C-ABI call against the CPU oracle, on seeded inputs.
+
+Sizes span several compaction tiles (4096 entries) and SpMM units with a
+ragged tail, empty rows, power-law rows, odd column counts and the degenerate
+cases (empty matrix, all-zero, fully dense, n = 1). Integer arrays are
+compared bit for bit; the prox step is bit-exact when fed the same G.
+"""
+
+import json
+import os
+
+import numpy as np
+import pytest
+
+import oracle as O
+from tests.parity import assert_close, csr_dense
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+F32 = np.float32
+
+
+@pytest.fixture(scope="module")
+def C():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_1905_07931_gb300 import csrtrain
+    csrtrain.lib()
+    return csrtrain
+
+
+def _ws(C, rows, cols, n):
+    return C.Workspace(max(rows, cols, 1), max(rows, cols, 1), max(n, 1))
+
+
+def _sparse(rng, m, k, density, zipf=False):
+    from paper_1905_07931_gb300 import synth
+    return synth.masked_weights(rng, m, k, density, std=1.0, zipf=zipf)
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _gpu_csr(C, dense, ws, transposed=True, capacity=None):
+    m, k = dense.shape
+    w = C.CSR(m, k, capacity=capacity, transposed=transposed)
+    C.csr_from_dense(_dev(dense.astype(F32)), w, ws)
+    return w
+
+
+def _check_csr_equal(w, ref: "O.CSR", transposed=True):
+    (rp, ci, v), t = w.to_host()
+    np.testing.assert_array_equal(rp, ref.row_ptr)
+    np.testing.assert_array_equal(ci, ref.col_idx)
+    np.testing.assert_array_equal(v.view(np.uint32), ref.val.astype(F32).view(np.uint32))
+    if transposed:
+        trp, tci, tv, tpos = O.csr_transpose(ref)
+        np.testing.assert_array_equal(t[0], trp)
+        np.testing.assert_array_equal(t[1], tci)
+        np.testing.assert_array_equal(t[2].view(np.uint32), tv.astype(F32).view(np.uint32))
+        np.testing.assert_array_equal(t[3], tpos)
+
+
+# --- csr_from_dense / csr_transpose -----------------------------------------
+
+def test_worked_example_on_gpu(C):
+    with open(os.path.join(GOLD, "csr_worked_example.json")) as f:
+        d = json.load(f)
+    a = np.array(d["dense"], dtype=F32)
+    ws = _ws(C, 4, 4, 1)
+    w = _gpu_csr(C, a, ws)
+    (rp, ci, v), t = w.to_host()
+    assert rp.tolist() == d["row_ptrs"]
+    assert ci.tolist() == d["col_indices"]
+    assert v.tolist() == d["elements"]
+    h = d["hand_derived"]
+    assert t[0].tolist() == h["transpose_row_ptrs"]
+    assert t[1].tolist() == h["transpose_col_indices"]
+    assert t[2].tolist() == h["transpose_elements"]
+    assert t[3].tolist() == h["transpose_pos_of_each_csr_entry"]
+    y = torch.zeros(4, 1, device="cuda")
+    C.spmm_fwd(w, torch.ones(4, 1, device="cuda"), y, ws)
+    assert y[:, 0].cpu().tolist() == h["A_times_ones"]
+    C.spmm_bwd_t(w, torch.ones(4, 1, device="cuda"), y, ws)
+    assert y[:, 0].cpu().tolist() == h["At_times_ones"]
+
+
+@pytest.mark.parametrize("m,k,density", [(1, 1, 1.0), (3, 5, 0.5), (33, 129, 0.3), (300, 784, 0.1),
+                                         (17, 1, 0.5), (5, 3, 1.0), (41, 9216, 0.05), (64, 64, 0.0),
+                                         (2, 70000, 0.01), (257, 31, 0.9)])
+def test_csr_from_dense_bit_exact(C, m, k, density):
+    rng = np.random.default_rng(m * 7 + k)
+    a = _sparse(rng, m, k, density)
+    if m > 2:
+        a[1, :] = 0.0
+        a[m - 1, :] = 0.0
+    ws = _ws(C, m, k, 1)
+    w = _gpu_csr(C, a, ws)
+    _check_csr_equal(w, O.csr_from_dense(a))
+    assert ws.status()[0] == 0
+
+
+def test_csr_from_dense_signed_zero_nan_inf(C):
+    a = np.array([[-0.0, 1.0, np.nan, 0.0, np.inf, -np.inf, -2.0]], dtype=F32)
+    ws = _ws(C, 1, 7, 1)
+    w = _gpu_csr(C, a, ws, transposed=False)
+    (rp, ci, v), _ = w.to_host()
+    assert ci.tolist() == [1, 2, 4, 5, 6]
+    assert rp.tolist() == [0, 5]
+
+
+def test_csr_capacity_overflow_is_reported_and_clamped(C):
+    rng = np.random.default_rng(3)
+    a = _sparse(rng, 40, 300, 0.5)
+    nnz = int((a != 0).sum())
+    ws = _ws(C, 40, 300, 1)
+    w = _gpu_csr(C, a, ws, transposed=False, capacity=nnz // 2)
+    flags, required = ws.status()
+    assert flags & C.CSRT_DEV_CAPACITY
+    assert required == nnz
+    rp = w.row_ptr.cpu().numpy()
+    assert (np.diff(rp) >= 0).all() and rp[-1] == nnz // 2
+    ref = O.csr_from_dense(a)
+    np.testing.assert_array_equal(w.col_idx.cpu().numpy()[: nnz // 2], ref.col_idx[: nnz // 2])
+    ws.clear_status()
+    assert ws.status()[0] == 0
+
+
+def test_empty_matrix_shapes(C):
+    ws = _ws(C, 8, 8, 4)
+    w = C.CSR(0, 5, transposed=True)
+    C.csr_from_dense(torch.zeros(1, device="cuda"), w, ws)
+    assert w.row_ptr.cpu().tolist() == [0]
+    assert w.t_row_ptr.cpu().tolist() == [0] * 6
+    w2 = C.CSR(4, 0, transposed=False)
+    C.csr_from_dense(torch.zeros(1, device="cuda"), w2, ws)
+    assert w2.row_ptr.cpu().tolist() == [0] * 5
+
+
+# --- spmm_fwd / spmm_bwd_t ----------------------------------------------------
+
+SPMM_CASES = [
+    (300, 784, 64, 0.1, False),
+    (37, 53, 1, 0.3, False),
+    (37, 53, 3, 0.3, False),
+    (129, 257, 32, 0.2, False),
+    (129, 257, 70, 0.2, False),
+    (500, 300, 256, 0.05, True),
+    (64, 2000, 130, 0.5, True),
+    (20, 25, 4100, 0.3, False),
+    (4, 9, 1, 1.0, False),
+    (50, 40, 7, 0.0, False),
+    (1000, 600, 1024, 0.02, True),
+]
+
+
+@pytest.mark.parametrize("m,k,n,density,zipf", SPMM_CASES)
+def test_spmm_fwd_and_bwd_against_oracle(C, m, k, n, density, zipf):
+    rng = np.random.default_rng(m + 3 * k + 7 * n)
+    a = _sparse(rng, m, k, density, zipf)
+    if m > 4:
+        a[2, :] = 0.0
+    x = rng.standard_normal((k, n)).astype(F32)
+    dy = rng.standard_normal((m, n)).astype(F32)
+    ws = _ws(C, m, k, n)
+    w = _gpu_csr(C, a, ws)
+    ref = O.csr_from_dense(a)
+    y = torch.zeros(m, n, device="cuda")
+    C.spmm_fwd(w, _dev(x), y, ws)
+    lens = np.diff(ref.row_ptr)[:, None]
+    assert_close(y.cpu().numpy(), O.spmm_fwd(ref, x), O.spmm_fwd(O.csr_abs(ref), np.abs(x)), lens,
+                 what="spmm_fwd")
+    dx = torch.zeros(k, n, device="cuda")
+    C.spmm_bwd_t(w, _dev(dy), dx, ws)
+    clens = np.bincount(ref.col_idx, minlength=k)[:, None]
+    assert_close(dx.cpu().numpy(), O.spmm_bwd_t(ref, dy), O.spmm_bwd_t(O.csr_abs(ref), np.abs(dy)), clens,
+                 what="spmm_bwd_t")
+    assert ws.status()[0] == 0
+
+
+def test_spmm_is_deterministic(C):
+    rng = np.random.default_rng(11)
+    a = _sparse(rng, 700, 900, 0.08, zipf=True)
+    x = _dev(rng.standard_normal((900, 96)).astype(F32))
+    ws = _ws(C, 900, 900, 96)
+    w = _gpu_csr(C, a, ws)
+    ys = []
+    for _ in range(3):
+        y = torch.zeros(700, 96, device="cuda")
+        C.spmm_fwd(w, x, y, ws)
+        ys.append(y.cpu().numpy())
+    np.testing.assert_array_equal(ys[0].view(np.uint32), ys[1].view(np.uint32))
+    np.testing.assert_array_equal(ys[0].view(np.uint32), ys[2].view(np.uint32))
+
+
+# --- weight gradients ----------------------------------------------------------
+
+@pytest.mark.parametrize("m,k,n", [(300, 784, 64), (10, 500, 128), (20, 25, 9000), (129, 67, 33),
+                                   (1, 1, 1), (256, 512, 256)])
+@pytest.mark.parametrize("prec", [0, 1])
+def test_weight_grad_dense(C, m, k, n, prec):
+    rng = np.random.default_rng(m + k + n + prec)
+    dy = rng.standard_normal((m, n)).astype(F32)
+    x = rng.standard_normal((k, n)).astype(F32)
+    ws = _ws(C, m, k, n)
+    g = torch.zeros(m, k, device="cuda")
+    C.weight_grad_dense(_dev(dy), _dev(x), g, ws, precision=prec)
+    ref = O.weight_grad_dense(dy, x)
+    bound = O.weight_grad_dense(np.abs(dy), np.abs(x))
+    assert_close(g.cpu().numpy(), ref, bound, n, rtol=1e-3 if prec else 1e-4, tf32=bool(prec),
+                 what=f"weight_grad_dense prec={prec}")
+
+
+@pytest.mark.parametrize("m,k,n,density,zipf", [(300, 784, 64, 0.1, False), (100, 300, 256, 0.09, True),
+                                                (20, 25, 9000, 0.3, False), (50, 40, 1, 0.5, False),
+                                                (33, 17, 5, 0.0, False)])
+def test_weight_grad_sddmm(C, m, k, n, density, zipf):
+    rng = np.random.default_rng(m * k + n)
+    a = _sparse(rng, m, k, density, zipf)
+    dy = rng.standard_normal((m, n)).astype(F32)
+    x = rng.standard_normal((k, n)).astype(F32)
+    ws = _ws(C, m, k, n)
+    w = _gpu_csr(C, a, ws, transposed=False)
+    ref = O.csr_from_dense(a)
+    g = torch.zeros(max(ref.nnz, 1), device="cuda")
+    C.weight_grad_sddmm(w, _dev(dy), _dev(x), g, ws)
+    got = g.cpu().numpy()[: ref.nnz]
+    assert_close(got, O.weight_grad_sddmm(ref, dy, x), O.weight_grad_sddmm(ref, np.abs(dy), np.abs(x)), n,
+                 what="sddmm")
+    # the same values as the dense gradient read at the pattern
+    dense = O.weight_grad_dense(dy, x)
+    assert_close(got, dense[ref.row_of_each_entry(), ref.col_idx],
+                 O.weight_grad_dense(np.abs(dy), np.abs(x))[ref.row_of_each_entry(), ref.col_idx], n,
+                 what="sddmm vs masked dense")
+
+
+# --- prox_update_compact / debias_update ---------------------------------------
+
+def test_prox_hand_cases_on_gpu(C):
+    with open(os.path.join(GOLD, "soft_threshold_cases.json")) as f:
+        d = json.load(f)
+    ws_ = np.array([[c["w"] for c in d["cases"]]], dtype=F32)
+    gs = np.array([[c["g"] for c in d["cases"]]], dtype=F32)
+    ws = _ws(C, 1, ws_.shape[1], 1)
+    w = _gpu_csr(C, ws_, ws)
+    out = C.CSR(1, ws_.shape[1])
+    C.prox_update_compact(w, _dev(gs), d["eta"], d["lambda"], out, ws)
+    (rp, ci, v), _ = out.to_host()
+    dense = csr_dense(rp, ci, v, 1, ws_.shape[1])[0]
+    for j, c in enumerate(d["cases"]):
+        assert (dense[j] != 0) == c["kept"], c
+        assert dense[j] == F32(c["out"]), c
+
+
+@pytest.mark.parametrize("m,k,density,gscale,eta,lam", [
+    (300, 784, 0.1, 1.0, 0.01, 1e-4),
+    (300, 784, 0.1, 1e-3, 0.5, 1e-2),
+    (37, 4099, 0.3, 0.1, 0.1, 0.3),
+    (1, 5000, 0.5, 1.0, 0.01, 50.0),
+    (4097, 3, 0.6, 1.0, 0.2, 0.5),
+    (100, 300, 0.09, 1.0, 0.0, 1e-4),
+    (64, 64, 0.0, 0.0, 0.1, 0.0),
+    (500, 800, 0.08, 1e-2, 0.01, 1e-2),
+])
+def test_prox_bit_exact(C, m, k, density, gscale, eta, lam):
+    rng = np.random.default_rng(m + k)
+    a = _sparse(rng, m, k, density)
+    g = (rng.standard_normal((m, k)) * gscale).astype(F32)
+    ws = _ws(C, m, k, 1)
+    w = _gpu_csr(C, a, ws)
+    out = C.CSR(m, k)
+    C.prox_update_compact(w, _dev(g), eta, lam, out, ws)
+    ref = O.prox_update_compact(O.csr_from_dense(a), g, eta, lam)
+    _check_csr_equal(out, ref)
+    assert ws.status()[0] == 0
+
+
+def test_prox_chain_of_steps_bit_exact(C):
+    # several prox steps in a row (double-buffered), each fed the same G as the oracle
+    rng = np.random.default_rng(21)
+    m, k = 200, 333
+    a = _sparse(rng, m, k, 0.2)
+    ws = _ws(C, m, k, 1)
+    bufs = [_gpu_csr(C, a, ws), C.CSR(m, k)]
+    ref = O.csr_from_dense(a)
+    for step in range(5):
+        g = (rng.standard_normal((m, k)) * 0.3).astype(F32)
+        C.prox_update_compact(bufs[step % 2], _dev(g), 0.05, 0.5, bufs[(step + 1) % 2], ws)
+        ref = O.prox_update_compact(ref, g, 0.05, 0.5)
+        _check_csr_equal(bufs[(step + 1) % 2], ref)
+
+
+def test_prox_nan_is_dropped_and_flagged(C):
+    a = np.array([[1.0, 0.0, 2.0, 0.0]], dtype=F32)
+    g = np.array([[np.nan, 1.0, 0.0, np.nan]], dtype=F32)
+    ws = _ws(C, 1, 4, 1)
+    w = _gpu_csr(C, a, ws)
+    out = C.CSR(1, 4)
+    C.prox_update_compact(w, _dev(g), 0.5, 0.25, out, ws)
+    (rp, ci, v), _ = out.to_host()
+    assert ci.tolist() == [1, 2]
+    assert ws.status()[0] & C.CSRT_DEV_NONFINITE
+
+
+def test_debias_bit_exact_and_pattern_fixed(C):
+    rng = np.random.default_rng(5)
+    m, k = 120, 90
+    a = _sparse(rng, m, k, 0.3)
+    ws = _ws(C, m, k, 1)
+    w = _gpu_csr(C, a, ws)
+    ref = O.csr_from_dense(a)
+    g = rng.standard_normal(ref.nnz).astype(F32)
+    g[0] = ref.val[0] / F32(0.25)
+    before = w.to_host()
+    C.debias_update(w, _dev(g), 0.25)
+    (rp, ci, v), t = w.to_host()
+    out = O.debias_update(ref, g, 0.25)
+    np.testing.assert_array_equal(rp, before[0][0])
+    np.testing.assert_array_equal(ci, before[0][1])
+    np.testing.assert_array_equal(v.view(np.uint32), out.val.view(np.uint32))
+    assert v[0] == 0.0
+    np.testing.assert_array_equal(t[0], before[1][0])
+    np.testing.assert_array_equal(t[1], before[1][1])
+    np.testing.assert_array_equal(t[2][t[3]].view(np.uint32), v.view(np.uint32))
+
+
+# --- glue ----------------------------------------------------------------------
+
+def test_glue_layers(C):
+    rng = np.random.default_rng(9)
+    c, b, h, w, k = 3, 4, 12, 10, 5
+    x = rng.standard_normal((c, b, h, w)).astype(F32)
+    ho, wo = h - k + 1, w - k + 1
+    cols = torch.zeros(c * k * k, b * ho * wo, device="cuda")
+    C.im2col(_dev(x.reshape(c, -1)), c, b, h, w, k, cols)
+    np.testing.assert_array_equal(cols.cpu().numpy(), O.im2col(x, k))
+    dcols = rng.standard_normal((c * k * k, b * ho * wo)).astype(F32)
+    dx = torch.zeros(c, b * h * w, device="cuda")
+    C.col2im(_dev(dcols), c, b, h, w, k, dx)
+    assert_close(dx.cpu().numpy().reshape(c, b, h, w), O.col2im(dcols, c, b, h, w, k), what="col2im")
+    xp = rng.standard_normal((c, b, 8, 6)).astype(F32)
+    xp[0, 0, 0, :2] = 7.0                                   # a tie: first maximum wins
+    y = torch.zeros(c, b * 4 * 3, device="cuda")
+    idx = torch.zeros(c * b * 12, dtype=torch.int8, device="cuda")
+    C.maxpool2_fwd(_dev(xp.reshape(c, -1)), c, b, 8, 6, y, idx)
+    ry, ridx = O.maxpool2_fwd(xp)
+    np.testing.assert_array_equal(y.cpu().numpy().reshape(ry.shape), ry)
+    np.testing.assert_array_equal(idx.cpu().numpy().reshape(ridx.shape), ridx)
+    dyp = rng.standard_normal(ry.shape).astype(F32)
+    dxp = torch.zeros(c, b * 48, device="cuda")
+    C.maxpool2_bwd(_dev(dyp.reshape(c, -1)), idx, c, b, 8, 6, dxp)
+    np.testing.assert_array_equal(dxp.cpu().numpy().reshape(xp.shape), O.maxpool2_bwd(dyp, ridx))
+    xf = torch.zeros(c * 48, b, device="cuda")
+    C.flatten(_dev(xp.reshape(c, -1)), c, b, 48, xf)
+    np.testing.assert_array_equal(xf.cpu().numpy(), O.flatten_cnhw(xp))
+    back = torch.zeros(c, b * 48, device="cuda")
+    C.unflatten(xf, c, b, 48, back)
+    np.testing.assert_array_equal(back.cpu().numpy().reshape(xp.shape), xp)
+
+
+def test_bias_relu_softmax(C):
+    rng = np.random.default_rng(10)
+    m, n = 37, 70
+    y0 = rng.standard_normal((m, n)).astype(F32)
+    bias = rng.standard_normal(m).astype(F32)
+    y = _dev(y0)
+    C.bias_act_fwd(y, _dev(bias), True)
+    np.testing.assert_array_equal(y.cpu().numpy(), np.maximum(y0 + bias[:, None], 0).astype(F32))
+    d0 = rng.standard_normal((m, n)).astype(F32)
+    d = _dev(d0)
+    C.relu_bwd(d, y)
+    np.testing.assert_array_equal(d.cpu().numpy(), np.where(y.cpu().numpy() > 0, d0, 0))
+    b = _dev(bias)
+    gb = torch.zeros(m, device="cuda")
+    C.bias_grad_sgd(d, b, 0.1, gb)
+    ref_gb = d.cpu().numpy().astype(np.float64).sum(axis=1)
+    assert_close(gb.cpu().numpy(), ref_gb, np.abs(d.cpu().numpy()).sum(axis=1), n, what="bias grad")
+    np.testing.assert_array_equal(b.cpu().numpy(), (bias - F32(0.1) * gb.cpu().numpy()).astype(F32))
+    for classes in (10, 1000):
+        z = rng.standard_normal((classes, n)).astype(F32) * 3
+        lab = rng.integers(0, classes, n).astype(np.int32)
+        dz = torch.zeros(classes, n, device="cuda")
+        loss = torch.zeros(n + 1, device="cuda")
+        C.softmax_xent(_dev(z), _dev(lab), dz, loss)
+        rl, rdz = O.softmax_xent(z, lab)
+        assert abs(loss[0].item() - rl) <= 1e-5 * max(1, abs(rl))
+        assert_close(dz.cpu().numpy(), rdz, rtol=1e-4, atol=1e-7, what="softmax dz")

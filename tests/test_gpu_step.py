@@ -1,0 +1,159 @@
+"""Whole training steps of the five workloads against the oracle.
+
+Each GPU step is compared with the oracle run on the same current weights:
+the loss, every layer's gradient (dense G in the prox phase, g at the stored
+entries in the debias phase), and the updated CSR, which must be bit-exact
+with the oracle's update re-fed the GPU's own gradient (the gradients agree
+only up to summation order, so a free-running pattern could differ where
+|w - eta*G| sits within rounding of eta*lambda).
+"""
+
+import numpy as np
+import pytest
+
+import oracle as O
+from tests.parity import assert_close, csr_dense
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+F32 = np.float32
+
+
+@pytest.fixture(scope="module")
+def C():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_1905_07931_gb300 import csrtrain
+    csrtrain.lib()
+    return csrtrain
+
+
+def _host_csr(w):
+    (rp, ci, v), t = w.to_host()
+    return O.CSR(w.rows, w.cols, rp.copy(), ci.copy(), v.copy()), t
+
+
+def _assert_csr_bits(w, ref):
+    got, t = _host_csr(w)
+    np.testing.assert_array_equal(got.row_ptr, ref.row_ptr)
+    np.testing.assert_array_equal(got.col_idx, ref.col_idx)
+    np.testing.assert_array_equal(got.val.view(np.uint32), ref.val.astype(F32).view(np.uint32))
+    if t is not None:
+        trp, tci, tv, tpos = O.csr_transpose(ref)
+        np.testing.assert_array_equal(t[0], trp)
+        np.testing.assert_array_equal(t[1], tci)
+        np.testing.assert_array_equal(t[2].view(np.uint32), tv.astype(F32).view(np.uint32))
+        np.testing.assert_array_equal(t[3], tpos)
+
+
+@pytest.mark.parametrize("prec", [0, 1])
+def test_single_fc_layer_step(C, prec):
+    from paper_1905_07931_gb300 import synth
+    from paper_1905_07931_gb300.train import SingleLayer
+    cfg = synth.single_fc(seed=0)
+    lay = SingleLayer(cfg["W"], cfg["X"].shape[1], precision=prec)
+    lay.x.copy_(torch.from_numpy(cfg["X"]))
+    lay.dy.copy_(torch.from_numpy(cfg["dY"]))
+    w0 = O.csr_from_dense(cfg["W"])
+    _assert_csr_bits(lay.W[0], w0)
+    lay.step(cfg["eta"], cfg["lambda"])
+    torch.cuda.synchronize()
+    x, dy = cfg["X"], cfg["dY"]
+    assert_close(lay.y.cpu().numpy(), O.spmm_fwd(w0, x), O.spmm_fwd(O.csr_abs(w0), np.abs(x)),
+                 np.diff(w0.row_ptr)[:, None], what="Y")
+    assert_close(lay.dx.cpu().numpy(), O.spmm_bwd_t(w0, dy), O.spmm_bwd_t(O.csr_abs(w0), np.abs(dy)),
+                 np.bincount(w0.col_idx, minlength=w0.cols)[:, None], what="dX")
+    G = lay.G.cpu().numpy()
+    assert_close(G, O.weight_grad_dense(dy, x), O.weight_grad_dense(np.abs(dy), np.abs(x)), x.shape[1],
+                 rtol=1e-3 if prec else 1e-4, tf32=bool(prec), what="G")
+    _assert_csr_bits(lay.W[1], O.prox_update_compact(w0, G, cfg["eta"], cfg["lambda"]))
+    nnz = lay.W[1].nnz()
+    assert nnz > w0.nnz                                 # zero weights re-enter (dense w - eta*G)
+
+
+def _oracle_net(layers, net):
+    onet = O.Net([dict(l) for l in layers], [])
+    pi = 0
+    for L in layers:
+        if L["kind"] in ("fc", "conv"):
+            w, _ = _host_csr(net.weights(pi))
+            onet.params.append({"W": w, "b": net.params[pi]["b"].cpu().numpy().copy()})
+            pi += 1
+        else:
+            onet.params.append(None)
+    return onet
+
+
+def _run_and_compare(C, net, layers, x_host, labels, eta, lam, phase, prec, gtol_scale=1.0):
+    onet = _oracle_net(layers, net)
+    logits, cache = O.net_forward(onet, x_host, len(labels))
+    oloss, dz = O.softmax_xent(logits, labels)
+    ograds = O.net_backward(onet, cache, dz, phase)
+    loss = net.step(phase, eta, lam)
+    torch.cuda.synchronize()
+    assert net.ws.status()[0] == 0
+    got_loss = float(loss[0].item())
+    assert abs(got_loss - oloss) <= 2e-5 * max(1.0, abs(oloss)), (got_loss, oloss)
+    pl = [i for i, l in enumerate(layers) if l["kind"] in ("fc", "conv")]
+    for pi, li in enumerate(pl):
+        L = net.params[pi]
+        og = ograds[li]
+        old = onet.params[li]
+        if og is None:
+            continue
+        n = og["x"].shape[1]
+        absx = np.abs(og["x"])
+        absd = np.abs(og["delta"])
+        if phase == "prox":
+            G = L["G"].cpu().numpy()
+            assert_close(G, og["G"], O.weight_grad_dense(absd, absx) * 1.01, n,
+                         rtol=1e-3 if prec else 1e-4, tf32=bool(prec), what=f"G layer {pi}")
+            _assert_csr_bits(net.weights(pi), O.prox_update_compact(old["W"], G, eta, lam))
+        else:
+            w = old["W"]
+            g = L["g"].cpu().numpy()[: w.nnz]
+            assert_close(g, og["g"], O.weight_grad_sddmm(w, absd, absx) * 1.01, n, what=f"g layer {pi}")
+            _assert_csr_bits(net.weights(pi), O.debias_update(w, g, eta))
+    return got_loss
+
+
+@pytest.mark.parametrize("prec", [0, 1])
+def test_mlp_prox_then_debias(C, prec):
+    from paper_1905_07931_gb300 import synth
+    from paper_1905_07931_gb300.train import SparseNet, mlp_layers
+    cfg = synth.mlp(seed=0)
+    layers = mlp_layers(3)
+    net = SparseNet(layers, cfg["W"], cfg["b"], 256, (784,), precision=prec, grad_per_layer=True)
+    net.x_in.copy_(torch.from_numpy(cfg["X"]))
+    net.labels.copy_(torch.from_numpy(cfg["labels"]))
+    for _ in range(3):
+        _run_and_compare(C, net, layers, cfg["X"], cfg["labels"], cfg["eta"], cfg["lambda"], "prox", prec)
+    for _ in range(3):
+        _run_and_compare(C, net, layers, cfg["X"], cfg["labels"], cfg["eta"], cfg["lambda"], "debias", prec)
+
+
+def test_lenet_prox_then_debias(C):
+    from paper_1905_07931_gb300 import synth
+    from paper_1905_07931_gb300.train import SparseNet, lenet_layers
+    cfg = synth.lenet(seed=0)
+    layers = lenet_layers()
+    net = SparseNet(layers, cfg["W"], cfg["b"], 128, (1, 28, 28), precision=1, grad_per_layer=True)
+    net.x_in.copy_(torch.from_numpy(cfg["X"].reshape(1, -1)))
+    net.labels.copy_(torch.from_numpy(cfg["labels"]))
+    for phase in ("prox", "prox", "debias", "debias"):
+        _run_and_compare(C, net, layers, cfg["X"], cfg["labels"], cfg["eta"], cfg["lambda"], phase, 1)
+
+
+def test_fc_head_full_size_step(C):
+    """The AlexNet-sized head (9216-4096-4096-1000, batch 256) at full size:
+    one prox step and one debias step, every layer checked."""
+    from paper_1905_07931_gb300 import synth
+    from paper_1905_07931_gb300.train import SparseNet, mlp_layers
+    cfg = synth.fc_head(seed=0)
+    layers = mlp_layers(3)
+    net = SparseNet(layers, cfg["W"], cfg["b"], 256, (9216,), precision=1, grad_per_layer=True)
+    net.x_in.copy_(torch.from_numpy(cfg["X"]))
+    net.labels.copy_(torch.from_numpy(cfg["labels"]))
+    _run_and_compare(C, net, layers, cfg["X"], cfg["labels"], cfg["eta"], cfg["lambda"], "prox", 1)
+    net.reset_weights()
+    _run_and_compare(C, net, layers, cfg["X"], cfg["labels"], cfg["eta"], cfg["lambda"], "debias", 1)
