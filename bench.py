@@ -1,0 +1,515 @@
+#!/usr/bin/env python3
+"""Throughput of the CSR-weight training step on one GB300 (or N replicas).
+
+Workload: the AlexNet-sized classifier head (FC 9216 -> 4096 -> 4096 -> 1000,
+ReLU, softmax cross-entropy) with CSR weights at 5% / 5% / 15% density,
+batch 256, on synthetic half-normal 9216-dim features and uniform labels
+(seed 0): one full training step of the l1-proximal phase = forward SpMM x3,
+loss, dense weight gradients (tcgen05 TF32), transposed SpMM x2, bias SGD,
+prox update + CSR re-compaction x3 (and the transposed pattern of the two
+layers whose input gradient is needed).
+
+Timing: W eager warm-up steps, then the step is captured in a CUDA graph and
+K replays are timed one by one with CUDA events on the replay stream. Before
+every step (outside the timed region) the biases are restored and a 256 MB
+buffer is written to flush the 126 MB L2. Every step starts from the initial
+CSR weights (the prox step writes the second buffer), so each timed step does
+the same work. `value` = samples of all ranks / max over ranks of the summed
+step times.
+
+Also reported: `e2e` (the same step with the batch copied from pinned host
+memory and the loss read back inside the timed region), `roofline` of the
+dominant kernel (timed with CUDA events in an instrumented eager step),
+`cpu_baseline` (the CPU oracle on a row sample of the same step) and the SM
+clocks sampled during the timed region.
+
+`--impl reference` times the CPU oracle instead (rank 0 only).
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "sparse train-step samples/sec at 1 GB300; SpMM/SDDMM/prox HBM GB/s vs peak"
+UNIT = "samples/s"
+SIZES = (9216, 4096, 4096, 1000)
+DENSITIES = (0.05, 0.05, 0.15)
+BATCH = 256
+WORKLOAD = "fc_head 9216-4096-4096-1000 CSR 5/5/15%, batch 256, prox-SGD step (eta 0.01, lambda 1e-4)"
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--precision", choices=["tf32", "fp32"], default="tf32")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--profile-ops", action="store_true", help="print the per-operation breakdown to stderr")
+    return p.parse_args()
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle on a row sample of the step (cpu_baseline and --impl reference)
+# ---------------------------------------------------------------------------
+
+class OracleSample:
+    """Every operation of the step is separable over the output rows of each
+    layer (forward rows, gradient rows, prox rows, the partial W^T dY of those
+    rows). A sample runs every operation on 1/F of each layer's rows, with the
+    true layer inputs precomputed once; its time times F estimates one full
+    step."""
+
+    def __init__(self, cfg, fraction_denominator: int):
+        import numpy as np
+
+        import oracle as O
+        self.O, self.np = O, np
+        self.F = int(fraction_denominator)
+        self.cfg = cfg
+        self.eta, self.lam = cfg["eta"], cfg["lambda"]
+        ws = [O.csr_from_dense(w) for w in cfg["W"]]
+        net = O.Net([{"kind": "fc", "relu": i < 2} for i in range(3)],
+                    [{"W": w, "b": b.copy()} for w, b in zip(ws, cfg["b"])])
+        logits, cache = O.net_forward(net, cfg["X"], BATCH)
+        _, dz = O.softmax_xent(logits, cfg["labels"])
+        grads = O.net_backward(net, cache, dz, "debias")   # deltas only (cheap phase)
+        self.layers = []
+        for li in range(3):
+            w = ws[li]
+            rows = np.arange(0, w.rows, self.F)
+            sub = self._rows(w, rows)
+            self.layers.append({"W": sub, "x": cache[li]["x"].astype(np.float32),
+                                "delta": grads[li]["delta"][rows].astype(np.float32),
+                                "b": cfg["b"][li][rows].copy(), "relu": li < 2, "dx": li > 0})
+        self.logits = logits.astype(np.float32)
+
+    def _rows(self, w, rows):
+        O, np = self.O, self.np
+        rp = w.row_ptr.astype(np.int64)
+        idx = np.concatenate([np.arange(rp[r], rp[r + 1]) for r in rows]) if len(rows) else np.zeros(0, np.int64)
+        lens = rp[rows + 1] - rp[rows]
+        new_rp = np.zeros(len(rows) + 1, np.int64)
+        new_rp[1:] = np.cumsum(lens)
+        return O.CSR(len(rows), w.cols, new_rp.astype(np.int32), w.col_idx[idx], w.val[idx])
+
+    def step(self) -> float:
+        """Run one sample; return the estimated seconds of one full step."""
+        O, np = self.O, self.np
+        t0 = time.perf_counter()
+        for L in self.layers:
+            pre = O.spmm_fwd(L["W"], L["x"]) + L["b"][:, None]
+            if L["relu"]:
+                pre = O.relu(pre)
+        t_rows = time.perf_counter() - t0
+        t1 = time.perf_counter()
+        O.softmax_xent(self.logits, self.cfg["labels"])     # the loss is computed once per step
+        t_once = time.perf_counter() - t1
+        t2 = time.perf_counter()
+        for L in self.layers:
+            G = O.weight_grad_dense(L["delta"], L["x"]).astype(np.float32)
+            if L["dx"]:
+                O.spmm_bwd_t(L["W"], L["delta"])
+            new = O.prox_update_compact(L["W"], G, self.eta, self.lam)
+            if L["dx"]:
+                O.csr_transpose(new)
+            L["delta"].sum(axis=1)
+        t_rows += time.perf_counter() - t2
+        return t_rows * self.F + t_once
+
+    def describe(self) -> str:
+        return (f"CPU oracle (numpy, float64 sums) on every operation of one step restricted to 1/{self.F} "
+                f"of each layer's output rows (forward, loss, weight gradient, W^T dY, prox + compaction, "
+                f"transposed pattern); time x {self.F}")
+
+
+def cpu_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_1905_07931_gb300 import synth
+    cfg = synth.fc_head(seed=0)
+    samp = OracleSample(cfg, fraction_denominator=8)
+    for _ in range(args.warmup):
+        samp.step()
+    times = [samp.step() for _ in range(args.steps)]
+    total = sum(times)
+    value = args.steps * BATCH / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": WORKLOAD, "global_batch": BATCH, "parallelism": "none"},
+        "cpu_baseline": {"kind": "oracle", "value": value, "unit": UNIT, "cores": cpu_cores(),
+                         "sample": samp.describe()},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for nm, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# Roofline bookkeeping
+# ---------------------------------------------------------------------------
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+def recorded_traffic(kernel: str):
+    """dram bytes per launch from the committed ncu summary, if it was taken
+    on the current source of the kernel's file (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f).get(kernel)
+        if not rec:
+            return None
+        src = os.path.join(ROOT, "paper_1905_07931_gb300", "csrc", rec["source"])
+        with open(src, "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()[:16]
+        return rec["dram_bytes_per_launch"] if sha == rec["sha256_16"] else None
+    except Exception:
+        return None
+
+
+def op_bytes(name, info):
+    """Algorithmic HBM bytes (each operand touched once) of one call."""
+    M, K, n = info["M"], info["K"], info.get("n", 0)
+    nnz, nnz_out = info.get("nnz", 0), info.get("nnz_out", 0)
+    if name == "spmm_fwd":
+        return 8 * nnz + 4 * (M + 1) + 4 * n * (K + M)
+    if name == "spmm_bwd_t":
+        return 8 * nnz + 4 * (K + 1) + 4 * n * (K + M)
+    if name == "weight_grad_dense":
+        return 4 * M * K + 4 * n * (M + K)
+    if name == "weight_grad_sddmm":
+        return 12 * nnz + 4 * (M + 1) + 4 * n * (K + M)
+    if name == "prox_update_compact":
+        b = 4 * M * K + 8 * nnz + 4 * (M + 1) + 8 * nnz_out + 4 * (M + 1)
+        if info.get("transposed"):
+            b += 8 * nnz_out + 4 * (M + 1) + 12 * nnz_out + 4 * (K + 1)
+        return b
+    return None
+
+
+# ---------------------------------------------------------------------------
+# Our arm
+# ---------------------------------------------------------------------------
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    rank, world, local_rank = dist_env()
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    from paper_1905_07931_gb300 import csrtrain as C
+    from paper_1905_07931_gb300 import synth
+    from paper_1905_07931_gb300.train import SparseNet, mlp_layers
+
+    prec = C.CSRT_PREC_TF32 if args.precision == "tf32" else C.CSRT_PREC_FP32
+    cfg = synth.fc_head(seed=0)
+    layers = mlp_layers(3)
+    net = SparseNet(layers, cfg["W"], cfg["b"], BATCH, (SIZES[0],), precision=prec)
+    x_host = torch.from_numpy(cfg["X"]).pin_memory()
+    lab_host = torch.from_numpy(cfg["labels"]).pin_memory()
+    net.x_in.copy_(x_host)
+    net.labels.copy_(lab_host)
+    b0 = [L["b"].clone() for L in net.params]
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
+    eta, lam = cfg["eta"], cfg["lambda"]
+
+    def restore():
+        for L, b in zip(net.params, b0):
+            L["b"].copy_(b)
+            L["cur"] = 0
+
+    # warm-up (eager)
+    for _ in range(max(args.warmup, 0)):
+        restore()
+        net.step("prox", eta, lam)
+    torch.cuda.synchronize()
+    flags, _ = net.ws.status()
+    if flags:
+        raise SystemExit(f"device status {flags} after warm-up")
+
+    # per-operation breakdown of one eager step (events around every library call)
+    restore()
+    prof = profile_ops(net, C, torch, eta, lam, flush)
+    restore()
+
+    # capture one step in a CUDA graph
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    C.launch_count(reset=True)
+    with torch.cuda.stream(s):
+        restore()
+        with torch.cuda.graph(graph, stream=s):
+            net.step("prox", eta, lam)
+    launches_per_step = C.launch_count(reset=True)
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+
+    stream = torch.cuda.current_stream()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    clocks = ClockSampler(local_rank)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    wall0 = time.perf_counter()
+    for i in range(args.steps):
+        restore()
+        flush.fill_(float(i))
+        starts[i].record(stream)
+        graph.replay()
+        ends[i].record(stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    times_ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
+    total_ms = sum(times_ms)
+    tot = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(tot, op=dist.ReduceOp.MAX)
+    total_max_ms = float(tot.item())
+    value = world * args.steps * BATCH / (total_max_ms / 1e3)
+    flags, _ = net.ws.status()
+    if flags:
+        raise SystemExit(f"device status {flags} after the timed steps")
+
+    # end to end: pinned host batch -> device, step, loss -> pinned host
+    loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
+    e_starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    e_ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    for i in range(args.steps):
+        restore()
+        flush.fill_(float(i))
+        e_starts[i].record(stream)
+        net.x_in.copy_(x_host, non_blocking=True)
+        net.labels.copy_(lab_host, non_blocking=True)
+        graph.replay()
+        loss_host.copy_(net.loss[:1], non_blocking=True)
+        e_ends[i].record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = sum(a.elapsed_time(b) for a, b in zip(e_starts, e_ends))
+    et = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(et, op=dist.ReduceOp.MAX)
+    e2e_value = world * args.steps * BATCH / (float(et.item()) / 1e3)
+
+    # roofline of the dominant kernel
+    peaks, peak_kind = measured_peaks()
+    dom = max(prof, key=lambda r: r["ms"])
+    bytes_ = op_bytes(dom["name"], dom["info"])
+    roof = None
+    if bytes_ is not None:
+        if dom["name"] == "weight_grad_dense":
+            flops = 2.0 * dom["info"]["M"] * dom["info"]["K"] * dom["info"]["n"]
+        achieved = bytes_ / (dom["ms"] / 1e3) / 1e9
+        kernel = dom["kernel"]
+        roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": recorded_traffic(kernel),
+                "kernel": kernel, "op": dom["label"], "algorithmic_bytes": int(bytes_),
+                "launch_ms": round(dom["ms"], 4), "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"
+                if peak_kind == "measured" else "fallback 6.8 TB/s"}
+
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(total_max_ms / args.steps, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "global_batch": BATCH * world, "per_gpu_batch": BATCH,
+                   "layers": list(SIZES), "densities": list(DENSITIES),
+                   "weight_grad": "tf32 tcgen05" if prec == C.CSRT_PREC_TF32 else "fp32 simt",
+                   "l2": "flushed between steps (256 MB write, outside the timed region)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "step_ops": [r["label"] for r in prof]},
+        "e2e": {"value": round(e2e_value, 1), "unit": UNIT,
+                "h2d_bytes_per_step": int(x_host.numel() * 4 + lab_host.numel() * 4), "d2h_bytes_per_step": 4},
+        "gpu_launches": int(launches_per_step * args.steps),
+        "roofline": roof,
+        "clocks": clk,
+        "wall_s_timed_region": round(wall, 3),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        samp = OracleSample(cfg, fraction_denominator=4)
+        est = [samp.step() for _ in range(2)]
+        v = BATCH / (sum(est) / len(est))
+        line["cpu_baseline"] = {"value": round(v, 3), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                                "sample": samp.describe() + ", 2 samples"}
+    if args.profile_ops and rank == 0:
+        for r in prof:
+            b = op_bytes(r["name"], r["info"])
+            gbs = f"{b / (r['ms'] / 1e3) / 1e9:8.1f} GB/s" if b else ""
+            print(f"{r['label']:<36s} {r['ms'] * 1e3:9.1f} us {gbs}", file=sys.stderr)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def profile_ops(net, C, torch, eta, lam, flush):
+    """Run one eager step with CUDA events around every library call on the
+    launching stream; return [{label, name, kernel, ms, info}] in call order."""
+    stream = torch.cuda.current_stream()
+    records = []
+    wrapped = {}
+    names = ["spmm_fwd", "spmm_bwd_t", "weight_grad_dense", "weight_grad_sddmm", "prox_update_compact",
+             "debias_update", "bias_act_fwd", "relu_bwd", "bias_grad_sgd", "softmax_xent"]
+    kernel_of = {"spmm_fwd": "spmm_merge_kernel", "spmm_bwd_t": "spmm_merge_kernel",
+                 "weight_grad_dense": "gemm", "weight_grad_sddmm": "sddmm_kernel",
+                 "prox_update_compact": "compact_kernel", "debias_update": "debias_kernel"}
+    layer_of = {}
+    for i, L in enumerate(net.params):
+        for W in L["W"]:
+            layer_of[id(W)] = i
+    for nm in names:
+        orig = getattr(C, nm)
+        wrapped[nm] = orig
+
+        def make(nm, orig):
+            def fn(*a, **k):
+                st = torch.cuda.Event(enable_timing=True)
+                en = torch.cuda.Event(enable_timing=True)
+                st.record(stream)
+                orig(*a, **k)
+                en.record(stream)
+                info = {}
+                W = a[0] if a and isinstance(a[0], C.CSR) else None
+                li = layer_of.get(id(W)) if W is not None else None
+                if nm in ("spmm_fwd", "spmm_bwd_t", "weight_grad_sddmm", "prox_update_compact", "debias_update"):
+                    info = {"M": W.rows, "K": W.cols, "W": W}
+                    if nm in ("spmm_fwd", "spmm_bwd_t", "weight_grad_sddmm"):
+                        info["n"] = a[1].shape[1] if a[1].dim() == 2 else 0
+                    if nm == "prox_update_compact":
+                        info["W_out"] = a[4]
+                        info["transposed"] = a[4].transposed
+                elif nm == "weight_grad_dense":
+                    dy, x = a[0], a[1]
+                    info = {"M": dy.shape[0], "K": x.shape[0], "n": dy.shape[1]}
+                    li = next((i for i, L in enumerate(net.params) if L["W"][0].rows == dy.shape[0]
+                               and L["W"][0].cols == x.shape[0]), None)
+                records.append({"name": nm, "st": st, "en": en, "info": info, "layer": li})
+            return fn
+        setattr(C, nm, make(nm, orig))
+    try:
+        flush.fill_(1.0)
+        torch.cuda.synchronize()
+        net.step("prox", eta, lam)
+        torch.cuda.synchronize()
+    finally:
+        for nm, orig in wrapped.items():
+            setattr(C, nm, orig)
+    out = []
+    for r in records:
+        info = r["info"]
+        if "W" in info:
+            info["nnz"] = info["W"].nnz()
+            del info["W"]
+        if "W_out" in info:
+            info["nnz_out"] = info["W_out"].nnz()
+            del info["W_out"]
+        lab = r["name"] + (f"[layer {r['layer']}]" if r["layer"] is not None else "")
+        out.append({"label": lab, "name": r["name"], "kernel": kernel_of.get(r["name"], r["name"]),
+                    "ms": r["st"].elapsed_time(r["en"]), "info": info})
+    return out
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -96,7 +96,7 @@ class SparseNet:
                 L["g"] = torch.zeros(M * K, **dev)
                 if grad_per_layer:
                     L["G"] = torch.zeros(M, K, **dev)
-                max_rows, max_cols, max_n = max(max_rows, M, K), max(max_cols, K, M), max(max_n, n)
+                max_rows, max_cols, max_n = max(max_rows, M), max(max_cols, K), max(max_n, n)
                 max_mk = max(max_mk, M * K)
                 cur = L["y"]
                 self.params.append(L)
@@ -125,7 +125,7 @@ class SparseNet:
         self.dlogits = torch.zeros_like(cur)
         self.loss = torch.zeros(B + 1, **dev)
         self.G = torch.zeros(max_mk, **dev)
-        self.ws = C.Workspace(max(max_rows, max_cols), max(max_rows, max_cols), max_n, device=device, stream=stream)
+        self.ws = C.Workspace(max_rows, max_cols, max_n, device=device, stream=stream)
         for L in self.params:
             C.csr_from_dense(L["W0"], L["W"][0], self.ws, stream)
 
@@ -241,7 +241,7 @@ class SingleLayer:
         self.y = torch.zeros(M, n, device=device)
         self.dx = torch.zeros(K, n, device=device)
         self.G = torch.zeros(M, K, device=device)
-        self.ws = C.Workspace(max(M, K), max(M, K), n, device=device, stream=stream)
+        self.ws = C.Workspace(M, K, n, device=device, stream=stream)
         C.csr_from_dense(self.W0, self.W[0], self.ws, stream)
 
     def step(self, eta: float, lam: float):

@@ -32,7 +32,7 @@ def C():
 
 
 def _ws(C, rows, cols, n):
-    return C.Workspace(max(rows, cols, 1), max(rows, cols, 1), max(n, 1))
+    return C.Workspace(max(rows, 1), max(cols, 1), max(n, 1))
 
 
 def _sparse(rng, m, k, density, zipf=False):
