@@ -257,6 +257,8 @@ def recorded_traffic(kernel: str):
 
 def op_bytes(name, info):
     """Algorithmic HBM bytes (each operand touched once) of one call."""
+    if "M" not in info:
+        return None
     M, K, n = info["M"], info["K"], info.get("n", 0)
     nnz, nnz_out = info.get("nnz", 0), info.get("nnz_out", 0)
     if name == "spmm_fwd":
@@ -395,7 +397,7 @@ def main():
 
     # roofline of the dominant kernel
     peaks, peak_kind = measured_peaks()
-    dom = max(prof, key=lambda r: r["ms"])
+    dom = max((r for r in prof if op_bytes(r["name"], r["info"]) is not None), key=lambda r: r["ms"])
     bytes_ = op_bytes(dom["name"], dom["info"])
     roof = None
     if bytes_ is not None:

@@ -304,7 +304,7 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
 // Transposed pattern (column-wise copy), deterministic.
 // ---------------------------------------------------------------------------
 constexpr int kTrRows = 32;      // rows per block: one bit each in a 32-bit word
-constexpr int kTrChunk = 8192;   // columns per block (32 KB of bitmask words)
+constexpr int kTrChunk = 4096;   // most columns per block (16 KB of bitmask words)
 
 size_t transpose_scratch_bytes(int32_t rows, int32_t cols) {
     const int64_t nb = ceil_div<int64_t>(rows, kTrRows);
@@ -333,10 +333,10 @@ __device__ __forceinline__ void tr_build_bits(unsigned int *bits, const int32_t 
 
 __global__ void __launch_bounds__(256) tr_count_kernel(const int32_t *__restrict__ row_ptr,
                                                        const int32_t *__restrict__ col, int32_t rows,
-                                                       int32_t cols, int32_t *__restrict__ cnt) {
+                                                       int32_t cols, int32_t chunk, int32_t *__restrict__ cnt) {
     __shared__ unsigned int bits[kTrChunk];
-    const int b = blockIdx.x, c0 = blockIdx.y * kTrChunk;
-    const int cw = min(kTrChunk, cols - c0);
+    const int b = blockIdx.x, c0 = blockIdx.y * chunk;
+    const int cw = min(chunk, cols - c0);
     tr_build_bits(bits, row_ptr, col, rows, b, c0, cw, gridDim.y > 1);
     int32_t *out = cnt + (int64_t)b * cols + c0;
     for (int j = threadIdx.x; j < cw; j += blockDim.x) out[j] = __popc(bits[j]);
@@ -402,14 +402,17 @@ __global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict
                                                        int32_t cols, const int32_t *__restrict__ off,
                                                        const int32_t *__restrict__ t_row_ptr,
                                                        int32_t *__restrict__ t_col, float *__restrict__ t_val,
-                                                       int32_t *__restrict__ t_pos, int64_t capacity) {
+                                                       int32_t *__restrict__ t_pos, int64_t capacity,
+                                                       int32_t chunk) {
     __shared__ unsigned int bits[kTrChunk];
-    const int b = blockIdx.x, c0 = blockIdx.y * kTrChunk;
-    const int cw = min(kTrChunk, cols - c0);
+    __shared__ int32_t base[kTrChunk];   // first position of this block's run in each column
+    const int b = blockIdx.x, c0 = blockIdx.y * chunk;
+    const int cw = min(chunk, cols - c0);
     const bool chunked = gridDim.y > 1;
+    const int32_t *boff = off + (int64_t)b * cols + c0;
+    for (int j = threadIdx.x; j < cw; j += blockDim.x) base[j] = t_row_ptr[c0 + j] + boff[j];
     tr_build_bits(bits, row_ptr, col, rows, b, c0, cw, chunked);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int32_t *boff = off + (int64_t)b * cols;
     for (int rr = warp; rr < kTrRows; rr += blockDim.x / 32) {
         const int r = b * kTrRows + rr;
         if (r >= rows) break;
@@ -420,8 +423,8 @@ __global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict
         }
         const unsigned int below = (1u << rr) - 1u;
         for (int64_t k = s + lane; k < e; k += 32) {
-            const int j = __ldg(col + k);
-            const int64_t p = (int64_t)t_row_ptr[j] + boff[j] + __popc(bits[j - c0] & below);
+            const int j = __ldg(col + k) - c0;
+            const int64_t p = (int64_t)base[j] + __popc(bits[j] & below);
             if (p < capacity) {
                 t_col[p] = r;
                 t_val[p] = __ldg(val + k);
@@ -441,15 +444,20 @@ int transpose_impl(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s) {
     }
     CSRT_ARG(ws_bytes >= kWsHeaderBytes + transpose_scratch_bytes(rows, cols), "workspace too small for transpose");
     const int nb = (int)ceil_div<int64_t>(rows, kTrRows);
-    const int nc = (int)ceil_div<int64_t>(cols, kTrChunk);
+    // Enough blocks to fill the GPU: split the columns into chunks of at least
+    // 256 (and at most kTrChunk) so that nb * nc reaches ~4 blocks per SM.
+    int nc = (int)imax<int64_t>(ceil_div<int64_t>(cols, kTrChunk),
+                                imin<int64_t>(ceil_div<int64_t>(4 * num_sms(), nb), ceil_div<int64_t>(cols, 256)));
+    const int chunk = (int)ceil_div<int64_t>(ceil_div<int64_t>(cols, nc), 32) * 32;
+    nc = (int)ceil_div<int64_t>(cols, chunk);
     int32_t *cnt = reinterpret_cast<int32_t *>(ws_scratch(ws));
     int32_t *coltot = cnt + (int64_t)nb * cols;
-    tr_count_kernel<<<dim3(nb, nc), 256, 0, s>>>(w->row_ptr, w->col_idx, rows, cols, cnt);
+    tr_count_kernel<<<dim3(nb, nc), 256, 0, s>>>(w->row_ptr, w->col_idx, rows, cols, chunk, cnt);
     tr_colscan_kernel<<<ceil_div(cols, 32), 256, 0, s>>>(cnt, nb, cols, coltot);
     scan_single_block_kernel<<<1, 1024, 0, s>>>(coltot, cols, w->t_row_ptr);
     tr_write_kernel<<<dim3(nb, nc), 256, 0, s>>>(w->row_ptr, w->col_idx, w->val, rows, cols, cnt,
                                                  w->t_row_ptr, w->t_col_idx, w->t_val, w->t_pos,
-                                                 w->capacity);
+                                                 w->capacity, chunk);
     count_launch(4);
     return check_launch("csr_transpose kernels");
 }
