@@ -55,6 +55,57 @@ struct CompactArgs {
     int64_t num_tiles;
 };
 
+// Decoupled look-back for tile `tile`, run by one whole warp: publishes the
+// tile's aggregate, sums predecessors' aggregates back to the nearest
+// published inclusive prefix, publishes this tile's inclusive prefix and
+// returns the exclusive prefix (the number of entries kept before the tile).
+// Every poll is bounded; a wait that runs out sets CSRT_DEV_TIMEOUT.
+__device__ __forceinline__ unsigned long long lookback_warp(unsigned long long *status, int64_t tile,
+                                                            uint32_t count, WsHeader *hdr) {
+    const int lane = threadIdx.x & 31;
+    unsigned long long prefix = 0;
+    if (tile == 0) {
+        if (lane == 0) st_release_u64(status, kFlagInc | count);
+        return 0;
+    }
+    if (lane == 0) st_release_u64(status + tile, kFlagAgg | count);
+    int64_t pred = tile - 1;
+    unsigned int spins = 0;
+    bool timed_out = false;
+    while (true) {
+        const int64_t idx = pred - lane;
+        unsigned long long st = idx >= 0 ? ld_acquire_u64(status + idx) : kFlagInc;
+        while (__any_sync(0xffffffffu, (st >> 32) == 0)) {
+            if (++spins > kSpinLimit) {
+                timed_out = true;
+                break;
+            }
+            __nanosleep(64);
+            if ((st >> 32) == 0) st = ld_acquire_u64(status + idx);
+        }
+        if (timed_out) break;
+        const unsigned inc_mask = __ballot_sync(0xffffffffu, (st >> 32) == 2);
+        unsigned long long part = st & 0xffffffffull;
+        if (inc_mask) {
+            const int first = __ffs(inc_mask) - 1;  // nearest inclusive predecessor
+            if (lane > first) part = 0;
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
+        prefix += part;
+        if (inc_mask) break;
+        pred -= 32;
+    }
+    if (lane == 0) {
+        if (timed_out) {
+            dev_flag(hdr, CSRT_DEV_TIMEOUT);
+            hdr->timeout_site = 1;
+        }
+        st_release_u64(status + tile, kFlagInc | (prefix + count));
+    }
+    return prefix;
+}
+
 template <bool kProx, bool kVec>
 __global__ void __launch_bounds__(kCThreads) compact_kernel(CompactArgs a) {
     __shared__ __align__(16) float w_tile[kProx ? kTile : 4];
@@ -177,43 +228,7 @@ __global__ void __launch_bounds__(kCThreads) compact_kernel(CompactArgs a) {
 
     // 5. Decoupled look-back for the number of entries kept before this tile.
     if (warp == 0) {
-        unsigned long long prefix = 0;
-        if (tile == 0) {
-            if (lane == 0) st_release_u64(a.status, kFlagInc | tile_count);
-        } else {
-            if (lane == 0) st_release_u64(a.status + tile, kFlagAgg | tile_count);
-            int64_t pred = tile - 1;
-            unsigned int spins = 0;
-            bool timed_out = false;
-            while (true) {
-                const int64_t idx = pred - lane;
-                unsigned long long st = idx >= 0 ? ld_acquire_u64(a.status + idx) : kFlagInc;
-                while (__any_sync(0xffffffffu, (st >> 32) == 0)) {
-                    if (++spins > kSpinLimit) { timed_out = true; break; }
-                    __nanosleep(64);
-                    if ((st >> 32) == 0) st = ld_acquire_u64(a.status + idx);
-                }
-                if (timed_out) break;
-                const unsigned inc_mask = __ballot_sync(0xffffffffu, (st >> 32) == 2);
-                unsigned long long part = st & 0xffffffffull;
-                if (inc_mask) {
-                    const int first = __ffs(inc_mask) - 1;  // nearest inclusive predecessor
-                    if (lane > first) part = 0;
-                }
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
-                prefix += part;
-                if (inc_mask) break;
-                pred -= 32;
-            }
-            if (lane == 0) {
-                if (timed_out) {
-                    dev_flag(a.hdr, CSRT_DEV_TIMEOUT);
-                    a.hdr->timeout_site = 1;
-                }
-                st_release_u64(a.status + tile, kFlagInc | (prefix + tile_count));
-            }
-        }
+        const unsigned long long prefix = lookback_warp(a.status, tile, tile_count, a.hdr);
         if (lane == 0) s_excl = prefix;
     }
     __syncthreads();
@@ -256,6 +271,208 @@ __global__ void __launch_bounds__(kCThreads) compact_kernel(CompactArgs a) {
     }
 }
 
+
+// ---------------------------------------------------------------------------
+// Row-tile compaction (the fast path: K % 4 == 0, K <= kRowMaxK, G 16-byte
+// aligned). A tile is R whole rows (R*K <= max(K, kRowBudget) entries), so the
+// old CSR entries of a tile are the contiguous range row_ptr[r0] ..
+// row_ptr[r0+R) and no search is needed. The grid is persistent (two blocks
+// per SM); each block takes tiles by ticket and, while it works on one tile,
+// its next tile's slice of G is already streaming into shared memory with a
+// bulk asynchronous copy (cp.async.bulk, completion on an mbarrier). Each warp
+// compacts a contiguous segment of the tile 32 entries at a time with ballots,
+// so kept entries leave as coalesced runs.
+// ---------------------------------------------------------------------------
+constexpr int kRowBudget = 8192;     // entries per tile when rows are short
+constexpr int kRowMaxK = 16384;      // longest row the row-tile path takes
+constexpr unsigned kRowWaitLimit = 1u << 22;
+
+__device__ __forceinline__ uint32_t cvta_smem(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ bool row_mbar_wait(uint64_t *bar, uint32_t parity) {
+    const uint32_t addr = cvta_smem(bar);
+    for (unsigned i = 0; i < kRowWaitLimit; ++i) {
+        uint32_t done;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            " selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(done)
+            : "r"(addr), "r"(parity)
+            : "memory");
+        if (done) return true;
+        if (i > 32) __nanosleep(32);
+    }
+    return false;
+}
+
+// Thread 0 only: stream `bytes` of G (16-byte aligned, multiple of 16) into smem.
+__device__ __forceinline__ void bulk_load(float *dst, const float *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(cvta_smem(bar)), "r"(bytes)
+                 : "memory");
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            cvta_smem(dst)),
+        "l"(src), "r"(bytes), "r"(cvta_smem(bar))
+        : "memory");
+}
+
+template <bool kProx>
+__global__ void __launch_bounds__(kCThreads, 2) compact_rows_kernel(CompactArgs a, int32_t rows_per_tile,
+                                                                     int32_t tile_elems) {
+    extern __shared__ __align__(128) float row_smem[];
+    float *const gbuf0 = row_smem;   // G of the current / next tile: gbuf0 + cb * tile_elems
+    float *wt = row_smem + 2 * tile_elems;                                     // old weights (prox)
+    int32_t *s_rp = reinterpret_cast<int32_t *>(wt + (kProx ? tile_elems : 0));  // rows_per_tile + 1
+    __shared__ __align__(8) uint64_t s_bar[2];
+    __shared__ unsigned int s_ticket[2];
+    __shared__ uint32_t s_wtot[kCThreads / 32];
+    __shared__ unsigned long long s_excl;
+    __shared__ int s_fail;
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int64_t K = a.cols;
+    const int R = rows_per_tile;
+    if (tid == 0) {
+        s_fail = 0;
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(cvta_smem(&s_bar[0])) : "memory");
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(cvta_smem(&s_bar[1])) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        const unsigned t = atomicAdd(&a.hdr->ticket, 1u);
+        s_ticket[0] = t;
+        if (t < a.num_tiles) {
+            const int64_t r0 = (int64_t)t * R;
+            const int64_t nrows = imin<int64_t>(R, a.rows - r0);
+            bulk_load(gbuf0, a.src + r0 * K, (uint32_t)(nrows * K * 4), &s_bar[0]);
+        }
+    }
+    __syncthreads();
+    uint32_t phases = 0;   // bit b: parity of the next completion of s_bar[b]
+    int cb = 0;
+    bool nonfinite = false;
+    for (;;) {
+        const int64_t tile = s_ticket[cb];
+        if (tile >= a.num_tiles) break;
+        // prefetch the next tile into the other buffer (its last reader finished
+        // before the trailing barrier of the previous iteration)
+        if (tid == 0) {
+            const unsigned t = atomicAdd(&a.hdr->ticket, 1u);
+            s_ticket[cb ^ 1] = t;
+            if (t < a.num_tiles) {
+                const int64_t r0 = (int64_t)t * R;
+                const int64_t nrows = imin<int64_t>(R, a.rows - r0);
+                bulk_load(gbuf0 + (cb ^ 1) * tile_elems, a.src + r0 * K, (uint32_t)(nrows * K * 4),
+                          &s_bar[cb ^ 1]);
+            }
+        }
+        const int64_t r0 = tile * R;
+        const int nrows = (int)imin<int64_t>(R, a.rows - r0);
+        const int n_el = (int)(nrows * K);
+        if (kProx) {
+            for (int i = tid; i <= nrows; i += kCThreads) s_rp[i] = a.in_row_ptr[r0 + i];
+            for (int i = tid; i < n_el; i += kCThreads) wt[i] = 0.f;
+            __syncthreads();
+            const int32_t s0 = s_rp[0], s1 = s_rp[nrows];
+            for (int32_t k = s0 + tid; k < s1; k += kCThreads) {
+                int lo = 0, hi = nrows - 1;  // row of entry k: last row whose start is <= k
+                while (lo < hi) {
+                    const int mid = (lo + hi + 1) >> 1;
+                    if (s_rp[mid] <= k) lo = mid; else hi = mid - 1;
+                }
+                wt[(int64_t)lo * K + __ldg(a.in_col + k)] = __ldg(a.in_val + k);
+            }
+        }
+        const bool landed = row_mbar_wait(&s_bar[cb], (phases >> cb) & 1u);
+        phases ^= 1u << cb;
+        if (!landed) s_fail = 1;
+        __syncthreads();
+        const float *g = gbuf0 + cb * tile_elems;
+
+        // pass 1: kept entries per warp segment
+        const int seg = ((n_el + 8 * 32 - 1) / (8 * 32)) * 32;   // multiple of 32
+        const int e_beg = imin(warp * seg, n_el), e_end = imin(e_beg + seg, n_el);
+        uint32_t cnt = 0;
+        for (int b = e_beg; b < e_end; b += 32) {
+            const int e = b + lane;
+            bool k = false;
+            if (e < e_end) {
+                if (kProx) {
+                    const float z = __fsub_rn(wt[e], __fmul_rn(a.eta, g[e]));
+                    k = fabsf(z) > a.thr;
+                    nonfinite |= isnan(z);
+                } else {
+                    k = g[e] != 0.f;
+                }
+            }
+            cnt += __popc(__ballot_sync(0xffffffffu, k));
+        }
+        if (lane == 0) s_wtot[warp] = cnt;
+        __syncthreads();
+        uint32_t wprefix = 0, tile_count = 0;
+#pragma unroll
+        for (int w = 0; w < kCThreads / 32; ++w) {
+            const uint32_t t = s_wtot[w];
+            if (w < warp) wprefix += t;
+            tile_count += t;
+        }
+        if (warp == 0) {
+            const unsigned long long prefix = lookback_warp(a.status, tile, tile_count, a.hdr);
+            if (lane == 0) s_excl = prefix;
+        }
+        __syncthreads();
+        const int64_t cap = a.capacity;
+        int64_t pos = (int64_t)s_excl + wprefix;
+
+        // pass 2: write the kept entries of this warp's segment, and the row starts
+        int64_t row = r0 + e_beg / K;
+        int64_t col = e_beg % K + lane;
+        while (col >= K) { col -= K; ++row; }
+        const unsigned lt = (1u << lane) - 1u;
+        for (int b = e_beg; b < e_end; b += 32) {
+            const int e = b + lane;
+            bool k = false;
+            float v = 0.f;
+            if (e < e_end) {
+                if (kProx) {
+                    const float z = __fsub_rn(wt[e], __fmul_rn(a.eta, g[e]));
+                    k = fabsf(z) > a.thr;
+                    v = z > 0.f ? __fsub_rn(z, a.thr) : __fadd_rn(z, a.thr);
+                } else {
+                    v = g[e];
+                    k = v != 0.f;
+                }
+            }
+            const unsigned m = __ballot_sync(0xffffffffu, k);
+            const int64_t p = pos + __popc(m & lt);
+            if (e < e_end && col == 0) a.out_row_ptr[row] = (int32_t)imin<int64_t>(p, cap);
+            if (k && p < cap) {
+                a.out_col[p] = (int32_t)col;
+                a.out_val[p] = v;
+            }
+            pos += __popc(m);
+            col += 32;
+            while (col >= K) { col -= K; ++row; }
+        }
+        if (tile == a.num_tiles - 1 && tid == 0) {
+            const int64_t total = (int64_t)s_excl + tile_count;
+            a.out_row_ptr[a.rows] = (int32_t)imin<int64_t>(total, cap);
+            if (total > cap) {
+                dev_flag(a.hdr, CSRT_DEV_CAPACITY);
+                atomicMax(&a.hdr->required, (unsigned long long)total);
+            }
+        }
+        __syncthreads();   // buffers of this tile are free from here on
+        cb ^= 1;
+    }
+    if (kProx && __syncthreads_or(nonfinite) && tid == 0) dev_flag(a.hdr, CSRT_DEV_NONFINITE);
+    if (tid == 0 && s_fail) {
+        dev_flag(a.hdr, CSRT_DEV_TIMEOUT);
+        a.hdr->timeout_site = 3;
+    }
+}
+
 static int compact_launch(bool prox, const float *src, int32_t rows, int32_t cols, const csrt_csr *in,
                           float eta, float thr, csrt_csr *out, void *ws, size_t ws_bytes,
                           cudaStream_t s) {
@@ -264,7 +481,9 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
         CSRT_CHECK_CUDA(cudaMemsetAsync(out->row_ptr, 0, sizeof(int32_t) * ((size_t)rows + 1), s));
         return CSRT_OK;
     }
-    const int64_t tiles = ceil_div<int64_t>(elems, kTile);
+    const bool row_path = cols % 4 == 0 && cols <= kRowMaxK && (reinterpret_cast<uintptr_t>(src) & 15) == 0;
+    const int32_t rows_per_tile = row_path ? imax<int32_t>(1, kRowBudget / cols) : 0;
+    const int64_t tiles = row_path ? ceil_div<int64_t>(rows, rows_per_tile) : ceil_div<int64_t>(elems, kTile);
     CSRT_ARG(ws_bytes >= kWsHeaderBytes + compact_scratch_bytes(elems), "workspace too small for compaction");
     WsHeader *hdr = static_cast<WsHeader *>(ws);
     unsigned long long *status = reinterpret_cast<unsigned long long *>(ws_scratch(ws));
@@ -287,6 +506,29 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
     a.hdr = hdr;
     a.status = status;
     a.num_tiles = tiles;
+    if (row_path) {
+        const int32_t tile_elems = rows_per_tile * cols;
+        const size_t smem = (size_t)(prox ? 3 : 2) * tile_elems * sizeof(float) +
+                            (prox ? ((size_t)rows_per_tile + 1) * sizeof(int32_t) : 0);
+        static bool attr_done[2][64] = {{false}};
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (dev >= 0 && dev < 64 && !attr_done[prox][dev]) {
+            const int max_smem = (int)(3 * (size_t)kRowMaxK * sizeof(float) + (kRowBudget + 2) * sizeof(int32_t));
+            if (prox)
+                CSRT_CHECK_CUDA(cudaFuncSetAttribute(compact_rows_kernel<true>,
+                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
+            else
+                CSRT_CHECK_CUDA(cudaFuncSetAttribute(compact_rows_kernel<false>,
+                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
+            attr_done[prox][dev] = true;
+        }
+        const unsigned grid = (unsigned)imin<int64_t>(tiles, 2 * (int64_t)num_sms());
+        if (prox) compact_rows_kernel<true><<<grid, kCThreads, smem, s>>>(a, rows_per_tile, tile_elems);
+        else compact_rows_kernel<false><<<grid, kCThreads, smem, s>>>(a, rows_per_tile, tile_elems);
+        count_launch();
+        return check_launch("compact_rows_kernel");
+    }
     const bool vec = (reinterpret_cast<uintptr_t>(src) & 15) == 0;
     dim3 grid((unsigned)tiles), block(kCThreads);
     if (prox) {

@@ -264,6 +264,10 @@ def test_prox_hand_cases_on_gpu(C):
     (100, 300, 0.09, 1.0, 0.0, 1e-4),
     (64, 64, 0.0, 0.0, 0.1, 0.0),
     (500, 800, 0.08, 1e-2, 0.01, 1e-2),
+    (1001, 784, 0.1, 1.0, 0.01, 1e-2),
+    (333, 64, 0.4, 1.0, 0.1, 1.0),
+    (3, 16384, 0.02, 1.0, 0.01, 0.5),
+    (2, 16388, 0.02, 1.0, 0.01, 0.5),
 ])
 def test_prox_bit_exact(C, m, k, density, gscale, eta, lam):
     rng = np.random.default_rng(m + k)
