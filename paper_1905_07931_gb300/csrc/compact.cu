@@ -276,201 +276,163 @@ __global__ void __launch_bounds__(kCThreads) compact_kernel(CompactArgs a) {
 // Row-tile compaction (the fast path: K % 4 == 0, K <= kRowMaxK, G 16-byte
 // aligned). A tile is R whole rows (R*K <= max(K, kRowBudget) entries), so the
 // old CSR entries of a tile are the contiguous range row_ptr[r0] ..
-// row_ptr[r0+R) and no search is needed. The grid is persistent (two blocks
-// per SM); each block takes tiles by ticket and, while it works on one tile,
-// its next tile's slice of G is already streaming into shared memory with a
-// bulk asynchronous copy (cp.async.bulk, completion on an mbarrier). Each warp
-// compacts a contiguous segment of the tile 32 entries at a time with ballots,
-// so kept entries leave as coalesced runs.
+// row_ptr[r0+R) and no search is needed: they are scattered into a
+// shared-memory copy of the tile's old weights. Each of the 8 warps owns a
+// contiguous segment of the tile and walks it 128 entries (one float4 per
+// lane) at a time: pass 1 counts the kept entries with four ballots per step,
+// the block learns its global offset by decoupled look-back, pass 2
+// re-evaluates the entries (G comes back from L1/L2) and writes them at ranks
+// taken from the same ballots, so a warp's output of one step is one
+// contiguous run. Positions are 32-bit (nnz < 2^31). Small per-block state
+// (the old-weight tile only) lets several blocks share an SM and hide the
+// look-back latency.
 // ---------------------------------------------------------------------------
 constexpr int kRowBudget = 8192;     // entries per tile when rows are short
 constexpr int kRowMaxK = 16384;      // longest row the row-tile path takes
-constexpr unsigned kRowWaitLimit = 1u << 22;
 
-__device__ __forceinline__ uint32_t cvta_smem(const void *p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
+struct Keep4 {
+    bool k[4];
+    float v[4];
+};
 
-__device__ __forceinline__ bool row_mbar_wait(uint64_t *bar, uint32_t parity) {
-    const uint32_t addr = cvta_smem(bar);
-    for (unsigned i = 0; i < kRowWaitLimit; ++i) {
-        uint32_t done;
-        asm volatile(
-            "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-            " selp.u32 %0, 1, 0, p;\n}\n"
-            : "=r"(done)
-            : "r"(addr), "r"(parity)
-            : "memory");
-        if (done) return true;
-        if (i > 32) __nanosleep(32);
+template <bool kProx>
+__device__ __forceinline__ Keep4 eval4(const float4 g, const float4 w, float eta, float thr) {
+    Keep4 r;
+    const float gv[4] = {g.x, g.y, g.z, g.w};
+    const float wv[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        if (kProx) {
+            const float z = __fsub_rn(wv[j], __fmul_rn(eta, gv[j]));
+            r.k[j] = fabsf(z) > thr;
+            r.v[j] = z > 0.f ? __fsub_rn(z, thr) : __fadd_rn(z, thr);
+        } else {
+            r.k[j] = gv[j] != 0.f;
+            r.v[j] = gv[j];
+        }
     }
-    return false;
-}
-
-// Thread 0 only: stream `bytes` of G (16-byte aligned, multiple of 16) into smem.
-__device__ __forceinline__ void bulk_load(float *dst, const float *src, uint32_t bytes, uint64_t *bar) {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(cvta_smem(bar)), "r"(bytes)
-                 : "memory");
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-            cvta_smem(dst)),
-        "l"(src), "r"(bytes), "r"(cvta_smem(bar))
-        : "memory");
+    return r;
 }
 
 template <bool kProx>
-__global__ void __launch_bounds__(kCThreads, 2) compact_rows_kernel(CompactArgs a, int32_t rows_per_tile,
-                                                                     int32_t tile_elems) {
-    extern __shared__ __align__(128) float row_smem[];
-    float *const gbuf0 = row_smem;   // G of the current / next tile: gbuf0 + cb * tile_elems
-    float *wt = row_smem + 2 * tile_elems;                                     // old weights (prox)
-    int32_t *s_rp = reinterpret_cast<int32_t *>(wt + (kProx ? tile_elems : 0));  // rows_per_tile + 1
-    __shared__ __align__(8) uint64_t s_bar[2];
-    __shared__ unsigned int s_ticket[2];
+__global__ void __launch_bounds__(kCThreads, 4) compact_rows_kernel(CompactArgs a, int32_t rows_per_tile) {
+    extern __shared__ __align__(16) float row_smem[];
+    float *wt = row_smem;                                                        // old weights (prox)
+    int32_t *s_rp = reinterpret_cast<int32_t *>(row_smem + (kProx ? rows_per_tile * a.cols : 0));
     __shared__ uint32_t s_wtot[kCThreads / 32];
-    __shared__ unsigned long long s_excl;
-    __shared__ int s_fail;
+    __shared__ uint32_t s_excl;
+    __shared__ unsigned int s_tile;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int64_t K = a.cols;
-    const int R = rows_per_tile;
-    if (tid == 0) {
-        s_fail = 0;
-        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(cvta_smem(&s_bar[0])) : "memory");
-        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(cvta_smem(&s_bar[1])) : "memory");
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        const unsigned t = atomicAdd(&a.hdr->ticket, 1u);
-        s_ticket[0] = t;
-        if (t < a.num_tiles) {
-            const int64_t r0 = (int64_t)t * R;
-            const int64_t nrows = imin<int64_t>(R, a.rows - r0);
-            bulk_load(gbuf0, a.src + r0 * K, (uint32_t)(nrows * K * 4), &s_bar[0]);
+    const int K = a.cols;
+    if (tid == 0) s_tile = atomicAdd(&a.hdr->ticket, 1u);
+    __syncthreads();
+    const int64_t tile = s_tile;
+    if (tile >= a.num_tiles) return;   // cannot happen: one block per tile
+    const int r0 = (int)(tile * rows_per_tile);
+    const int nrows = imin(rows_per_tile, a.rows - r0);
+    const int n_el = nrows * K;
+    const float *g = a.src + (int64_t)r0 * K;
+    bool nonfinite = false;
+
+    if (kProx) {
+        for (int i = tid; i <= nrows; i += kCThreads) s_rp[i] = a.in_row_ptr[r0 + i];
+        float4 *w4 = reinterpret_cast<float4 *>(wt);
+        for (int i = tid; i < n_el / 4; i += kCThreads) w4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        __syncthreads();
+        const int32_t s0 = s_rp[0], s1 = s_rp[nrows];
+        for (int32_t k = s0 + tid; k < s1; k += kCThreads) {
+            int lo = 0, hi = nrows - 1;  // row of entry k: last row whose start is <= k
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (s_rp[mid] <= k) lo = mid; else hi = mid - 1;
+            }
+            wt[lo * K + __ldg(a.in_col + k)] = __ldg(a.in_val + k);
         }
+        __syncthreads();
+    }
+
+    // warp segment [e_beg, e_end), a multiple of 128 entries except at the end
+    const int seg = ((n_el + 8 * 128 - 1) / (8 * 128)) * 128;
+    const int e_beg = imin(warp * seg, n_el), e_end = imin(e_beg + seg, n_el);
+
+    // pass 1: count
+    uint32_t cnt = 0;
+    for (int b = e_beg + 4 * lane; b - 4 * lane < e_end; b += 128) {
+        const bool in = b < e_end;
+        float4 gv = make_float4(0.f, 0.f, 0.f, 0.f), wv = gv;
+        if (in) {
+            gv = ldg_f4(g + b);
+            if (kProx) wv = *reinterpret_cast<const float4 *>(wt + b);
+        }
+        const Keep4 r = eval4<kProx>(gv, wv, a.eta, a.thr);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            cnt += __popc(__ballot_sync(0xffffffffu, in && r.k[j]));
+            if (kProx) nonfinite |= in && isnan(r.v[j]);
+        }
+    }
+    if (lane == 0) s_wtot[warp] = cnt;
+    __syncthreads();
+    uint32_t pos = 0, tile_count = 0;
+#pragma unroll
+    for (int w = 0; w < kCThreads / 32; ++w) {
+        const uint32_t t = s_wtot[w];
+        if (w < warp) pos += t;
+        tile_count += t;
+    }
+    if (warp == 0) {
+        const unsigned long long prefix = lookback_warp(a.status, tile, tile_count, a.hdr);
+        if (lane == 0) s_excl = (uint32_t)prefix;
     }
     __syncthreads();
-    uint32_t phases = 0;   // bit b: parity of the next completion of s_bar[b]
-    int cb = 0;
-    bool nonfinite = false;
-    for (;;) {
-        const int64_t tile = s_ticket[cb];
-        if (tile >= a.num_tiles) break;
-        // prefetch the next tile into the other buffer (its last reader finished
-        // before the trailing barrier of the previous iteration)
-        if (tid == 0) {
-            const unsigned t = atomicAdd(&a.hdr->ticket, 1u);
-            s_ticket[cb ^ 1] = t;
-            if (t < a.num_tiles) {
-                const int64_t r0 = (int64_t)t * R;
-                const int64_t nrows = imin<int64_t>(R, a.rows - r0);
-                bulk_load(gbuf0 + (cb ^ 1) * tile_elems, a.src + r0 * K, (uint32_t)(nrows * K * 4),
-                          &s_bar[cb ^ 1]);
-            }
-        }
-        const int64_t r0 = tile * R;
-        const int nrows = (int)imin<int64_t>(R, a.rows - r0);
-        const int n_el = (int)(nrows * K);
-        if (kProx) {
-            for (int i = tid; i <= nrows; i += kCThreads) s_rp[i] = a.in_row_ptr[r0 + i];
-            for (int i = tid; i < n_el; i += kCThreads) wt[i] = 0.f;
-            __syncthreads();
-            const int32_t s0 = s_rp[0], s1 = s_rp[nrows];
-            for (int32_t k = s0 + tid; k < s1; k += kCThreads) {
-                int lo = 0, hi = nrows - 1;  // row of entry k: last row whose start is <= k
-                while (lo < hi) {
-                    const int mid = (lo + hi + 1) >> 1;
-                    if (s_rp[mid] <= k) lo = mid; else hi = mid - 1;
-                }
-                wt[(int64_t)lo * K + __ldg(a.in_col + k)] = __ldg(a.in_val + k);
-            }
-        }
-        const bool landed = row_mbar_wait(&s_bar[cb], (phases >> cb) & 1u);
-        phases ^= 1u << cb;
-        if (!landed) s_fail = 1;
-        __syncthreads();
-        const float *g = gbuf0 + cb * tile_elems;
+    pos += s_excl;
+    const uint32_t cap = (uint32_t)imin<int64_t>(a.capacity, 0x7fffffff);
 
-        // pass 1: kept entries per warp segment
-        const int seg = ((n_el + 8 * 32 - 1) / (8 * 32)) * 32;   // multiple of 32
-        const int e_beg = imin(warp * seg, n_el), e_end = imin(e_beg + seg, n_el);
-        uint32_t cnt = 0;
-        for (int b = e_beg; b < e_end; b += 32) {
-            const int e = b + lane;
-            bool k = false;
-            if (e < e_end) {
-                if (kProx) {
-                    const float z = __fsub_rn(wt[e], __fmul_rn(a.eta, g[e]));
-                    k = fabsf(z) > a.thr;
-                    nonfinite |= isnan(z);
-                } else {
-                    k = g[e] != 0.f;
-                }
-            }
-            cnt += __popc(__ballot_sync(0xffffffffu, k));
+    // pass 2: write the kept entries and the row starts
+    int row = e_beg / K;
+    int col = e_beg - row * K + 4 * lane;
+    while (col >= K) { col -= K; ++row; }
+    const unsigned lt = (1u << lane) - 1u;
+    for (int b = e_beg + 4 * lane; b - 4 * lane < e_end; b += 128) {
+        const bool in = b < e_end;
+        float4 gv = make_float4(0.f, 0.f, 0.f, 0.f), wv = gv;
+        if (in) {
+            gv = ldg_f4(g + b);
+            if (kProx) wv = *reinterpret_cast<const float4 *>(wt + b);
         }
-        if (lane == 0) s_wtot[warp] = cnt;
-        __syncthreads();
-        uint32_t wprefix = 0, tile_count = 0;
+        const Keep4 r = eval4<kProx>(gv, wv, a.eta, a.thr);
+        uint32_t p = pos, step = 0;
 #pragma unroll
-        for (int w = 0; w < kCThreads / 32; ++w) {
-            const uint32_t t = s_wtot[w];
-            if (w < warp) wprefix += t;
-            tile_count += t;
+        for (int j = 0; j < 4; ++j) {
+            const unsigned m = __ballot_sync(0xffffffffu, in && r.k[j]);
+            p += __popc(m & lt);
+            step += __popc(m);
         }
-        if (warp == 0) {
-            const unsigned long long prefix = lookback_warp(a.status, tile, tile_count, a.hdr);
-            if (lane == 0) s_excl = prefix;
-        }
-        __syncthreads();
-        const int64_t cap = a.capacity;
-        int64_t pos = (int64_t)s_excl + wprefix;
-
-        // pass 2: write the kept entries of this warp's segment, and the row starts
-        int64_t row = r0 + e_beg / K;
-        int64_t col = e_beg % K + lane;
-        while (col >= K) { col -= K; ++row; }
-        const unsigned lt = (1u << lane) - 1u;
-        for (int b = e_beg; b < e_end; b += 32) {
-            const int e = b + lane;
-            bool k = false;
-            float v = 0.f;
-            if (e < e_end) {
-                if (kProx) {
-                    const float z = __fsub_rn(wt[e], __fmul_rn(a.eta, g[e]));
-                    k = fabsf(z) > a.thr;
-                    v = z > 0.f ? __fsub_rn(z, a.thr) : __fadd_rn(z, a.thr);
-                } else {
-                    v = g[e];
-                    k = v != 0.f;
+        if (in && col == 0) a.out_row_ptr[r0 + row] = (int32_t)min(p, cap);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (in && r.k[j]) {
+                if (p < cap) {
+                    a.out_col[p] = col + j;
+                    a.out_val[p] = r.v[j];
                 }
-            }
-            const unsigned m = __ballot_sync(0xffffffffu, k);
-            const int64_t p = pos + __popc(m & lt);
-            if (e < e_end && col == 0) a.out_row_ptr[row] = (int32_t)imin<int64_t>(p, cap);
-            if (k && p < cap) {
-                a.out_col[p] = (int32_t)col;
-                a.out_val[p] = v;
-            }
-            pos += __popc(m);
-            col += 32;
-            while (col >= K) { col -= K; ++row; }
-        }
-        if (tile == a.num_tiles - 1 && tid == 0) {
-            const int64_t total = (int64_t)s_excl + tile_count;
-            a.out_row_ptr[a.rows] = (int32_t)imin<int64_t>(total, cap);
-            if (total > cap) {
-                dev_flag(a.hdr, CSRT_DEV_CAPACITY);
-                atomicMax(&a.hdr->required, (unsigned long long)total);
+                ++p;
             }
         }
-        __syncthreads();   // buffers of this tile are free from here on
-        cb ^= 1;
+        pos += step;
+        col += 128;
+        while (col >= K) { col -= K; ++row; }
+    }
+    if (tile == a.num_tiles - 1 && tid == 0) {
+        const int64_t total = (int64_t)s_excl + tile_count;
+        a.out_row_ptr[a.rows] = (int32_t)imin<int64_t>(total, cap);
+        if (total > (int64_t)cap) {
+            dev_flag(a.hdr, CSRT_DEV_CAPACITY);
+            atomicMax(&a.hdr->required, (unsigned long long)total);
+        }
     }
     if (kProx && __syncthreads_or(nonfinite) && tid == 0) dev_flag(a.hdr, CSRT_DEV_NONFINITE);
-    if (tid == 0 && s_fail) {
-        dev_flag(a.hdr, CSRT_DEV_TIMEOUT);
-        a.hdr->timeout_site = 3;
-    }
 }
 
 static int compact_launch(bool prox, const float *src, int32_t rows, int32_t cols, const csrt_csr *in,
@@ -507,25 +469,18 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
     a.status = status;
     a.num_tiles = tiles;
     if (row_path) {
-        const int32_t tile_elems = rows_per_tile * cols;
-        const size_t smem = (size_t)(prox ? 3 : 2) * tile_elems * sizeof(float) +
-                            (prox ? ((size_t)rows_per_tile + 1) * sizeof(int32_t) : 0);
-        static bool attr_done[2][64] = {{false}};
+        const size_t smem = prox ? ((size_t)rows_per_tile * cols + rows_per_tile + 1) * sizeof(float) : 0;
+        static bool attr_done[64] = {false};
         int dev = 0;
         cudaGetDevice(&dev);
-        if (dev >= 0 && dev < 64 && !attr_done[prox][dev]) {
-            const int max_smem = (int)(3 * (size_t)kRowMaxK * sizeof(float) + (kRowBudget + 2) * sizeof(int32_t));
-            if (prox)
-                CSRT_CHECK_CUDA(cudaFuncSetAttribute(compact_rows_kernel<true>,
-                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
-            else
-                CSRT_CHECK_CUDA(cudaFuncSetAttribute(compact_rows_kernel<false>,
-                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
-            attr_done[prox][dev] = true;
+        if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+            const int max_smem = (int)((size_t)(kRowMaxK + kRowBudget + 1) * sizeof(float));
+            CSRT_CHECK_CUDA(cudaFuncSetAttribute(compact_rows_kernel<true>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
+            attr_done[dev] = true;
         }
-        const unsigned grid = (unsigned)imin<int64_t>(tiles, 2 * (int64_t)num_sms());
-        if (prox) compact_rows_kernel<true><<<grid, kCThreads, smem, s>>>(a, rows_per_tile, tile_elems);
-        else compact_rows_kernel<false><<<grid, kCThreads, smem, s>>>(a, rows_per_tile, tile_elems);
+        if (prox) compact_rows_kernel<true><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile);
+        else compact_rows_kernel<false><<<(unsigned)tiles, kCThreads, 0, s>>>(a, rows_per_tile);
         count_launch();
         return check_launch("compact_rows_kernel");
     }
