@@ -356,20 +356,26 @@ __global__ void __launch_bounds__(kCThreads, 4) compact_rows_kernel(CompactArgs 
     const int seg = ((n_el + 8 * 128 - 1) / (8 * 128)) * 128;
     const int e_beg = imin(warp * seg, n_el), e_end = imin(e_beg + seg, n_el);
 
-    // pass 1: count
+    // pass 1: count; four steps of loads in flight per lane
     uint32_t cnt = 0;
-    for (int b = e_beg + 4 * lane; b - 4 * lane < e_end; b += 128) {
-        const bool in = b < e_end;
-        float4 gv = make_float4(0.f, 0.f, 0.f, 0.f), wv = gv;
-        if (in) {
-            gv = ldg_f4(g + b);
-            if (kProx) wv = *reinterpret_cast<const float4 *>(wt + b);
-        }
-        const Keep4 r = eval4<kProx>(gv, wv, a.eta, a.thr);
+    for (int base = e_beg; base < e_end; base += 4 * 128) {
+        float4 gv[4], wv[4];
+        bool in[4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            cnt += __popc(__ballot_sync(0xffffffffu, in && r.k[j]));
-            if (kProx) nonfinite |= in && isnan(r.v[j]);
+        for (int u = 0; u < 4; ++u) {
+            const int b = base + 128 * u + 4 * lane;
+            in[u] = b < e_end;
+            gv[u] = in[u] ? ldg_f4(g + b) : make_float4(0.f, 0.f, 0.f, 0.f);
+            wv[u] = (kProx && in[u]) ? *reinterpret_cast<const float4 *>(wt + b) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const Keep4 r = eval4<kProx>(gv[u], wv[u], a.eta, a.thr);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                cnt += __popc(__ballot_sync(0xffffffffu, in[u] && r.k[j]));
+                if (kProx) nonfinite |= in[u] && isnan(r.v[j]);
+            }
         }
     }
     if (lane == 0) s_wtot[warp] = cnt;
@@ -394,35 +400,41 @@ __global__ void __launch_bounds__(kCThreads, 4) compact_rows_kernel(CompactArgs 
     int col = e_beg - row * K + 4 * lane;
     while (col >= K) { col -= K; ++row; }
     const unsigned lt = (1u << lane) - 1u;
-    for (int b = e_beg + 4 * lane; b - 4 * lane < e_end; b += 128) {
-        const bool in = b < e_end;
-        float4 gv = make_float4(0.f, 0.f, 0.f, 0.f), wv = gv;
-        if (in) {
-            gv = ldg_f4(g + b);
-            if (kProx) wv = *reinterpret_cast<const float4 *>(wt + b);
-        }
-        const Keep4 r = eval4<kProx>(gv, wv, a.eta, a.thr);
-        uint32_t p = pos, step = 0;
+    for (int base = e_beg; base < e_end; base += 4 * 128) {
+        float4 gv[4], wv[4];
+        bool in[4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const unsigned m = __ballot_sync(0xffffffffu, in && r.k[j]);
-            p += __popc(m & lt);
-            step += __popc(m);
+        for (int u = 0; u < 4; ++u) {
+            const int b = base + 128 * u + 4 * lane;
+            in[u] = b < e_end;
+            gv[u] = in[u] ? ldg_f4(g + b) : make_float4(0.f, 0.f, 0.f, 0.f);
+            wv[u] = (kProx && in[u]) ? *reinterpret_cast<const float4 *>(wt + b) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        if (in && col == 0) a.out_row_ptr[r0 + row] = (int32_t)min(p, cap);
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            if (in && r.k[j]) {
-                if (p < cap) {
-                    a.out_col[p] = col + j;
-                    a.out_val[p] = r.v[j];
-                }
-                ++p;
+        for (int u = 0; u < 4; ++u) {
+            const Keep4 r = eval4<kProx>(gv[u], wv[u], a.eta, a.thr);
+            uint32_t p = pos, step = 0;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const unsigned m = __ballot_sync(0xffffffffu, in[u] && r.k[j]);
+                p += __popc(m & lt);
+                step += __popc(m);
             }
+            if (in[u] && col == 0) a.out_row_ptr[r0 + row] = (int32_t)min(p, cap);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                if (in[u] && r.k[j]) {
+                    if (p < cap) {
+                        a.out_col[p] = col + j;
+                        a.out_val[p] = r.v[j];
+                    }
+                    ++p;
+                }
+            }
+            pos += step;
+            col += 128;
+            while (col >= K) { col -= K; ++row; }
         }
-        pos += step;
-        col += 128;
-        while (col >= K) { col -= K; ++row; }
     }
     if (tile == a.num_tiles - 1 && tid == 0) {
         const int64_t total = (int64_t)s_excl + tile_count;
@@ -593,24 +605,34 @@ __global__ void __launch_bounds__(1024) scan_single_block_kernel(const int32_t *
     if (tid == 0) out[n] = total;
 }
 
+// Write kernel: one block per (32-row block, 256-column chunk). Phase A
+// gathers the block's entries into a shared 32 x 256 value tile and the row
+// bitmask of each column; phase B walks the columns one warp each, lane = row,
+// so each column's run of entries leaves as one coalesced store; phase C
+// writes t_pos in CSR order.
+constexpr int kTwCols = 256;
+
 __global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict__ row_ptr,
                                                        const int32_t *__restrict__ col,
                                                        const float *__restrict__ val, int32_t rows,
                                                        int32_t cols, const int32_t *__restrict__ off,
                                                        const int32_t *__restrict__ t_row_ptr,
                                                        int32_t *__restrict__ t_col, float *__restrict__ t_val,
-                                                       int32_t *__restrict__ t_pos, int64_t capacity,
-                                                       int32_t chunk) {
-    __shared__ unsigned int bits[kTrChunk];
-    __shared__ int32_t base[kTrChunk];   // first position of this block's run in each column
-    const int b = blockIdx.x, c0 = blockIdx.y * chunk;
-    const int cw = min(chunk, cols - c0);
+                                                       int32_t *__restrict__ t_pos, int64_t capacity) {
+    __shared__ unsigned int bits[kTwCols];
+    __shared__ int32_t base[kTwCols];            // first position of this block's run in each column
+    __shared__ float vt[kTrRows][kTwCols + 1];   // values of the block's entries, padded
+    const int b = blockIdx.x, c0 = blockIdx.y * kTwCols;
+    const int cw = min(kTwCols, cols - c0);
     const bool chunked = gridDim.y > 1;
-    const int32_t *boff = off + (int64_t)b * cols + c0;
-    for (int j = threadIdx.x; j < cw; j += blockDim.x) base[j] = t_row_ptr[c0 + j] + boff[j];
-    tr_build_bits(bits, row_ptr, col, rows, b, c0, cw, chunked);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int rr = warp; rr < kTrRows; rr += blockDim.x / 32) {
+    for (int j = threadIdx.x; j < cw; j += blockDim.x) {
+        bits[j] = 0u;
+        base[j] = t_row_ptr[c0 + j] + off[(int64_t)b * cols + c0 + j];
+    }
+    __syncthreads();
+    // phase A
+    for (int rr = warp; rr < kTrRows; rr += 8) {
         const int r = b * kTrRows + rr;
         if (r >= rows) break;
         int64_t s = row_ptr[r], e = row_ptr[r + 1];
@@ -618,15 +640,40 @@ __global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict
             s = warp_lower_bound(col, s, e, c0);
             e = warp_lower_bound(col, s, e, c0 + cw);
         }
-        const unsigned int below = (1u << rr) - 1u;
         for (int64_t k = s + lane; k < e; k += 32) {
             const int j = __ldg(col + k) - c0;
-            const int64_t p = (int64_t)base[j] + __popc(bits[j] & below);
+            atomicOr(&bits[j], 1u << rr);
+            vt[rr][j] = __ldg(val + k);
+        }
+    }
+    __syncthreads();
+    // phase B: lane = row within the block
+    const int my_row = b * kTrRows + lane;
+    const unsigned below = (1u << lane) - 1u;
+    for (int j = warp; j < cw; j += 8) {
+        const unsigned m = bits[j];
+        if ((m >> lane) & 1u) {
+            const int64_t p = (int64_t)base[j] + __popc(m & below);
             if (p < capacity) {
-                t_col[p] = r;
-                t_val[p] = __ldg(val + k);
-                t_pos[k] = (int32_t)p;
+                t_col[p] = my_row;
+                t_val[p] = vt[lane][j];
             }
+        }
+    }
+    // phase C: t_pos in CSR order
+    for (int rr = warp; rr < kTrRows; rr += 8) {
+        const int r = b * kTrRows + rr;
+        if (r >= rows) break;
+        int64_t s = row_ptr[r], e = row_ptr[r + 1];
+        if (chunked) {
+            s = warp_lower_bound(col, s, e, c0);
+            e = warp_lower_bound(col, s, e, c0 + cw);
+        }
+        const unsigned below_rr = (1u << rr) - 1u;
+        for (int64_t k = s + lane; k < e; k += 32) {
+            const int j = __ldg(col + k) - c0;
+            const int64_t p = (int64_t)base[j] + __popc(bits[j] & below_rr);
+            if (p < capacity) t_pos[k] = (int32_t)p;
         }
     }
 }
@@ -652,9 +699,9 @@ int transpose_impl(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s) {
     tr_count_kernel<<<dim3(nb, nc), 256, 0, s>>>(w->row_ptr, w->col_idx, rows, cols, chunk, cnt);
     tr_colscan_kernel<<<ceil_div(cols, 32), 256, 0, s>>>(cnt, nb, cols, coltot);
     scan_single_block_kernel<<<1, 1024, 0, s>>>(coltot, cols, w->t_row_ptr);
-    tr_write_kernel<<<dim3(nb, nc), 256, 0, s>>>(w->row_ptr, w->col_idx, w->val, rows, cols, cnt,
-                                                 w->t_row_ptr, w->t_col_idx, w->t_val, w->t_pos,
-                                                 w->capacity, chunk);
+    tr_write_kernel<<<dim3(nb, (unsigned)ceil_div<int64_t>(cols, kTwCols)), 256, 0, s>>>(
+        w->row_ptr, w->col_idx, w->val, rows, cols, cnt, w->t_row_ptr, w->t_col_idx, w->t_val, w->t_pos,
+        w->capacity);
     count_launch(4);
     return check_launch("csr_transpose kernels");
 }
