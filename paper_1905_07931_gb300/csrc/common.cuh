@@ -59,7 +59,7 @@ inline cudaStream_t as_stream(void *s) { return static_cast<cudaStream_t>(s); }
 // ---------------------------------------------------------------------------
 // Workspace sizes of the individual operations (bytes after the header).
 // ---------------------------------------------------------------------------
-size_t compact_scratch_bytes(int64_t elems);
+size_t compact_scratch_bytes(int32_t rows, int32_t cols);
 size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
 size_t spmm_scratch_bytes(int32_t max_n);
 size_t sddmm_scratch_bytes(int64_t capacity, int32_t max_n);

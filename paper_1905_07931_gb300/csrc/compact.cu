@@ -34,8 +34,22 @@ constexpr int kTile = kCThreads * kCQuads * 4;       // 4096 entries per tile
 constexpr unsigned long long kFlagAgg = 1ull << 32;  // tile aggregate published
 constexpr unsigned long long kFlagInc = 2ull << 32;  // inclusive prefix published
 
-size_t compact_scratch_bytes(int64_t elems) {
-    return (size_t)ceil_div<int64_t>(elems, kTile) * sizeof(unsigned long long);
+// Look-back status words: one per tile; flat tiles (4096 entries) are the
+// smallest, so their count bounds every path.
+static size_t status_bytes(int64_t elems) {
+    return ((size_t)ceil_div<int64_t>(elems, kTile) * sizeof(unsigned long long) + 255) / 256 * 256;
+}
+// Keep-bitmask and word positions emitted by the prox kernel for the transposed copy.
+static size_t bits_bytes(int32_t rows, int32_t cols) {
+    return ((size_t)rows * (size_t)ceil_div<int32_t>(cols, 32) * sizeof(uint32_t) + 255) / 256 * 256;
+}
+
+size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
+
+// Scratch of csr_from_dense / prox_update_compact / csr_transpose.
+size_t compact_scratch_bytes(int32_t rows, int32_t cols) {
+    const int64_t elems = (int64_t)rows * cols;
+    return status_bytes(elems) + 2 * bits_bytes(rows, cols) + transpose_scratch_bytes(rows, cols);
 }
 
 struct CompactArgs {
@@ -447,9 +461,182 @@ __global__ void __launch_bounds__(kCThreads, 4) compact_rows_kernel(CompactArgs 
     if (kProx && __syncthreads_or(nonfinite) && tid == 0) dev_flag(a.hdr, CSRT_DEV_NONFINITE);
 }
 
+
+// ---------------------------------------------------------------------------
+// Prox row-tile kernel (the prox update's fast path). Same tiling as
+// compact_rows_kernel, one read of G: pass 1 evaluates every entry once,
+// counts the kept ones per lane and parks each result in the shared old-weight
+// tile (the kept value, or NaN for a dropped entry: a kept value is never
+// NaN); pass 2 reads only shared memory. With kBits (K % 32 == 0 and a
+// transposed copy wanted) pass 2 also emits, per 32-entry word of a row, the
+// keep bitmask and the CSR position of the word's first entry, from which the
+// transposed copy is built without re-reading the CSR.
+// ---------------------------------------------------------------------------
+// bit t of x (t < 8) -> bit 4t
+__device__ __forceinline__ uint32_t spread8(uint32_t x) {
+    x &= 0xFFu;
+    x = (x | (x << 12)) & 0x000F000Fu;
+    x = (x | (x << 6)) & 0x03030303u;
+    x = (x | (x << 3)) & 0x11111111u;
+    return x;
+}
+
+template <bool kBits>
+__global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, int32_t rows_per_tile,
+                                                                  uint32_t *__restrict__ keepbits,
+                                                                  int32_t *__restrict__ wordpos, int32_t wpr) {
+    extern __shared__ __align__(16) float row_smem[];
+    float *wt = row_smem;
+    int32_t *s_rp = reinterpret_cast<int32_t *>(row_smem + rows_per_tile * a.cols);
+    __shared__ uint32_t s_wtot[kCThreads / 32];
+    __shared__ uint32_t s_excl;
+    __shared__ unsigned int s_tile;
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int K = a.cols;
+    if (tid == 0) s_tile = atomicAdd(&a.hdr->ticket, 1u);
+    __syncthreads();
+    const int64_t tile = s_tile;
+    if (tile >= a.num_tiles) return;
+    const int r0 = (int)(tile * rows_per_tile);
+    const int nrows = imin(rows_per_tile, a.rows - r0);
+    const int n_el = nrows * K;
+    const float *g = a.src + (int64_t)r0 * K;
+    const float eta = a.eta, thr = a.thr;
+
+    for (int i = tid; i <= nrows; i += kCThreads) s_rp[i] = a.in_row_ptr[r0 + i];
+    {
+        float4 *w4 = reinterpret_cast<float4 *>(wt);
+        for (int i = tid; i < n_el / 4; i += kCThreads) w4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    __syncthreads();
+    {
+        const int32_t s0 = s_rp[0], s1 = s_rp[nrows];
+        for (int32_t k = s0 + tid; k < s1; k += kCThreads) {
+            int lo = 0, hi = nrows - 1;
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (s_rp[mid] <= k) lo = mid; else hi = mid - 1;
+            }
+            wt[lo * K + __ldg(a.in_col + k)] = __ldg(a.in_val + k);
+        }
+    }
+    __syncthreads();
+
+    const int seg = ((n_el + 8 * 128 - 1) / (8 * 128)) * 128;
+    const int e_beg = imin(warp * seg, n_el), e_end = imin(e_beg + seg, n_el);
+
+    // pass 1: evaluate once, park results, count
+    uint32_t cnt = 0;
+    bool nonfinite = false;
+    for (int base = e_beg; base < e_end; base += 4 * 128) {
+        float4 gv[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int b = base + 128 * u + 4 * lane;
+            gv[u] = b < e_end ? ldg_f4(g + b) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int b = base + 128 * u + 4 * lane;
+            if (b < e_end) {
+                float4 *wp = reinterpret_cast<float4 *>(wt + b);
+                const float4 w = *wp;
+                const float gg[4] = {gv[u].x, gv[u].y, gv[u].z, gv[u].w};
+                const float ww[4] = {w.x, w.y, w.z, w.w};
+                float o[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float z = __fsub_rn(ww[j], __fmul_rn(eta, gg[j]));
+                    const bool k = fabsf(z) > thr;
+                    nonfinite |= z != z;
+                    o[j] = k ? (z > 0.f ? __fsub_rn(z, thr) : __fadd_rn(z, thr)) : __int_as_float(0x7fc00000);
+                    cnt += k;
+                }
+                *wp = make_float4(o[0], o[1], o[2], o[3]);
+            }
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, off);
+    if (lane == 0) s_wtot[warp] = cnt;
+    __syncthreads();
+    uint32_t pos = 0, tile_count = 0;
+#pragma unroll
+    for (int w = 0; w < kCThreads / 32; ++w) {
+        const uint32_t t = s_wtot[w];
+        if (w < warp) pos += t;
+        tile_count += t;
+    }
+    if (warp == 0) {
+        const unsigned long long prefix = lookback_warp(a.status, tile, tile_count, a.hdr);
+        if (lane == 0) s_excl = (uint32_t)prefix;
+    }
+    __syncthreads();
+    pos += s_excl;
+    const uint32_t cap = (uint32_t)imin<int64_t>(a.capacity, 0x7fffffff);
+
+    // pass 2: positions from ballots, writes
+    int row = e_beg / K;
+    int col = e_beg - row * K + 4 * lane;
+    while (col >= K) { col -= K; ++row; }
+    const unsigned lt = (1u << lane) - 1u;
+    for (int base = e_beg; base < e_end; base += 128) {
+        const int b = base + 4 * lane;
+        const bool in = b < e_end;
+        const float4 v = in ? *reinterpret_cast<const float4 *>(wt + b) : make_float4(__int_as_float(0x7fc00000),
+                                                                                   __int_as_float(0x7fc00000),
+                                                                                   __int_as_float(0x7fc00000),
+                                                                                   __int_as_float(0x7fc00000));
+        const float vv[4] = {v.x, v.y, v.z, v.w};
+        unsigned m[4];
+        uint32_t p = pos, step = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            m[j] = __ballot_sync(0xffffffffu, vv[j] == vv[j]);
+            p += __popc(m[j] & lt);
+            step += __popc(m[j]);
+        }
+        if (in && col == 0) a.out_row_ptr[r0 + row] = (int32_t)min(p, cap);
+        if (kBits && in && (lane & 7) == 0) {
+            const int q = lane >> 3;   // word q of this step = lanes 8q .. 8q+7
+            const uint32_t word = spread8(m[0] >> (8 * q)) | (spread8(m[1] >> (8 * q)) << 1) |
+                                  (spread8(m[2] >> (8 * q)) << 2) | (spread8(m[3] >> (8 * q)) << 3);
+            const int64_t wi = (int64_t)(r0 + row) * wpr + (col >> 5);
+            keepbits[wi] = word;
+            wordpos[wi] = (int32_t)p;
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (vv[j] == vv[j]) {
+                if (p < cap) {
+                    a.out_col[p] = col + j;
+                    a.out_val[p] = vv[j];
+                }
+                ++p;
+            }
+        }
+        pos += step;
+        col += 128;
+        while (col >= K) { col -= K; ++row; }
+    }
+    if (tile == a.num_tiles - 1 && tid == 0) {
+        const int64_t total = (int64_t)s_excl + tile_count;
+        a.out_row_ptr[a.rows] = (int32_t)imin<int64_t>(total, cap);
+        if (total > (int64_t)cap) {
+            dev_flag(a.hdr, CSRT_DEV_CAPACITY);
+            atomicMax(&a.hdr->required, (unsigned long long)total);
+        }
+    }
+    if (__syncthreads_or(nonfinite) && tid == 0) dev_flag(a.hdr, CSRT_DEV_NONFINITE);
+}
+
+// Returns through *bits_done whether the prox kernel emitted the keep bitmask
+// (then the transposed copy is built from it).
 static int compact_launch(bool prox, const float *src, int32_t rows, int32_t cols, const csrt_csr *in,
                           float eta, float thr, csrt_csr *out, void *ws, size_t ws_bytes,
-                          cudaStream_t s) {
+                          cudaStream_t s, bool want_bits = false, bool *bits_done = nullptr) {
+    if (bits_done) *bits_done = false;
     const int64_t elems = (int64_t)rows * cols;
     if (elems == 0) {
         CSRT_CHECK_CUDA(cudaMemsetAsync(out->row_ptr, 0, sizeof(int32_t) * ((size_t)rows + 1), s));
@@ -458,7 +645,7 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
     const bool row_path = cols % 4 == 0 && cols <= kRowMaxK && (reinterpret_cast<uintptr_t>(src) & 15) == 0;
     const int32_t rows_per_tile = row_path ? imax<int32_t>(1, kRowBudget / cols) : 0;
     const int64_t tiles = row_path ? ceil_div<int64_t>(rows, rows_per_tile) : ceil_div<int64_t>(elems, kTile);
-    CSRT_ARG(ws_bytes >= kWsHeaderBytes + compact_scratch_bytes(elems), "workspace too small for compaction");
+    CSRT_ARG(ws_bytes >= kWsHeaderBytes + status_bytes(elems), "workspace too small for compaction");
     WsHeader *hdr = static_cast<WsHeader *>(ws);
     unsigned long long *status = reinterpret_cast<unsigned long long *>(ws_scratch(ws));
     CSRT_CHECK_CUDA(cudaMemsetAsync(&hdr->ticket, 0, sizeof(unsigned int), s));
@@ -487,14 +674,31 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
         cudaGetDevice(&dev);
         if (dev >= 0 && dev < 64 && !attr_done[dev]) {
             const int max_smem = (int)((size_t)(kRowMaxK + kRowBudget + 1) * sizeof(float));
-            CSRT_CHECK_CUDA(cudaFuncSetAttribute(compact_rows_kernel<true>,
+            CSRT_CHECK_CUDA(cudaFuncSetAttribute(prox_rows_kernel<true>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
+            CSRT_CHECK_CUDA(cudaFuncSetAttribute(prox_rows_kernel<false>,
                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
             attr_done[dev] = true;
         }
-        if (prox) compact_rows_kernel<true><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile);
-        else compact_rows_kernel<false><<<(unsigned)tiles, kCThreads, 0, s>>>(a, rows_per_tile);
+        if (prox) {
+            const bool bits = want_bits && cols % 32 == 0 &&
+                              ws_bytes >= kWsHeaderBytes + status_bytes(elems) + 2 * bits_bytes(rows, cols) +
+                                              transpose_scratch_bytes(rows, cols);
+            char *base = ws_scratch(ws);
+            uint32_t *keepbits = reinterpret_cast<uint32_t *>(base + status_bytes(elems));
+            int32_t *wordpos = reinterpret_cast<int32_t *>(base + status_bytes(elems) + bits_bytes(rows, cols));
+            if (bits)
+                prox_rows_kernel<true><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile, keepbits, wordpos,
+                                                                                 cols / 32);
+            else
+                prox_rows_kernel<false><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile, nullptr, nullptr,
+                                                                                  0);
+            if (bits_done) *bits_done = bits;
+        } else {
+            compact_rows_kernel<false><<<(unsigned)tiles, kCThreads, 0, s>>>(a, rows_per_tile);
+        }
         count_launch();
-        return check_launch("compact_rows_kernel");
+        return check_launch("row-tile compaction kernel");
     }
     const bool vec = (reinterpret_cast<uintptr_t>(src) & 15) == 0;
     dim3 grid((unsigned)tiles), block(kCThreads);
@@ -678,6 +882,101 @@ __global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict
     }
 }
 
+
+// ---------------------------------------------------------------------------
+// Transposed copy from the prox kernel's keep bitmask (K % 32 == 0). One warp
+// per (32-row block b, 32-column word c).
+//  count: lane r loads row r's word; a 32 x 32 bit transpose (five shuffle
+//         stages) gives lane j the rows present in column 32c + j; its popcount
+//         is the block's count for that column.
+//  write: the block walks its 32 rows in order; lane j handles column 32c + j.
+//         In row r the CSR positions of the kept columns are consecutive
+//         (word position + rank in the word), so the values are gathered and
+//         t_pos is written coalesced; each column's transposed run advances by
+//         one per kept row.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int sft = 16; sft >= 1; sft >>= 1) {
+        const uint32_t lo = sft == 16 ? 0x0000FFFFu : sft == 8 ? 0x00FF00FFu : sft == 4 ? 0x0F0F0F0Fu
+                          : sft == 2 ? 0x33333333u : 0x55555555u;
+        const uint32_t other = __shfl_xor_sync(0xffffffffu, x, sft);
+        if ((lane & sft) == 0) x = (x & lo) | ((other & lo) << sft);
+        else x = (x & ~lo) | ((other & ~lo) >> sft);
+    }
+    return x;
+}
+
+__global__ void __launch_bounds__(256) trb_count_kernel(const uint32_t *__restrict__ keepbits, int32_t rows,
+                                                        int32_t wpr, int32_t cols, int32_t *__restrict__ cnt) {
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nb = ceil_div<int64_t>(rows, 32);
+    if (gw >= nb * wpr) return;
+    const int b = (int)(gw / wpr), c = (int)(gw % wpr);
+    const int row = b * 32 + lane;
+    const uint32_t x = row < rows ? __ldg(keepbits + (int64_t)row * wpr + c) : 0u;
+    const uint32_t colmask = warp_transpose32(x);
+    cnt[(int64_t)b * cols + c * 32 + lane] = __popc(colmask);
+}
+
+__global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restrict__ keepbits,
+                                                        const int32_t *__restrict__ wordpos, int32_t rows,
+                                                        int32_t wpr, int32_t cols, const int32_t *__restrict__ off,
+                                                        const int32_t *__restrict__ t_row_ptr,
+                                                        const float *__restrict__ val, int32_t *__restrict__ t_col,
+                                                        float *__restrict__ t_val, int32_t *__restrict__ t_pos,
+                                                        int64_t capacity) {
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nb = ceil_div<int64_t>(rows, 32);
+    if (gw >= nb * wpr) return;
+    const int b = (int)(gw / wpr), c = (int)(gw % wpr);
+    const int my_row = b * 32 + lane;
+    const uint32_t rw_mine = my_row < rows ? __ldg(keepbits + (int64_t)my_row * wpr + c) : 0u;
+    const int32_t rp_mine = my_row < rows ? __ldg(wordpos + (int64_t)my_row * wpr + c) : 0;
+    const int col = c * 32 + lane;
+    int64_t pc = (int64_t)__ldg(t_row_ptr + col) + __ldg(off + (int64_t)b * cols + col);
+    const unsigned lt = (1u << lane) - 1u;
+    const int nr = imin(32, rows - b * 32);
+    for (int r = 0; r < nr; ++r) {
+        const uint32_t rw = __shfl_sync(0xffffffffu, rw_mine, r);
+        const int32_t rp = __shfl_sync(0xffffffffu, rp_mine, r);
+        if ((rw >> lane) & 1u) {
+            const int64_t pr = (int64_t)rp + __popc(rw & lt);
+            if (pc < capacity && pr < capacity) {
+                t_col[pc] = b * 32 + r;
+                t_val[pc] = __ldg(val + pr);
+                t_pos[pr] = (int32_t)pc;
+            }
+            ++pc;
+        }
+    }
+}
+
+// Transposed copy from the keep bitmask; scratch: [status][keepbits][wordpos][cnt][coltot].
+static int transpose_from_bits(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s) {
+    const int32_t rows = w->rows, cols = w->cols;
+    const int32_t wpr = cols / 32;
+    const int64_t elems = (int64_t)rows * cols;
+    char *base = ws_scratch(ws);
+    const uint32_t *keepbits = reinterpret_cast<const uint32_t *>(base + status_bytes(elems));
+    const int32_t *wordpos = reinterpret_cast<const int32_t *>(base + status_bytes(elems) + bits_bytes(rows, cols));
+    int32_t *cnt = reinterpret_cast<int32_t *>(base + status_bytes(elems) + 2 * bits_bytes(rows, cols));
+    const int nb = (int)ceil_div<int64_t>(rows, 32);
+    int32_t *coltot = cnt + (int64_t)nb * cols;
+    const int64_t warps = (int64_t)nb * wpr;
+    const unsigned grid = (unsigned)ceil_div<int64_t>(warps * 32, 256);
+    trb_count_kernel<<<grid, 256, 0, s>>>(keepbits, rows, wpr, cols, cnt);
+    tr_colscan_kernel<<<ceil_div(cols, 32), 256, 0, s>>>(cnt, nb, cols, coltot);
+    scan_single_block_kernel<<<1, 1024, 0, s>>>(coltot, cols, w->t_row_ptr);
+    trb_write_kernel<<<grid, 256, 0, s>>>(keepbits, wordpos, rows, wpr, cols, cnt, w->t_row_ptr, w->val,
+                                          w->t_col_idx, w->t_val, w->t_pos, w->capacity);
+    count_launch(4);
+    return check_launch("transpose-from-bits kernels");
+}
+
 int transpose_impl(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s) {
     CSRT_ARG(w->t_row_ptr && w->t_col_idx && w->t_val && w->t_pos, "transposed arrays not set");
     const int32_t rows = w->rows, cols = w->cols;
@@ -759,9 +1058,12 @@ int prox_update_compact(const csrt_csr *w_in, const float *g, float eta, float l
     CSRT_ARG(ws != nullptr, "workspace is NULL");
     const float thr = eta * lambda;  // fl32(eta*lambda), the threshold of Eq. prox
     cudaStream_t s = as_stream(stream);
-    rc = compact_launch(true, g, w_in->rows, w_in->cols, w_in, eta, thr, w_out, ws, ws_bytes, s);
+    const bool want_t = w_out->t_row_ptr != nullptr;
+    if (want_t) CSRT_ARG(w_out->t_col_idx && w_out->t_val && w_out->t_pos, "transposed arrays partly set");
+    bool bits = false;
+    rc = compact_launch(true, g, w_in->rows, w_in->cols, w_in, eta, thr, w_out, ws, ws_bytes, s, want_t, &bits);
     if (rc) return rc;
-    if (w_out->t_row_ptr) rc = transpose_impl(w_out, ws, ws_bytes, s);
+    if (want_t) rc = bits ? transpose_from_bits(w_out, ws, ws_bytes, s) : transpose_impl(w_out, ws, ws_bytes, s);
     return rc;
 }
 

@@ -50,7 +50,7 @@ int csrt_workspace_bytes(int32_t rows, int32_t cols, int32_t max_n, size_t *byte
     CSRT_ARG(rows >= 0 && cols >= 0 && max_n >= 0, "negative size");
     CSRT_ARG((int64_t)rows * cols < (int64_t)1 << 31, "rows*cols must be below 2^31");
     int64_t elems = (int64_t)rows * cols;
-    size_t need = compact_scratch_bytes(elems);
+    size_t need = compact_scratch_bytes(rows, cols);
     size_t t = transpose_scratch_bytes(rows, cols);
     if (t > need) need = t;
     t = spmm_scratch_bytes(max_n);

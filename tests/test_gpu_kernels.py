@@ -282,10 +282,10 @@ def test_prox_bit_exact(C, m, k, density, gscale, eta, lam):
     assert ws.status()[0] == 0
 
 
-def test_prox_chain_of_steps_bit_exact(C):
+@pytest.mark.parametrize("m,k", [(200, 333), (200, 320), (70, 4096)])
+def test_prox_chain_of_steps_bit_exact(C, m, k):
     # several prox steps in a row (double-buffered), each fed the same G as the oracle
-    rng = np.random.default_rng(21)
-    m, k = 200, 333
+    rng = np.random.default_rng(21 + k)
     a = _sparse(rng, m, k, 0.2)
     ws = _ws(C, m, k, 1)
     bufs = [_gpu_csr(C, a, ws), C.CSR(m, k)]
