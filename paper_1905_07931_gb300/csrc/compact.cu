@@ -73,42 +73,73 @@ struct CompactArgs {
 // tile's aggregate, sums predecessors' aggregates back to the nearest
 // published inclusive prefix, publishes this tile's inclusive prefix and
 // returns the exclusive prefix (the number of entries kept before the tile).
-// Every poll is bounded; a wait that runs out sets CSRT_DEV_TIMEOUT.
+// Each round reads a window of 32 * kLbWays predecessors (kLbWays per lane),
+// so inclusive prefixes propagate kLbWays times faster than with one word per
+// lane. Every poll is bounded; a wait that runs out sets CSRT_DEV_TIMEOUT.
+constexpr int kLbWays = 4;
+
 __device__ __forceinline__ unsigned long long lookback_warp(unsigned long long *status, int64_t tile,
                                                             uint32_t count, WsHeader *hdr) {
     const int lane = threadIdx.x & 31;
-    unsigned long long prefix = 0;
     if (tile == 0) {
         if (lane == 0) st_release_u64(status, kFlagInc | count);
         return 0;
     }
     if (lane == 0) st_release_u64(status + tile, kFlagAgg | count);
-    int64_t pred = tile - 1;
+    unsigned long long prefix = 0;
+    int64_t pred = tile - 1;   // window entry (v, lane) is predecessor pred - 32 v - lane
     unsigned int spins = 0;
     bool timed_out = false;
     while (true) {
-        const int64_t idx = pred - lane;
-        unsigned long long st = idx >= 0 ? ld_acquire_u64(status + idx) : kFlagInc;
-        while (__any_sync(0xffffffffu, (st >> 32) == 0)) {
+        unsigned long long st[kLbWays];
+#pragma unroll
+        for (int v = 0; v < kLbWays; ++v) {
+            const int64_t idx = pred - 32 * v - lane;
+            st[v] = idx >= 0 ? ld_acquire_u64(status + idx) : kFlagInc;
+        }
+        int first_v = kLbWays, first_lane = 32;   // nearest inclusive prefix in the window
+        while (true) {
+            first_v = kLbWays;
+            first_lane = 32;
+#pragma unroll
+            for (int v = kLbWays - 1; v >= 0; --v) {
+                const unsigned inc = __ballot_sync(0xffffffffu, (st[v] >> 32) == 2);
+                if (inc) {
+                    first_v = v;
+                    first_lane = __ffs(inc) - 1;
+                }
+            }
+            // every entry nearer than the inclusive one must have published its aggregate
+            bool missing = false;
+#pragma unroll
+            for (int v = 0; v < kLbWays; ++v) {
+                const bool nearer = v < first_v || (v == first_v && lane < first_lane);
+                missing |= nearer && (st[v] >> 32) == 0;
+            }
+            if (!__any_sync(0xffffffffu, missing)) break;
             if (++spins > kSpinLimit) {
                 timed_out = true;
                 break;
             }
-            __nanosleep(64);
-            if ((st >> 32) == 0) st = ld_acquire_u64(status + idx);
+            __nanosleep(32);
+#pragma unroll
+            for (int v = 0; v < kLbWays; ++v) {
+                const int64_t idx = pred - 32 * v - lane;
+                if ((st[v] >> 32) == 0 && idx >= 0) st[v] = ld_acquire_u64(status + idx);
+            }
         }
         if (timed_out) break;
-        const unsigned inc_mask = __ballot_sync(0xffffffffu, (st >> 32) == 2);
-        unsigned long long part = st & 0xffffffffull;
-        if (inc_mask) {
-            const int first = __ffs(inc_mask) - 1;  // nearest inclusive predecessor
-            if (lane > first) part = 0;
+        unsigned long long part = 0;
+#pragma unroll
+        for (int v = 0; v < kLbWays; ++v) {
+            const bool take = v < first_v || (v == first_v && lane <= first_lane);
+            if (take) part += st[v] & 0xffffffffull;
         }
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
         prefix += part;
-        if (inc_mask) break;
-        pred -= 32;
+        if (first_v < kLbWays) break;
+        pred -= 32 * kLbWays;
     }
     if (lane == 0) {
         if (timed_out) {
