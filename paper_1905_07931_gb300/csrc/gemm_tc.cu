@@ -247,6 +247,181 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
 }
 
+
+// ---------------------------------------------------------------------------
+// Persistent variant (the default): one CTA per SM walks its share of the
+// 128 x 256 tiles. The accumulator is double-buffered in tensor memory (512
+// columns), so the epilogue of one tile overlaps the TMA loads and MMAs of the
+// next. The epilogue goes through shared memory: each epilogue warp writes its
+// 32 rows x 32 columns (128-byte swizzled, bank-conflict free) into one of two
+// 4 KB staging buffers and one lane stores it with a TMA tensor store, so G
+// leaves in full lines; rows and columns beyond the matrix are clipped by TMA.
+// ---------------------------------------------------------------------------
+constexpr int kPEpiBytes = 32 * 32 * 4;   // one 32 x 32 float staging buffer
+constexpr int kPSmemBytes = kTcStages * kTcStageBytes + 4 * 2 * kPEpiBytes + 1024 + 256;
+
+// Bounded wait that also gives up early once another role has aborted.
+__device__ __forceinline__ bool mbar_wait_or_abort(uint64_t *bar, uint32_t parity, volatile int *abort_flag) {
+    const uint32_t addr = smem_u32(bar);
+    for (unsigned i = 0; i < kTcWaitLimit; ++i) {
+        uint32_t done;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            " selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(done)
+            : "r"(addr), "r"(parity)
+            : "memory");
+        if (done) return true;
+        if ((i & 63) == 63 && *abort_flag) return false;
+        if (i > 64) __nanosleep(32);
+    }
+    *abort_flag = 1;
+    return false;
+}
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, int x, int y, const void *src) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y), "r"(smem_u32(src))
+                 : "memory");
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(kTcThreads, 1)
+    gemm_tf32_tc_persistent_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
+                                   const __grid_constant__ CUtensorMap map_g, TcArgs a, int32_t tiles_n,
+                                   int32_t num_tiles) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sa = smem;
+    uint8_t *sb = smem + kTcStages * kTcABytes;
+    uint8_t *epi = smem + kTcStages * kTcStageBytes;                       // 1024-aligned
+    uint64_t *full = reinterpret_cast<uint64_t *>(epi + 4 * 2 * kPEpiBytes);
+    uint64_t *empty = full + kTcStages;
+    uint64_t *accf = empty + kTcStages;    // [2] accumulator ready
+    uint64_t *acce = accf + 2;             // [2] accumulator drained
+    uint64_t *fin = acce + 2;              // all MMAs of this CTA complete
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(fin + 1);
+    __shared__ volatile int s_abort;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int num_kb = (a.n + kTcBK - 1) / kTcBK;
+
+    if (threadIdx.x == 0) {
+        s_abort = 0;
+        for (int s = 0; s < kTcStages; ++s) {
+            mbar_init(full + s, 1);
+            mbar_init(empty + s, 1);
+        }
+        mbar_init(accf, 1);
+        mbar_init(accf + 1, 1);
+        mbar_init(acce, 4);
+        mbar_init(acce + 1, 4);
+        mbar_init(fin, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_a)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_b)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_g)) : "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(2 * kTcBN)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int it = 0;
+            for (int t = blockIdx.x; t < num_tiles && !s_abort; t += gridDim.x) {
+                const int m0 = (t / tiles_n) * kTcBM, n0 = (t % tiles_n) * kTcBN;
+                for (int kb = 0; kb < num_kb; ++kb, ++it) {
+                    const int s = it % kTcStages;
+                    if (!mbar_wait_or_abort(empty + s, ((it / kTcStages) & 1) ^ 1, &s_abort)) break;
+                    mbar_expect_tx(full + s, kTcStageBytes);
+                    tma_load_2d(sa + s * kTcABytes, &map_a, kb * kTcBK, m0, full + s);
+                    tma_load_2d(sb + s * kTcBBytes, &map_b, kb * kTcBK, n0, full + s);
+                }
+            }
+            // every issued load must land before the CTA may exit
+            for (int i = imax(0, it - kTcStages); i < it; ++i) mbar_wait(full + i % kTcStages, (i / kTcStages) & 1);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            int it = 0, j = 0;
+            for (int t = blockIdx.x; t < num_tiles && !s_abort; t += gridDim.x, ++j) {
+                const int acc = j & 1;
+                if (!mbar_wait_or_abort(acce + acc, ((j >> 1) & 1) ^ 1, &s_abort)) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t d = tmem + (uint32_t)(acc * kTcBN);
+                for (int kb = 0; kb < num_kb; ++kb, ++it) {
+                    const int s = it % kTcStages;
+                    if (!mbar_wait_or_abort(full + s, (it / kTcStages) & 1, &s_abort)) break;
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll
+                    for (int k = 0; k < kTcBK / 8; ++k) {
+                        const uint64_t ad = smem_desc_sw128(sa + s * kTcABytes + k * 32);
+                        const uint64_t bd = smem_desc_sw128(sb + s * kTcBBytes + k * 32);
+                        mma_tf32(d, ad, bd, (kb > 0 || k > 0) ? 1u : 0u);
+                    }
+                    mma_commit(empty + s);
+                }
+                mma_commit(accf + acc);
+            }
+            mma_commit(fin);
+            mbar_wait(fin, 0);   // nothing of ours still runs on the tensor core
+        }
+    } else {
+        const int q = warp & 3;   // TMEM lanes 32q .. 32q+31 = tile rows 32q ..
+        uint8_t *stage0 = epi + (q * 2) * kPEpiBytes;
+        int chunk = 0, j = 0;
+        for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++j) {
+            const int acc = j & 1;
+            const bool ok = __all_sync(0xffffffffu, mbar_wait_or_abort(accf + acc, (j >> 1) & 1, &s_abort));
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const int m0 = (t / tiles_n) * kTcBM, n0 = (t % tiles_n) * kTcBN;
+            for (int c = 0; c < kTcBN; c += 32, ++chunk) {
+                uint8_t *buf = stage0 + (chunk & 1) * kPEpiBytes;
+                if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+                __syncwarp();
+                uint32_t r[32];
+                tmem_ld_32cols(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kTcBN + c), r);
+                // row `lane` of the 32 x 32 block, 16-byte chunk i at (i ^ (lane & 7)) (128-byte swizzle)
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    float4 *dst = reinterpret_cast<float4 *>(buf + lane * 128 + ((i ^ (lane & 7)) << 4));
+                    *dst = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
+                                       __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
+                }
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) tma_store_2d(&map_g, n0 + c, m0 + q * 32, buf);
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(acce + acc)) : "memory");
+        }
+        if (lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        __syncwarp();
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (threadIdx.x == 0 && s_abort) {
+        dev_flag(a.hdr, CSRT_DEV_TIMEOUT);
+        a.hdr->timeout_site = 4;
+    }
+    if (warp == 1) {
+        __syncwarp();
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * kTcBN) : "memory");
+    }
+}
+
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     static bool tried = false;
@@ -262,13 +437,14 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// Row-major rows x cols float32 matrix, box of `box_rows` rows x 32 columns, 128-byte swizzle.
+// Row-major rows x cols float32 matrix, box of `box_rows` rows x 32 columns, 128-byte swizzle
+// (the operand stages and the 32 x 32 epilogue blocks share this layout).
 static bool make_map(CUtensorMap *map, const float *base, int64_t rows, int64_t cols, int box_rows) {
     auto fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)cols * sizeof(float)};
-    cuuint32_t box[2] = {(cuuint32_t)kTcBK, (cuuint32_t)box_rows};
+    cuuint32_t box[2] = {32u, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
     CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float *>(base), dims, strides, box, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -296,14 +472,18 @@ int gemm_tc_tf32(const float *dy, const float *x, int32_t m, int32_t k, int32_t 
     if (m < 64 || k < 64) return CSRT_OK;       // tiny outputs: the CUDA-core kernel is as fast
     CSRT_ARG(ws != nullptr && ws_bytes >= kWsHeaderBytes, "weight_grad_dense (tf32) needs the workspace");
     if (!device_is_sm10x()) return CSRT_OK;
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, mg;
     if (!make_map(&ma, dy, m, n, kTcBM) || !make_map(&mb, x, k, n, kTcBN)) return CSRT_OK;
+    // the TMA-store epilogue needs a 16-byte aligned G with rows a multiple of 16 bytes
+    const bool tma_out = k % 4 == 0 && (reinterpret_cast<uintptr_t>(g) & 15) == 0 && make_map(&mg, g, m, k, 32);
     static bool attr_set[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
         CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_tf32_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              kTcSmemBytes));
+        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_tf32_tc_persistent_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kPSmemBytes));
         attr_set[dev] = true;
     }
     TcArgs a;
@@ -312,7 +492,16 @@ int gemm_tc_tf32(const float *dy, const float *x, int32_t m, int32_t k, int32_t 
     a.k = k;
     a.n = n;
     a.hdr = static_cast<WsHeader *>(ws);
-    dim3 grid((unsigned)ceil_div<int64_t>(k, kTcBN), (unsigned)ceil_div<int64_t>(m, kTcBM));
+    const int tiles_m = (int)ceil_div<int64_t>(m, kTcBM), tiles_n = (int)ceil_div<int64_t>(k, kTcBN);
+    if (tma_out) {
+        const int tiles = tiles_m * tiles_n;
+        const int grid = imin(tiles, num_sms());
+        gemm_tf32_tc_persistent_kernel<<<grid, kTcThreads, kPSmemBytes, s>>>(ma, mb, mg, a, tiles_n, tiles);
+        count_launch();
+        *handled = true;
+        return check_launch("gemm_tf32_tc_persistent_kernel");
+    }
+    dim3 grid((unsigned)tiles_n, (unsigned)tiles_m);
     gemm_tf32_tc_kernel<<<grid, kTcThreads, kTcSmemBytes, s>>>(ma, mb, a);
     count_launch();
     *handled = true;
