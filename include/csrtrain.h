@@ -150,6 +150,18 @@ int spmm_fwd(const csrt_csr *w, const float *x, int32_t n, float *y,
 int spmm_bwd_t(const csrt_csr *w, const float *dy, int32_t n, float *dx,
                void *ws, size_t ws_bytes, void *stream);
 
+/* spmm_fwd with the layer epilogue fused (same arithmetic as spmm_fwd then
+ * csrt_bias_act_fwd): Y[i, c] = act(fl32(sum + bias[i])), act = ReLU when
+ * relu != 0, identity otherwise. bias (M floats) may be NULL. */
+int spmm_fwd_bias_act(const csrt_csr *w, const float *x, int32_t n, const float *bias, int32_t relu,
+                      float *y, void *ws, size_t ws_bytes, void *stream);
+
+/* spmm_bwd_t with the ReLU backward of the layer below fused (same result as
+ * spmm_bwd_t then csrt_relu_bwd): dX[j, c] = (W^T dY)[j, c] where
+ * y_below[j, c] > 0, else 0. y_below is K x n, the output of the layer below. */
+int spmm_bwd_t_relu(const csrt_csr *w, const float *dy, int32_t n, const float *y_below, float *dx,
+                    void *ws, size_t ws_bytes, void *stream);
+
 /* weight_grad_dense -- gradient of every weight for the prox phase (the
  * matrix w - eta*G of Section 3.3 needs G at all M x K entries).
  * G[i, j] = sum_c dY[i, c] X[j, c]; dY is m x n, X is k x n, G is m x k,

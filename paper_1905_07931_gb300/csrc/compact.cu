@@ -512,10 +512,10 @@ __device__ __forceinline__ uint32_t spread8(uint32_t x) {
     return x;
 }
 
-template <bool kBits, int V>
-__global__ void __launch_bounds__(kCThreads, V <= 9 ? 3 : 2) prox_rows_kernel(CompactArgs a, int32_t rows_per_tile,
-                                                                        uint32_t *__restrict__ keepbits,
-                                                                        int32_t *__restrict__ wordpos, int32_t wpr) {
+template <bool kBits>
+__global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, int32_t rows_per_tile,
+                                                                  uint32_t *__restrict__ keepbits,
+                                                                  int32_t *__restrict__ wordpos, int32_t wpr) {
     extern __shared__ __align__(16) float row_smem[];
     float *wt = row_smem;
     int32_t *s_rp = reinterpret_cast<int32_t *>(row_smem + rows_per_tile * a.cols);
@@ -532,22 +532,9 @@ __global__ void __launch_bounds__(kCThreads, V <= 9 ? 3 : 2) prox_rows_kernel(Co
     const int r0 = (int)(tile * rows_per_tile);
     const int nrows = imin(rows_per_tile, a.rows - r0);
     const int n_el = nrows * K;
+    const float *g = a.src + (int64_t)r0 * K;
     const float eta = a.eta, thr = a.thr;
 
-    // warp segment of V steps of 128 entries; lane owns float4 i at e_beg + 128 i + 4 lane
-    const int e_beg = warp * V * 128;
-    const int e_end = imin(e_beg + V * 128, n_el);
-    // 1. issue this thread's loads of G first: they stream while the old weights are merged
-    float4 gv[V];
-    {
-        const float *g = a.src + (int64_t)r0 * K;
-#pragma unroll
-        for (int i = 0; i < V; ++i) {
-            const int b = e_beg + 128 * i + 4 * lane;
-            gv[i] = b < e_end ? ldg_f4(g + b) : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-    }
-    // 2. old weights of the tile's rows into the shared tile
     for (int i = tid; i <= nrows; i += kCThreads) s_rp[i] = a.in_row_ptr[r0 + i];
     {
         float4 *w4 = reinterpret_cast<float4 *>(wt);
@@ -567,29 +554,38 @@ __global__ void __launch_bounds__(kCThreads, V <= 9 ? 3 : 2) prox_rows_kernel(Co
     }
     __syncthreads();
 
-    // 3. evaluate: the kept value, or NaN for a dropped entry (a kept value is never NaN)
+    const int seg = ((n_el + 8 * 128 - 1) / (8 * 128)) * 128;
+    const int e_beg = imin(warp * seg, n_el), e_end = imin(e_beg + seg, n_el);
+
+    // pass 1: evaluate once, park results, count
     uint32_t cnt = 0;
     bool nonfinite = false;
+    for (int base = e_beg; base < e_end; base += 4 * 128) {
+        float4 gv[4];
 #pragma unroll
-    for (int i = 0; i < V; ++i) {
-        const int b = e_beg + 128 * i + 4 * lane;
-        if (b < e_end) {
-            const float4 w = *reinterpret_cast<const float4 *>(wt + b);
-            const float gg[4] = {gv[i].x, gv[i].y, gv[i].z, gv[i].w};
-            const float ww[4] = {w.x, w.y, w.z, w.w};
-            float o[4];
+        for (int u = 0; u < 4; ++u) {
+            const int b = base + 128 * u + 4 * lane;
+            gv[u] = b < e_end ? ldg_f4(g + b) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const float z = __fsub_rn(ww[j], __fmul_rn(eta, gg[j]));
-                const bool k = fabsf(z) > thr;
-                nonfinite |= z != z;
-                o[j] = k ? (z > 0.f ? __fsub_rn(z, thr) : __fadd_rn(z, thr)) : __int_as_float(0x7fc00000);
-                cnt += k;
+        for (int u = 0; u < 4; ++u) {
+            const int b = base + 128 * u + 4 * lane;
+            if (b < e_end) {
+                float4 *wp = reinterpret_cast<float4 *>(wt + b);
+                const float4 w = *wp;
+                const float gg[4] = {gv[u].x, gv[u].y, gv[u].z, gv[u].w};
+                const float ww[4] = {w.x, w.y, w.z, w.w};
+                float o[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float z = __fsub_rn(ww[j], __fmul_rn(eta, gg[j]));
+                    const bool k = fabsf(z) > thr;
+                    nonfinite |= z != z;
+                    o[j] = k ? (z > 0.f ? __fsub_rn(z, thr) : __fadd_rn(z, thr)) : __int_as_float(0x7fc00000);
+                    cnt += k;
+                }
+                *wp = make_float4(o[0], o[1], o[2], o[3]);
             }
-            gv[i] = make_float4(o[0], o[1], o[2], o[3]);
-        } else {
-            gv[i] = make_float4(__int_as_float(0x7fc00000), __int_as_float(0x7fc00000), __int_as_float(0x7fc00000),
-                                __int_as_float(0x7fc00000));
         }
     }
 #pragma unroll
@@ -603,7 +599,6 @@ __global__ void __launch_bounds__(kCThreads, V <= 9 ? 3 : 2) prox_rows_kernel(Co
         if (w < warp) pos += t;
         tile_count += t;
     }
-    // 4. offset of the tile
     if (warp == 0) {
         const unsigned long long prefix = lookback_warp(a.status, tile, tile_count, a.hdr);
         if (lane == 0) s_excl = (uint32_t)prefix;
@@ -612,16 +607,19 @@ __global__ void __launch_bounds__(kCThreads, V <= 9 ? 3 : 2) prox_rows_kernel(Co
     pos += s_excl;
     const uint32_t cap = (uint32_t)imin<int64_t>(a.capacity, 0x7fffffff);
 
-    // 5. write: ranks from ballots, each step's kept entries form one run
+    // pass 2: positions from ballots, writes
     int row = e_beg / K;
     int col = e_beg - row * K + 4 * lane;
     while (col >= K) { col -= K; ++row; }
     const unsigned lt = (1u << lane) - 1u;
-#pragma unroll
-    for (int i = 0; i < V; ++i) {
-        if (e_beg + 128 * i >= e_end) break;   // warp-uniform
-        const bool in = e_beg + 128 * i + 4 * lane < e_end;
-        const float vv[4] = {gv[i].x, gv[i].y, gv[i].z, gv[i].w};
+    for (int base = e_beg; base < e_end; base += 128) {
+        const int b = base + 4 * lane;
+        const bool in = b < e_end;
+        const float4 v = in ? *reinterpret_cast<const float4 *>(wt + b) : make_float4(__int_as_float(0x7fc00000),
+                                                                                   __int_as_float(0x7fc00000),
+                                                                                   __int_as_float(0x7fc00000),
+                                                                                   __int_as_float(0x7fc00000));
+        const float vv[4] = {v.x, v.y, v.z, v.w};
         unsigned m[4];
         uint32_t p = pos, step = 0;
 #pragma unroll
@@ -664,6 +662,8 @@ __global__ void __launch_bounds__(kCThreads, V <= 9 ? 3 : 2) prox_rows_kernel(Co
     if (__syncthreads_or(nonfinite) && tid == 0) dev_flag(a.hdr, CSRT_DEV_NONFINITE);
 }
 
+// Returns through *bits_done whether the prox kernel emitted the keep bitmask
+// (then the transposed copy is built from it).
 static int compact_launch(bool prox, const float *src, int32_t rows, int32_t cols, const csrt_csr *in,
                           float eta, float thr, csrt_csr *out, void *ws, size_t ws_bytes,
                           cudaStream_t s, bool want_bits = false, bool *bits_done = nullptr) {
@@ -705,13 +705,9 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
         cudaGetDevice(&dev);
         if (dev >= 0 && dev < 64 && !attr_done[dev]) {
             const int max_smem = (int)((size_t)(kRowMaxK + kRowBudget + 1) * sizeof(float));
-            CSRT_CHECK_CUDA(cudaFuncSetAttribute(prox_rows_kernel<true, 9>,
+            CSRT_CHECK_CUDA(cudaFuncSetAttribute(prox_rows_kernel<true>,
                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
-            CSRT_CHECK_CUDA(cudaFuncSetAttribute(prox_rows_kernel<false, 9>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
-            CSRT_CHECK_CUDA(cudaFuncSetAttribute(prox_rows_kernel<true, 16>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
-            CSRT_CHECK_CUDA(cudaFuncSetAttribute(prox_rows_kernel<false, 16>,
+            CSRT_CHECK_CUDA(cudaFuncSetAttribute(prox_rows_kernel<false>,
                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
             attr_done[dev] = true;
         }
@@ -722,19 +718,12 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
             char *base = ws_scratch(ws);
             uint32_t *keepbits = reinterpret_cast<uint32_t *>(base + status_bytes(elems));
             int32_t *wordpos = reinterpret_cast<int32_t *>(base + status_bytes(elems) + bits_bytes(rows, cols));
-            // V float4 per thread hold a whole tile: 8 warps x V steps x 128 entries
-            const bool v9 = (int64_t)rows_per_tile * cols <= 8 * 9 * 128;
-            if (bits) {
-                if (v9) prox_rows_kernel<true, 9><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile, keepbits,
-                                                                                        wordpos, cols / 32);
-                else prox_rows_kernel<true, 16><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile, keepbits,
-                                                                                      wordpos, cols / 32);
-            } else {
-                if (v9) prox_rows_kernel<false, 9><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile, nullptr,
-                                                                                         nullptr, 0);
-                else prox_rows_kernel<false, 16><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile, nullptr,
-                                                                                       nullptr, 0);
-            }
+            if (bits)
+                prox_rows_kernel<true><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile, keepbits, wordpos,
+                                                                                 cols / 32);
+            else
+                prox_rows_kernel<false><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile, nullptr, nullptr,
+                                                                                  0);
             if (bits_done) *bits_done = bits;
         } else {
             compact_rows_kernel<false><<<(unsigned)tiles, kCThreads, 0, s>>>(a, rows_per_tile);

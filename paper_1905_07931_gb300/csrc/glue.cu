@@ -48,40 +48,53 @@ __global__ void bias_grad_sgd_kernel(const float *__restrict__ dy, int32_t m, in
     }
 }
 
-// Softmax cross-entropy, 32 samples per block, 8 warps over the classes.
+// Softmax cross-entropy: a block of 256 threads takes 8 samples (columns);
+// thread (class group g = 0..31, column c = 0..7) walks classes g, g+32, ...
+// so every warp load covers 4 classes x 8 consecutive columns (32-byte
+// segments). One pass keeps a running maximum and rescaled sum; the groups
+// are combined in a fixed order in shared memory; a second pass writes dz.
 __global__ void __launch_bounds__(256) softmax_xent_kernel(const float *__restrict__ z,
                                                            const int32_t *__restrict__ labels, int32_t classes,
                                                            int32_t n, float *__restrict__ dz,
                                                            float *__restrict__ per_sample) {
-    __shared__ float red[8][32];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int64_t col = (int64_t)blockIdx.x * 32 + lane;
+    __shared__ float s_m[32][8], s_s[32][8];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int cl = lane & 7;
+    const int grp = warp * 4 + (lane >> 3);
+    const int64_t col = (int64_t)blockIdx.x * 8 + cl;
     const bool ok = col < n;
+    float m = -INFINITY, sum = 0.f;
+    if (ok) {
+        for (int c = grp; c < classes; c += 32) {
+            const float x = __ldg(z + (int64_t)c * n + col);
+            if (x > m) {
+                sum = sum * expf(m - x) + 1.f;
+                m = x;
+            } else {
+                sum += expf(x - m);
+            }
+        }
+    }
+    s_m[grp][cl] = m;
+    s_s[grp][cl] = sum;
+    __syncthreads();
     float mx = -INFINITY;
-    if (ok)
-        for (int c = warp; c < classes; c += 8) mx = fmaxf(mx, __ldg(z + (int64_t)c * n + col));
-    red[warp][lane] = mx;
-    __syncthreads();
-    mx = red[0][lane];
-    for (int w = 1; w < 8; ++w) mx = fmaxf(mx, red[w][lane]);
-    __syncthreads();
+    for (int g = 0; g < 32; ++g) mx = fmaxf(mx, s_m[g][cl]);
     float se = 0.f;
-    if (ok)
-        for (int c = warp; c < classes; c += 8) se += expf(__ldg(z + (int64_t)c * n + col) - mx);
-    red[warp][lane] = se;
-    __syncthreads();
-    se = 0.f;
-    for (int w = 0; w < 8; ++w) se += red[w][lane];
+    for (int g = 0; g < 32; ++g) {
+        const float mg = s_m[g][cl];
+        if (mg != -INFINITY) se += s_s[g][cl] * expf(mg - mx);
+    }
     if (!ok) return;
     const float inv = 1.f / se;
     const float inv_n = 1.f / (float)n;
     const int lab = __ldg(labels + col);
     const bool lab_ok = lab >= 0 && lab < classes;   // an invalid label gives a NaN loss
-    for (int c = warp; c < classes; c += 8) {
+    for (int c = grp; c < classes; c += 32) {
         const float p = expf(__ldg(z + (int64_t)c * n + col) - mx) * inv;
         dz[(int64_t)c * n + col] = (p - (c == lab ? 1.f : 0.f)) * inv_n;
     }
-    if (warp == 0)
+    if (grp == 0)
         per_sample[col] = lab_ok ? -((__ldg(z + (int64_t)lab * n + col) - mx) - logf(se)) : __int_as_float(0x7fc00000);
 }
 
@@ -230,7 +243,7 @@ int csrt_softmax_xent(const float *z, const int32_t *labels, int32_t classes, in
     CSRT_ARG(z && labels && dz && loss, "NULL pointer");
     cudaStream_t s = as_stream(stream);
     if (n > 0) {
-        softmax_xent_kernel<<<(unsigned)ceil_div<int64_t>(n, 32), 256, 0, s>>>(z, labels, classes, n, dz, loss + 1);
+        softmax_xent_kernel<<<(unsigned)ceil_div<int64_t>(n, 8), 256, 0, s>>>(z, labels, classes, n, dz, loss + 1);
         count_launch();
     }
     mean_kernel<<<1, 1024, 0, s>>>(loss + 1, n, loss);

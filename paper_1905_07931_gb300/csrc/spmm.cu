@@ -68,7 +68,32 @@ struct SpmmArgs {
     int32_t n_tiles;
     float *carry;     // [n_tiles][units][TN]
     int32_t *carry_row;  // [units]
+    // optional epilogue on each finished row i: + bias[i], then ReLU, then
+    // zero where mask[i, c] <= 0 (the ReLU backward of the layer below)
+    const float *bias;
+    int32_t relu;
+    const float *mask;
 };
+
+// The epilogue of one row segment held by a lane (VW floats at column c).
+template <int VW>
+__device__ __forceinline__ void spmm_epilogue(const SpmmArgs &a, int64_t row, int c, float (&v)[VW]) {
+    if (a.bias) {
+        const float b = __ldg(a.bias + row);
+#pragma unroll
+        for (int e = 0; e < VW; ++e) v[e] = __fadd_rn(v[e], b);
+    }
+    if (a.relu) {
+#pragma unroll
+        for (int e = 0; e < VW; ++e) v[e] = fmaxf(v[e], 0.f);
+    }
+    if (a.mask) {
+        const float *mp = a.mask + row * a.n + c;
+#pragma unroll
+        for (int e = 0; e < VW; ++e)
+            if (!(__ldg(mp + e) > 0.f)) v[e] = 0.f;
+    }
+}
 
 template <int VW, int NV>
 __device__ __forceinline__ void spmm_consume(const SpmmArgs &a, int64_t k, int64_t kend, int n0,
@@ -151,15 +176,22 @@ __global__ void __launch_bounds__(kSpThreads) spmm_merge_kernel(SpmmArgs a) {
 #pragma unroll
         for (int e = 0; e < VW; ++e) acc[v][e] = 0.f;
 
+    // a row that began in an earlier unit receives carries; the fix-up applies its epilogue
+    const bool first_row_cut = i0 < a.rows && k0 > __ldg(a.row_ptr + i0);
+    const bool epi = a.bias || a.relu || a.mask;
     int64_t k = k0;
     for (int i = i0; i < i1; ++i) {
         const int64_t kend = __ldg(a.row_ptr + i + 1);
         spmm_consume<VW, NV>(a, k, kend, n0, acc);
         k = kend;
         float *yrow = a.y + (int64_t)i * a.n + n0;
+        const bool apply = epi && !(i == i0 && first_row_cut);
 #pragma unroll
         for (int v = 0; v < NV; ++v) {
-            if (n0 + v * kStride < a.n) stv<VW>(yrow + v * kStride, acc[v]);
+            if (n0 + v * kStride < a.n) {
+                if (apply) spmm_epilogue<VW>(a, i, n0 + v * kStride, acc[v]);
+                stv<VW>(yrow + v * kStride, acc[v]);
+            }
 #pragma unroll
             for (int e = 0; e < VW; ++e) acc[v][e] = 0.f;
         }
@@ -193,12 +225,29 @@ __global__ void __launch_bounds__(256) spmm_fixup_kernel(SpmmArgs a) {
     for (int v = u; v < a.units && a.carry_row[v] == r; ++v)
         sum += a.carry[((int64_t)t * a.units + v) * TN + j];
     float *yp = a.y + (int64_t)r * a.n + col;
-    *yp = *yp + sum;
+    float out[1] = {*yp + sum};
+    if (a.bias || a.relu || a.mask) spmm_epilogue<1>(a, r, col, out);
+    *yp = out[0];
 }
 
 struct SpmmShape {
     int vw, nv, tn, n_tiles, units;
 };
+
+template <int VW, int NV>
+static int spmm_warps_per_sm() {
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return kWarpsPerSM;
+    if (cache[dev] == 0) {
+        int blocks = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, spmm_merge_kernel<VW, NV>, kSpThreads, 0) !=
+                cudaSuccess || blocks <= 0)
+            blocks = kWarpsPerSM / (kSpThreads / 32);
+        cache[dev] = imin(blocks * (kSpThreads / 32), kWarpsPerSM);
+    }
+    return cache[dev];
+}
 
 static SpmmShape spmm_shape(int32_t n, int64_t max_items, bool vec4_ok, bool vec2_ok) {
     SpmmShape s;
@@ -207,7 +256,10 @@ static SpmmShape spmm_shape(int32_t n, int64_t max_items, bool vec4_ok, bool vec
     else { s.vw = 1; s.nv = 1; }
     s.tn = 32 * s.vw * s.nv;
     s.n_tiles = (int)ceil_div<int64_t>(n, s.tn);
-    const int64_t target = (int64_t)num_sms() * kWarpsPerSM;
+    // one full wave of resident warps (a partial second wave would run at low occupancy)
+    const int wps = s.vw == 4 ? (s.nv == 2 ? spmm_warps_per_sm<4, 2>() : spmm_warps_per_sm<4, 1>())
+                    : s.vw == 2 ? spmm_warps_per_sm<2, 1>() : spmm_warps_per_sm<1, 1>();
+    const int64_t target = (int64_t)num_sms() * wps;
     int64_t units = ceil_div<int64_t>(target, s.n_tiles);
     units = imax<int64_t>(1, imin<int64_t>(units, max_items));
     s.units = (int)units;
@@ -223,7 +275,7 @@ size_t spmm_scratch_bytes(int32_t max_n) {
 
 static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *val, int32_t rows,
                        int64_t capacity, const float *x, int32_t n, float *y, void *ws, size_t ws_bytes,
-                       cudaStream_t s) {
+                       cudaStream_t s, const float *bias = nullptr, int32_t relu = 0, const float *mask = nullptr) {
     if (rows == 0 || n == 0) return CSRT_OK;
     const bool v4 = (n % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15) == 0;
     const bool v2 = (n % 2 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 7) == 0;
@@ -238,6 +290,9 @@ static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *
     a.y = y;
     a.units = sh.units;
     a.n_tiles = sh.n_tiles;
+    a.bias = bias;
+    a.relu = relu;
+    a.mask = mask;
     const size_t carry_floats = (size_t)sh.units * sh.n_tiles * sh.tn;
     a.carry = reinterpret_cast<float *>(ws_scratch(ws));
     a.carry_row = reinterpret_cast<int32_t *>(a.carry + ((carry_floats + 63) / 64) * 64);
@@ -403,6 +458,27 @@ int spmm_bwd_t(const csrt_csr *w, const float *dy, int32_t n, float *dx, void *w
     CSRT_ARG((dy && dx) || n == 0 || w->cols == 0, "dY or dX is NULL");
     return spmm_launch(w->t_row_ptr, w->t_col_idx, w->t_val, w->cols, w->capacity, dy, n, dx, ws, ws_bytes,
                        as_stream(stream));
+}
+
+int spmm_fwd_bias_act(const csrt_csr *w, const float *x, int32_t n, const float *bias, int32_t relu, float *y,
+                      void *ws, size_t ws_bytes, void *stream) {
+    int rc = check_csr_basic(w);
+    if (rc) return rc;
+    CSRT_ARG(n >= 0, "n < 0");
+    CSRT_ARG((x && y) || n == 0 || w->rows == 0, "X or Y is NULL");
+    return spmm_launch(w->row_ptr, w->col_idx, w->val, w->rows, w->capacity, x, n, y, ws, ws_bytes,
+                       as_stream(stream), bias, relu ? 1 : 0, nullptr);
+}
+
+int spmm_bwd_t_relu(const csrt_csr *w, const float *dy, int32_t n, const float *y_below, float *dx, void *ws,
+                    size_t ws_bytes, void *stream) {
+    int rc = check_csr_basic(w);
+    if (rc) return rc;
+    CSRT_ARG(w->t_row_ptr && w->t_col_idx && w->t_val, "transposed arrays not set");
+    CSRT_ARG(n >= 0, "n < 0");
+    CSRT_ARG((dy && dx && y_below) || n == 0 || w->cols == 0, "dY, dX or the mask is NULL");
+    return spmm_launch(w->t_row_ptr, w->t_col_idx, w->t_val, w->cols, w->capacity, dy, n, dx, ws, ws_bytes,
+                       as_stream(stream), nullptr, 0, y_below);
 }
 
 int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_t n, float *g_nnz, void *ws,

@@ -46,6 +46,9 @@ _SIGS = {
     "csr_transpose": [POINTER(csrt_csr), c_void_p, c_size_t, c_void_p],
     "spmm_fwd": [POINTER(csrt_csr), c_void_p, c_int32, c_void_p, c_void_p, c_size_t, c_void_p],
     "spmm_bwd_t": [POINTER(csrt_csr), c_void_p, c_int32, c_void_p, c_void_p, c_size_t, c_void_p],
+    "spmm_fwd_bias_act": [POINTER(csrt_csr), c_void_p, c_int32, c_void_p, c_int32, c_void_p, c_void_p, c_size_t,
+                          c_void_p],
+    "spmm_bwd_t_relu": [POINTER(csrt_csr), c_void_p, c_int32, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p],
     "weight_grad_dense": [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32, c_void_p,
                           c_size_t, c_void_p],
     "weight_grad_sddmm": [POINTER(csrt_csr), c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_size_t,
@@ -229,6 +232,25 @@ def spmm_bwd_t(w: CSR, dy: torch.Tensor, dx: torch.Tensor, ws: Workspace, stream
     _f32(dy, "dY", w.rows * n)
     _f32(dx, "dX", w.cols * n)
     _check(lib().spmm_bwd_t(w.struct, _ptr(dy), n, _ptr(dx), ws.ptr, ws.nbytes, _stream(stream)), "spmm_bwd_t")
+
+
+def spmm_fwd_bias_act(w: CSR, x: torch.Tensor, bias, relu: bool, y: torch.Tensor, ws: Workspace, stream=None):
+    n = x.shape[1] if x.dim() == 2 else x.numel() // max(w.cols, 1)
+    _f32(x, "X", w.cols * n)
+    _f32(y, "Y", w.rows * n)
+    if bias is not None:
+        _f32(bias, "bias", w.rows)
+    _check(lib().spmm_fwd_bias_act(w.struct, _ptr(x), n, _ptr(bias), 1 if relu else 0, _ptr(y), ws.ptr, ws.nbytes,
+                                   _stream(stream)), "spmm_fwd_bias_act")
+
+
+def spmm_bwd_t_relu(w: CSR, dy: torch.Tensor, y_below: torch.Tensor, dx: torch.Tensor, ws: Workspace, stream=None):
+    n = dy.shape[1] if dy.dim() == 2 else dy.numel() // max(w.rows, 1)
+    _f32(dy, "dY", w.rows * n)
+    _f32(dx, "dX", w.cols * n)
+    _f32(y_below, "y_below", w.cols * n)
+    _check(lib().spmm_bwd_t_relu(w.struct, _ptr(dy), n, _ptr(y_below), _ptr(dx), ws.ptr, ws.nbytes, _stream(stream)),
+           "spmm_bwd_t_relu")
 
 
 def weight_grad_dense(dy: torch.Tensor, x: torch.Tensor, g: torch.Tensor, ws: Workspace,

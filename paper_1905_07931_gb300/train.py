@@ -140,14 +140,12 @@ class SparseNet:
             kind = L["kind"]
             if kind == "fc":
                 W = L["W"][L["cur"]]
-                C.spmm_fwd(W, L["x"], L["y"], self.ws, s)
-                C.bias_act_fwd(L["y"], L["b"], L["relu"], s)
+                C.spmm_fwd_bias_act(W, L["x"], L["b"], L["relu"], L["y"], self.ws, s)
             elif kind == "conv":
                 ci, h, w = L["in_shape"]
                 C.im2col(L["x"], ci, self.batch, h, w, L["k"], L["cols"], s)
                 W = L["W"][L["cur"]]
-                C.spmm_fwd(W, L["cols"], L["y"], self.ws, s)
-                C.bias_act_fwd(L["y"], L["b"], L["relu"], s)
+                C.spmm_fwd_bias_act(W, L["cols"], L["b"], L["relu"], L["y"], self.ws, s)
             elif kind == "pool2":
                 c, h, w = L["shape"]
                 C.maxpool2_fwd(L["x"], c, self.batch, h, w, L["y"], L["idx"], s)
@@ -163,13 +161,16 @@ class SparseNet:
         self.forward()
         C.softmax_xent(self.logits, self.labels, self.dlogits, self.loss, s)
         d = self.dlogits
-        for L in reversed(self.layers):
+        d_masked = False   # d already carries the ReLU backward of the layer that produced it
+        for li in range(len(self.layers) - 1, -1, -1):
+            L = self.layers[li]
             kind = L["kind"]
             if kind in ("fc", "conv"):
                 W = L["W"][L["cur"]]
                 dpre = d
-                if L["relu"]:
+                if L["relu"] and not d_masked:
                     C.relu_bwd(dpre, L["y"], s)
+                d_masked = False
                 M, K = W.rows, W.cols
                 if phase == "prox":
                     G = L["G"] if self.grad_per_layer else self.G[: M * K].view(M, K)
@@ -178,7 +179,12 @@ class SparseNet:
                     C.weight_grad_sddmm(W, dpre, L["xmat"], L["g"], self.ws, s)
                 C.bias_grad_sgd(dpre, L["b"], eta, None, s)
                 if L["needs_dx"]:
-                    if kind == "fc":
+                    below = self.layers[li - 1] if li > 0 else None
+                    if kind == "fc" and below is not None and below["kind"] == "fc" and below["relu"]:
+                        # ReLU backward of the layer below fused into the transposed product
+                        C.spmm_bwd_t_relu(W, dpre, below["y"], L["dx"], self.ws, s)
+                        d_masked = True
+                    elif kind == "fc":
                         C.spmm_bwd_t(W, dpre, L["dx"], self.ws, s)
                     else:
                         ci, h, w = L["in_shape"]

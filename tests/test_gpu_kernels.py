@@ -181,6 +181,32 @@ def test_spmm_fwd_and_bwd_against_oracle(C, m, k, n, density, zipf):
     assert ws.status()[0] == 0
 
 
+@pytest.mark.parametrize("m,k,n,zipf", [(700, 900, 256, True), (129, 257, 70, False), (50, 40, 1, False),
+                                         (300, 784, 64, False)])
+def test_fused_epilogues_match_unfused(C, m, k, n, zipf):
+    rng = np.random.default_rng(m + k + n)
+    a = _sparse(rng, m, k, 0.1, zipf)
+    x = _dev(rng.standard_normal((k, n)).astype(F32))
+    dy = _dev(rng.standard_normal((m, n)).astype(F32))
+    bias = _dev(rng.standard_normal(m).astype(F32))
+    below = _dev(np.maximum(rng.standard_normal((k, n)), 0).astype(F32))
+    ws = _ws(C, m, k, n)
+    w = _gpu_csr(C, a, ws)
+    for relu in (False, True):
+        y_ref = torch.zeros(m, n, device="cuda")
+        C.spmm_fwd(w, x, y_ref, ws)
+        C.bias_act_fwd(y_ref, bias, relu)
+        y = torch.zeros(m, n, device="cuda")
+        C.spmm_fwd_bias_act(w, x, bias, relu, y, ws)
+        np.testing.assert_array_equal(y.cpu().numpy().view(np.uint32), y_ref.cpu().numpy().view(np.uint32))
+    dx_ref = torch.zeros(k, n, device="cuda")
+    C.spmm_bwd_t(w, dy, dx_ref, ws)
+    C.relu_bwd(dx_ref, below)
+    dx = torch.zeros(k, n, device="cuda")
+    C.spmm_bwd_t_relu(w, dy, below, dx, ws)
+    np.testing.assert_array_equal(dx.cpu().numpy().view(np.uint32), dx_ref.cpu().numpy().view(np.uint32))
+
+
 def test_spmm_is_deterministic(C):
     rng = np.random.default_rng(11)
     a = _sparse(rng, 700, 900, 0.08, zipf=True)
