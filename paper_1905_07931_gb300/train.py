@@ -171,6 +171,7 @@ class SparseNet:
                 if L["relu"] and not d_masked:
                     C.relu_bwd(dpre, L["y"], s)
                 d_masked = False
+                L["dpre"] = dpre   # dL/d(pre-activation) of this layer (a view kept for inspection)
                 M, K = W.rows, W.cols
                 if phase == "prox":
                     G = L["G"] if self.grad_per_layer else self.G[: M * K].view(M, K)

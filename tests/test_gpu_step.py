@@ -84,36 +84,65 @@ def _oracle_net(layers, net):
     return onet
 
 
-def _run_and_compare(C, net, layers, x_host, labels, eta, lam, phase, prec, gtol_scale=1.0):
+def _run_and_compare(C, net, layers, x_host, labels, eta, lam, phase, prec):
+    """One GPU step, checked against the oracle.
+
+    Kernel parity is checked on the GPU's own inputs: each layer's gradient
+    against the oracle fed the GPU's dL/dpre and layer input, the update
+    bit-exact against the oracle update fed the GPU's gradient. The chain as
+    a whole is checked against the oracle's own forward/backward: the loss
+    tightly, max-pool winners exactly except at near-ties (where either
+    winner is correct), dL/dpre loosely (fp32 vs fp64 through several layers).
+    """
     onet = _oracle_net(layers, net)
-    logits, cache = O.net_forward(onet, x_host, len(labels))
-    oloss, dz = O.softmax_xent(logits, labels)
-    ograds = O.net_backward(onet, cache, dz, phase)
+    batch = len(labels)
     loss = net.step(phase, eta, lam)
     torch.cuda.synchronize()
     assert net.ws.status()[0] == 0
+    logits, cache = O.net_forward(onet, x_host, batch)
+    for li, L in enumerate(layers):
+        if L["kind"] == "pool2":
+            gidx = net.layers[li]["idx"].cpu().numpy().reshape(cache[li]["idx"].shape)
+            diff = gidx != cache[li]["idx"]
+            if diff.any():
+                c, b, h, w = cache[li]["shape"]
+                xin = net.layers[li]["x"].cpu().numpy().reshape(c, b, h, w).astype(np.float64)
+                win = xin.reshape(c, b, h // 2, 2, w // 2, 2).transpose(0, 1, 2, 4, 3, 5).reshape(
+                    c, b, h // 2, w // 2, 4)
+                picked = np.take_along_axis(win, gidx[..., None].astype(np.int64), axis=-1)[..., 0]
+                best = win.max(axis=-1)
+                assert np.all(picked[diff] >= best[diff]), "GPU pooling picked a non-maximum"
+                assert diff.mean() < 1e-3, diff.mean()
+                cache[li]["idx"] = gidx.astype(np.int8)
+    oloss, dz = O.softmax_xent(logits, labels)
+    ograds = O.net_backward(onet, cache, dz, phase)
     got_loss = float(loss[0].item())
     assert abs(got_loss - oloss) <= 2e-5 * max(1.0, abs(oloss)), (got_loss, oloss)
     pl = [i for i, l in enumerate(layers) if l["kind"] in ("fc", "conv")]
     for pi, li in enumerate(pl):
         L = net.params[pi]
         og = ograds[li]
-        old = onet.params[li]
         if og is None:
             continue
-        n = og["x"].shape[1]
-        absx = np.abs(og["x"])
-        absd = np.abs(og["delta"])
+        old = onet.params[li]
+        W = old["W"]
+        M = W.rows
+        d_gpu = L["dpre"].cpu().numpy().reshape(M, -1).astype(np.float64)
+        x_gpu = L["xmat"].cpu().numpy().reshape(W.cols, -1).astype(np.float64)
+        n = x_gpu.shape[1]
+        scale = np.abs(og["delta"]).max() + 1e-30
+        assert np.abs(d_gpu - og["delta"]).max() <= 1e-3 * scale, f"dL/dpre of layer {pi}"
+        absx, absd = np.abs(x_gpu), np.abs(d_gpu)
         if phase == "prox":
             G = L["G"].cpu().numpy()
-            assert_close(G, og["G"], O.weight_grad_dense(absd, absx) * 1.01, n,
+            assert_close(G, O.weight_grad_dense(d_gpu, x_gpu), O.weight_grad_dense(absd, absx), n,
                          rtol=1e-3 if prec else 1e-4, tf32=bool(prec), what=f"G layer {pi}")
-            _assert_csr_bits(net.weights(pi), O.prox_update_compact(old["W"], G, eta, lam))
+            _assert_csr_bits(net.weights(pi), O.prox_update_compact(W, G, eta, lam))
         else:
-            w = old["W"]
-            g = L["g"].cpu().numpy()[: w.nnz]
-            assert_close(g, og["g"], O.weight_grad_sddmm(w, absd, absx) * 1.01, n, what=f"g layer {pi}")
-            _assert_csr_bits(net.weights(pi), O.debias_update(w, g, eta))
+            g = L["g"].cpu().numpy()[: W.nnz]
+            assert_close(g, O.weight_grad_sddmm(W, d_gpu, x_gpu), O.weight_grad_sddmm(W, absd, absx), n,
+                         what=f"g layer {pi}")
+            _assert_csr_bits(net.weights(pi), O.debias_update(W, g, eta))
     return got_loss
 
 
