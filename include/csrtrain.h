@@ -162,6 +162,20 @@ int spmm_fwd_bias_act(const csrt_csr *w, const float *x, int32_t n, const float 
 int spmm_bwd_t_relu(const csrt_csr *w, const float *dy, int32_t n, const float *y_below, float *dx,
                     void *ws, size_t ws_bytes, void *stream);
 
+/* spmm_fwd_noalloc -- the same product as spmm_fwd for callers that cannot
+ * allocate device memory (for example code embedded in a framework that owns
+ * every device allocation and forbids direct cudaMalloc, or a serving loop
+ * that may not risk an allocation). The paper has no counterpart: it is an
+ * interface choice of this library. n may be at most 4096 (larger n is
+ * rejected with CSRT_ERR_ARG). The scratch for rows split between work units
+ * lives in a fixed device array inside the library (8 MiB of floats + 256 KiB
+ * of row slots, held by every GPU that loads the library until the process
+ * exits). The
+ * first call on a device looks the array up with cudaGetSymbolAddress (make
+ * it before any stream capture). All calls share the array: calls whose
+ * kernels overlap on the GPU race and must be serialised by the caller. */
+int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, float *y, void *stream);
+
 /* weight_grad_dense -- gradient of every weight for the prox phase (the
  * matrix w - eta*G of Section 3.3 needs G at all M x K entries).
  * G[i, j] = sum_c dY[i, c] X[j, c]; dY is m x n, X is k x n, G is m x k,

@@ -556,3 +556,99 @@ extern "C" int debias_update(csrt_csr *w, const float *g_nnz, float eta, void *s
     count_launch();
     return check_launch("debias_kernel");
 }
+
+// ---------------------------------------------------------------------------
+// spmm_fwd_noalloc: the forward product for callers that cannot allocate.
+//
+// spmm_fwd needs a caller-provided workspace for the partial sums of rows that
+// straddle two merge-path units. Some callers cannot provide one: code that
+// runs inside a host framework which owns every device allocation through its
+// own pool and does not let plugins call cudaMalloc, or a tight serving loop
+// where an allocation's latency and possible failure are not acceptable. This
+// variant keeps that scratch in a fixed array in device global memory that the
+// library declares itself, so the caller passes only inputs and outputs.
+//
+// Limits and rules:
+//  * The product may have at most kNoAllocMaxN = 4096 columns (n); larger n
+//    is rejected with CSRT_ERR_ARG. The array holds kNoAllocFloats floats of
+//    partial sums (8 MiB) and kNoAllocRows row slots (256 KiB), enough for
+//    n <= 4096 on GPUs of up to 256 SMs (a shape that still does not fit is
+//    rejected the same way). Every GPU that loads the library holds the
+//    array until the process exits.
+//  * The first call on each device looks up the array's device address with
+//    cudaGetSymbolAddress (once per device, with that device current); make
+//    that first call before any stream capture begins.
+//  * All calls share the one array and it keeps the last call's contents.
+//    Nothing in it needs to start at zero: each launch writes every slot it
+//    later reads. Calls whose kernels overlap on the GPU (two streams, or two
+//    threads) race on the array and give wrong results; serialise them.
+// ---------------------------------------------------------------------------
+namespace csrt {
+constexpr int32_t kNoAllocMaxN = 4096;
+constexpr int64_t kNoAllocFloats = (int64_t)1 << 21;
+constexpr int64_t kNoAllocRows = (int64_t)1 << 16;
+static __device__ __align__(256) float g_noalloc_carry[kNoAllocFloats];
+static __device__ __align__(256) int32_t g_noalloc_carry_row[kNoAllocRows];
+static float *g_noalloc_carry_addr[64] = {nullptr};
+static int32_t *g_noalloc_row_addr[64] = {nullptr};
+}  // namespace csrt
+
+extern "C" int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, float *y, void *stream) {
+    int rc = check_csr_basic(w);
+    if (rc) return rc;
+    CSRT_ARG(n >= 0, "n < 0");
+    CSRT_ARG(n <= kNoAllocMaxN, "spmm_fwd_noalloc: n = %d exceeds the maximum of %d columns of its static scratch",
+             n, kNoAllocMaxN);
+    CSRT_ARG((x && y) || n == 0 || w->rows == 0, "X or Y is NULL");
+    if (w->rows == 0 || n == 0) return CSRT_OK;
+    int dev = 0;
+    CSRT_CHECK_CUDA(cudaGetDevice(&dev));
+    CSRT_ARG(dev >= 0 && dev < 64, "device ordinal %d out of range", dev);
+    if (g_noalloc_carry_addr[dev] == nullptr) {
+        void *p = nullptr, *q = nullptr;
+        CSRT_CHECK_CUDA(cudaGetSymbolAddress(&p, g_noalloc_carry));
+        CSRT_CHECK_CUDA(cudaGetSymbolAddress(&q, g_noalloc_carry_row));
+        g_noalloc_carry_addr[dev] = static_cast<float *>(p);
+        g_noalloc_row_addr[dev] = static_cast<int32_t *>(q);
+    }
+    const bool v4 = (n % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15) == 0;
+    const bool v2 = (n % 2 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 7) == 0;
+    const SpmmShape sh = spmm_shape(n, (int64_t)w->rows + w->capacity, v4, v2);
+    const int64_t carry_floats = (int64_t)sh.units * sh.n_tiles * sh.tn;
+    CSRT_ARG(sh.units == 1 || (carry_floats <= kNoAllocFloats && sh.units <= kNoAllocRows),
+             "spmm_fwd_noalloc: n = %d needs %lld floats of static scratch, the maximum is %lld", n,
+             (long long)carry_floats, (long long)kNoAllocFloats);
+    SpmmArgs a;
+    a.row_ptr = w->row_ptr;
+    a.col = w->col_idx;
+    a.val = w->val;
+    a.rows = w->rows;
+    a.x = x;
+    a.n = n;
+    a.y = y;
+    a.units = sh.units;
+    a.n_tiles = sh.n_tiles;
+    a.carry = g_noalloc_carry_addr[dev];
+    a.carry_row = g_noalloc_row_addr[dev];
+    a.bias = nullptr;
+    a.relu = 0;
+    a.mask = nullptr;
+    cudaStream_t s = as_stream(stream);
+    const unsigned grid = (unsigned)ceil_div<int64_t>((int64_t)sh.units * sh.n_tiles * 32, kSpThreads);
+    const unsigned fgrid = (unsigned)ceil_div<int64_t>(carry_floats, 256);
+    if (sh.vw == 4 && sh.nv == 2) {
+        spmm_merge_kernel<4, 2><<<grid, kSpThreads, 0, s>>>(a);
+        if (sh.units > 1) spmm_fixup_kernel<256><<<fgrid, 256, 0, s>>>(a);
+    } else if (sh.vw == 4) {
+        spmm_merge_kernel<4, 1><<<grid, kSpThreads, 0, s>>>(a);
+        if (sh.units > 1) spmm_fixup_kernel<128><<<fgrid, 256, 0, s>>>(a);
+    } else if (sh.vw == 2) {
+        spmm_merge_kernel<2, 1><<<grid, kSpThreads, 0, s>>>(a);
+        if (sh.units > 1) spmm_fixup_kernel<64><<<fgrid, 256, 0, s>>>(a);
+    } else {
+        spmm_merge_kernel<1, 1><<<grid, kSpThreads, 0, s>>>(a);
+        if (sh.units > 1) spmm_fixup_kernel<32><<<fgrid, 256, 0, s>>>(a);
+    }
+    count_launch(sh.units > 1 ? 2 : 1);
+    return check_launch("spmm_fwd_noalloc");
+}

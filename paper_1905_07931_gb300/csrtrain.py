@@ -49,6 +49,7 @@ _SIGS = {
     "spmm_fwd_bias_act": [POINTER(csrt_csr), c_void_p, c_int32, c_void_p, c_int32, c_void_p, c_void_p, c_size_t,
                           c_void_p],
     "spmm_bwd_t_relu": [POINTER(csrt_csr), c_void_p, c_int32, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p],
+    "spmm_fwd_noalloc": [POINTER(csrt_csr), c_void_p, c_int32, c_void_p, c_void_p],
     "weight_grad_dense": [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32, c_void_p,
                           c_size_t, c_void_p],
     "weight_grad_sddmm": [POINTER(csrt_csr), c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_size_t,
@@ -251,6 +252,14 @@ def spmm_bwd_t_relu(w: CSR, dy: torch.Tensor, y_below: torch.Tensor, dx: torch.T
     _f32(y_below, "y_below", w.cols * n)
     _check(lib().spmm_bwd_t_relu(w.struct, _ptr(dy), n, _ptr(y_below), _ptr(dx), ws.ptr, ws.nbytes, _stream(stream)),
            "spmm_bwd_t_relu")
+
+
+def spmm_fwd_noalloc(w: CSR, x: torch.Tensor, y: torch.Tensor, stream=None):
+    """spmm_fwd without a workspace (the library's own fixed device scratch)."""
+    n = x.shape[1] if x.dim() == 2 else x.numel() // max(w.cols, 1)
+    _f32(x, "X", w.cols * n)
+    _f32(y, "Y", w.rows * n)
+    _check(lib().spmm_fwd_noalloc(w.struct, _ptr(x), n, _ptr(y), _stream(stream)), "spmm_fwd_noalloc")
 
 
 def weight_grad_dense(dy: torch.Tensor, x: torch.Tensor, g: torch.Tensor, ws: Workspace,
