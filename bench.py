@@ -263,8 +263,12 @@ def op_bytes(name, info):
     nnz, nnz_out = info.get("nnz", 0), info.get("nnz_out", 0)
     if name == "spmm_fwd":
         return 8 * nnz + 4 * (M + 1) + 4 * n * (K + M)
+    if name == "spmm_fwd_bias_act":
+        return 8 * nnz + 4 * (M + 1) + 4 * n * (K + M) + 4 * M
     if name == "spmm_bwd_t":
         return 8 * nnz + 4 * (K + 1) + 4 * n * (K + M)
+    if name == "spmm_bwd_t_relu":
+        return 8 * nnz + 4 * (K + 1) + 4 * n * (2 * K + M)
     if name == "weight_grad_dense":
         return 4 * M * K + 4 * n * (M + K)
     if name == "weight_grad_sddmm":
@@ -452,11 +456,13 @@ def profile_ops(net, C, torch, eta, lam, flush):
     stream = torch.cuda.current_stream()
     records = []
     wrapped = {}
-    names = ["spmm_fwd", "spmm_bwd_t", "weight_grad_dense", "weight_grad_sddmm", "prox_update_compact",
-             "debias_update", "bias_act_fwd", "relu_bwd", "bias_grad_sgd", "softmax_xent"]
+    names = ["spmm_fwd", "spmm_bwd_t", "spmm_fwd_bias_act", "spmm_bwd_t_relu", "weight_grad_dense",
+             "weight_grad_sddmm", "prox_update_compact", "debias_update", "bias_act_fwd", "relu_bwd",
+             "bias_grad_sgd", "softmax_xent"]
     kernel_of = {"spmm_fwd": "spmm_merge_kernel", "spmm_bwd_t": "spmm_merge_kernel",
-                 "weight_grad_dense": "gemm", "weight_grad_sddmm": "sddmm_kernel",
-                 "prox_update_compact": "compact_kernel", "debias_update": "debias_kernel"}
+                 "spmm_fwd_bias_act": "spmm_merge_kernel", "spmm_bwd_t_relu": "spmm_merge_kernel",
+                 "weight_grad_dense": "gemm_tf32_tc_persistent_kernel", "weight_grad_sddmm": "sddmm_kernel",
+                 "prox_update_compact": "prox_rows_kernel", "debias_update": "debias_kernel"}
     layer_of = {}
     for i, L in enumerate(net.params):
         for W in L["W"]:
@@ -475,9 +481,10 @@ def profile_ops(net, C, torch, eta, lam, flush):
                 info = {}
                 W = a[0] if a and isinstance(a[0], C.CSR) else None
                 li = layer_of.get(id(W)) if W is not None else None
-                if nm in ("spmm_fwd", "spmm_bwd_t", "weight_grad_sddmm", "prox_update_compact", "debias_update"):
+                if nm in ("spmm_fwd", "spmm_bwd_t", "spmm_fwd_bias_act", "spmm_bwd_t_relu", "weight_grad_sddmm",
+                          "prox_update_compact", "debias_update"):
                     info = {"M": W.rows, "K": W.cols, "W": W}
-                    if nm in ("spmm_fwd", "spmm_bwd_t", "weight_grad_sddmm"):
+                    if nm in ("spmm_fwd", "spmm_bwd_t", "spmm_fwd_bias_act", "spmm_bwd_t_relu", "weight_grad_sddmm"):
                         info["n"] = a[1].shape[1] if a[1].dim() == 2 else 0
                     if nm == "prox_update_compact":
                         info["W_out"] = a[4]
