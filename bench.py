@@ -282,6 +282,25 @@ def op_bytes(name, info):
 
 
 # ---------------------------------------------------------------------------
+# Multi-rank bookkeeping (replicas: no collective on the data path)
+# ---------------------------------------------------------------------------
+
+def max_over_ranks(x: float, world: int, device="cpu") -> float:
+    """The largest value of x over all ranks (the slowest rank's timed region)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank_per_step: int, steps: int, world: int, max_total_ms: float) -> float:
+    """Units processed by all ranks divided by the slowest rank's time."""
+    return world * steps * units_per_rank_per_step / (max_total_ms / 1e3)
+
+
+# ---------------------------------------------------------------------------
 # Our arm
 # ---------------------------------------------------------------------------
 
@@ -369,12 +388,8 @@ def main():
     if world > 1:
         dist.barrier()
     times_ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
-    total_ms = sum(times_ms)
-    tot = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(tot, op=dist.ReduceOp.MAX)
-    total_max_ms = float(tot.item())
-    value = world * args.steps * BATCH / (total_max_ms / 1e3)
+    total_max_ms = max_over_ranks(sum(times_ms), world, "cuda")
+    value = whole_job_rate(BATCH, args.steps, world, total_max_ms)
     flags, _ = net.ws.status()
     if flags:
         raise SystemExit(f"device status {flags} after the timed steps")
@@ -393,11 +408,8 @@ def main():
         loss_host.copy_(net.loss[:1], non_blocking=True)
         e_ends[i].record(stream)
     torch.cuda.synchronize()
-    e2e_ms = sum(a.elapsed_time(b) for a, b in zip(e_starts, e_ends))
-    et = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(et, op=dist.ReduceOp.MAX)
-    e2e_value = world * args.steps * BATCH / (float(et.item()) / 1e3)
+    e2e_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in zip(e_starts, e_ends)), world, "cuda")
+    e2e_value = whole_job_rate(BATCH, args.steps, world, e2e_ms)
 
     # roofline of the dominant kernel
     peaks, peak_kind = measured_peaks()

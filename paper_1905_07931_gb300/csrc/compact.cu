@@ -581,7 +581,8 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
                     const float z = __fsub_rn(ww[j], __fmul_rn(eta, gg[j]));
                     const bool k = fabsf(z) > thr;
                     nonfinite |= z != z;
-                    o[j] = k ? (z > 0.f ? __fsub_rn(z, thr) : __fadd_rn(z, thr)) : __int_as_float(0x7fc00000);
+                    // z - sgn(z)*thr: z - thr for z > 0, z + thr for z < 0 (same rounding)
+                    o[j] = k ? __fsub_rn(z, copysignf(thr, z)) : __int_as_float(0x7fc00000);
                     cnt += k;
                 }
                 *wp = make_float4(o[0], o[1], o[2], o[3]);
@@ -611,7 +612,6 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
     int row = e_beg / K;
     int col = e_beg - row * K + 4 * lane;
     while (col >= K) { col -= K; ++row; }
-    const unsigned lt = (1u << lane) - 1u;
     for (int base = e_beg; base < e_end; base += 128) {
         const int b = base + 4 * lane;
         const bool in = b < e_end;
@@ -620,34 +620,43 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
                                                                                    __int_as_float(0x7fc00000),
                                                                                    __int_as_float(0x7fc00000));
         const float vv[4] = {v.x, v.y, v.z, v.w};
-        unsigned m[4];
-        uint32_t p = pos, step = 0;
+        // keep bits of this lane's four entries; warp scan of their counts gives the ranks
+        const unsigned nib = (unsigned)(vv[0] == vv[0]) | ((unsigned)(vv[1] == vv[1]) << 1) |
+                             ((unsigned)(vv[2] == vv[2]) << 2) | ((unsigned)(vv[3] == vv[3]) << 3);
+        const uint32_t c = __popc(nib);
+        uint32_t incl = c;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            m[j] = __ballot_sync(0xffffffffu, vv[j] == vv[j]);
-            p += __popc(m[j] & lt);
-            step += __popc(m[j]);
+        for (int off = 1; off < 32; off <<= 1) {
+            const uint32_t t = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += t;
         }
+        uint32_t p = pos + incl - c;
         if (in && col == 0) a.out_row_ptr[r0 + row] = (int32_t)min(p, cap);
-        if (kBits && in && (lane & 7) == 0) {
-            const int q = lane >> 3;   // word q of this step = lanes 8q .. 8q+7
-            const uint32_t word = spread8(m[0] >> (8 * q)) | (spread8(m[1] >> (8 * q)) << 1) |
-                                  (spread8(m[2] >> (8 * q)) << 2) | (spread8(m[3] >> (8 * q)) << 3);
-            const int64_t wi = (int64_t)(r0 + row) * wpr + (col >> 5);
-            keepbits[wi] = word;
-            wordpos[wi] = (int32_t)p;
-        }
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            if (vv[j] == vv[j]) {
-                if (p < cap) {
-                    a.out_col[p] = col + j;
-                    a.out_val[p] = vv[j];
-                }
-                ++p;
+        if (kBits) {
+            // 32-entry word of lanes 8q .. 8q+7 (four bits per lane, in order)
+            uint32_t word = nib << (4 * (lane & 7));
+            word |= __shfl_xor_sync(0xffffffffu, word, 1);
+            word |= __shfl_xor_sync(0xffffffffu, word, 2);
+            word |= __shfl_xor_sync(0xffffffffu, word, 4);
+            if (in && (lane & 7) == 0) {
+                const int64_t wi = (int64_t)(r0 + row) * wpr + (col >> 5);
+                keepbits[wi] = word;
+                wordpos[wi] = (int32_t)p;
             }
         }
-        pos += step;
+        if (nib) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                if ((nib >> j) & 1u) {
+                    if (p < cap) {
+                        a.out_col[p] = col + j;
+                        a.out_val[p] = vv[j];
+                    }
+                    ++p;
+                }
+            }
+        }
+        pos += __shfl_sync(0xffffffffu, incl, 31);
         col += 128;
         while (col >= K) { col -= K; ++row; }
     }
