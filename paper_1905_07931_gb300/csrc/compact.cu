@@ -335,6 +335,41 @@ __global__ void __launch_bounds__(kCThreads) compact_kernel(CompactArgs a) {
 constexpr int kRowBudget = 8192;     // entries per tile when rows are short
 constexpr int kRowMaxK = 16384;      // longest row the row-tile path takes
 
+constexpr unsigned kRowWaitLimit = 1u << 22;
+
+__device__ __forceinline__ uint32_t cvta_smem(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// Bounded wait for the phase with the given parity of an mbarrier.
+__device__ __forceinline__ bool row_mbar_wait(uint64_t *bar, uint32_t parity) {
+    const uint32_t addr = cvta_smem(bar);
+    for (unsigned i = 0; i < kRowWaitLimit; ++i) {
+        uint32_t done;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            " selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(done)
+            : "r"(addr), "r"(parity)
+            : "memory");
+        if (done) return true;
+        if (i > 32) __nanosleep(32);
+    }
+    return false;
+}
+
+// Thread 0 only: stream `bytes` (16-byte aligned source, multiple of 16) into
+// shared memory with one bulk asynchronous copy that completes on `bar`.
+__device__ __forceinline__ void bulk_load(float *dst, const float *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(cvta_smem(bar)), "r"(bytes)
+                 : "memory");
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     cvta_smem(dst)),
+                 "l"(src), "r"(bytes), "r"(cvta_smem(bar))
+                 : "memory");
+}
+
 struct Keep4 {
     bool k[4];
     float v[4];
@@ -516,77 +551,106 @@ template <bool kBits>
 __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, int32_t rows_per_tile,
                                                                   uint32_t *__restrict__ keepbits,
                                                                   int32_t *__restrict__ wordpos, int32_t wpr) {
-    extern __shared__ __align__(16) float row_smem[];
-    float *wt = row_smem;
-    int32_t *s_rp = reinterpret_cast<int32_t *>(row_smem + rows_per_tile * a.cols);
+    // shared: the tile's G (bulk-copied), then z in place, then the kept values
+    // (NaN = dropped); a bitmask of the positions that hold a stored weight;
+    // the tile's row pointers.
+    extern __shared__ __align__(128) float row_smem[];
+    float *tile_v = row_smem;
+    const int tile_cap = rows_per_tile * a.cols;
+    uint32_t *onbits = reinterpret_cast<uint32_t *>(row_smem + tile_cap);
+    int32_t *s_rp = reinterpret_cast<int32_t *>(onbits + (tile_cap + 31) / 32);
+    __shared__ __align__(8) uint64_t s_bar;
     __shared__ uint32_t s_wtot[kCThreads / 32];
     __shared__ uint32_t s_excl;
     __shared__ unsigned int s_tile;
+    __shared__ int s_fail;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int K = a.cols;
-    if (tid == 0) s_tile = atomicAdd(&a.hdr->ticket, 1u);
+    if (tid == 0) {
+        s_fail = 0;
+        const unsigned t = atomicAdd(&a.hdr->ticket, 1u);
+        s_tile = t;
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(cvta_smem(&s_bar)) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        if (t < a.num_tiles) {
+            const int64_t r0 = (int64_t)t * rows_per_tile;
+            const int64_t nrows = imin<int64_t>(rows_per_tile, a.rows - r0);
+            bulk_load(tile_v, a.src + r0 * K, (uint32_t)(nrows * K * 4), &s_bar);
+        }
+    }
     __syncthreads();
     const int64_t tile = s_tile;
     if (tile >= a.num_tiles) return;
     const int r0 = (int)(tile * rows_per_tile);
     const int nrows = imin(rows_per_tile, a.rows - r0);
     const int n_el = nrows * K;
-    const float *g = a.src + (int64_t)r0 * K;
     const float eta = a.eta, thr = a.thr;
 
+    // while G streams in: row pointers, cleared bitmask, this thread's old entries
     for (int i = tid; i <= nrows; i += kCThreads) s_rp[i] = a.in_row_ptr[r0 + i];
-    {
-        float4 *w4 = reinterpret_cast<float4 *>(wt);
-        for (int i = tid; i < n_el / 4; i += kCThreads) w4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
+    for (int i = tid; i < (n_el + 31) / 32; i += kCThreads) onbits[i] = 0u;
     __syncthreads();
-    {
-        const int32_t s0 = s_rp[0], s1 = s_rp[nrows];
-        for (int32_t k = s0 + tid; k < s1; k += kCThreads) {
-            int lo = 0, hi = nrows - 1;
-            while (lo < hi) {
-                const int mid = (lo + hi + 1) >> 1;
-                if (s_rp[mid] <= k) lo = mid; else hi = mid - 1;
+    const int32_t s0 = s_rp[0], s1 = s_rp[nrows];
+    constexpr int kOld = 4;   // old entries held per thread per pass
+    bool waited = false;
+    for (int32_t kb = s0; kb < s1; kb += kOld * kCThreads) {
+        int32_t pos_e[kOld];
+        float wv[kOld];
+#pragma unroll
+        for (int q = 0; q < kOld; ++q) {
+            const int32_t k = kb + q * kCThreads + tid;
+            pos_e[q] = -1;
+            wv[q] = 0.f;
+            if (k < s1) {
+                int lo = 0, hi = nrows - 1;
+                while (lo < hi) {
+                    const int mid = (lo + hi + 1) >> 1;
+                    if (s_rp[mid] <= k) lo = mid; else hi = mid - 1;
+                }
+                pos_e[q] = lo * K + __ldg(a.in_col + k);
+                wv[q] = __ldg(a.in_val + k);
             }
-            wt[lo * K + __ldg(a.in_col + k)] = __ldg(a.in_val + k);
+        }
+        if (!waited) {   // the first batch of old entries was loaded while G streamed in
+            if (!row_mbar_wait(&s_bar, 0)) s_fail = 1;
+            waited = true;
+        }
+#pragma unroll
+        for (int q = 0; q < kOld; ++q) {
+            if (pos_e[q] >= 0) {
+                const int e = pos_e[q];
+                tile_v[e] = __fsub_rn(wv[q], __fmul_rn(eta, tile_v[e]));   // z of a stored weight
+                atomicOr(&onbits[e >> 5], 1u << (e & 31));
+            }
         }
     }
+    if (!waited && !row_mbar_wait(&s_bar, 0)) s_fail = 1;
     __syncthreads();
 
     const int seg = ((n_el + 8 * 128 - 1) / (8 * 128)) * 128;
     const int e_beg = imin(warp * seg, n_el), e_end = imin(e_beg + seg, n_el);
 
-    // pass 1: evaluate once, park results, count
+    // pass 1: z (-eta*G off the pattern), keep, kept value parked in place, count
     uint32_t cnt = 0;
     bool nonfinite = false;
-    for (int base = e_beg; base < e_end; base += 4 * 128) {
-        float4 gv[4];
+    for (int b = e_beg + 4 * lane; b - 4 * lane < e_end; b += 128) {
+        if (b < e_end) {
+            float4 *vp = reinterpret_cast<float4 *>(tile_v + b);
+            const float4 t4 = *vp;
+            const unsigned on = (onbits[b >> 5] >> (b & 31)) & 0xFu;
+            const float tv[4] = {t4.x, t4.y, t4.z, t4.w};
+            float o[4];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int b = base + 128 * u + 4 * lane;
-            gv[u] = b < e_end ? ldg_f4(g + b) : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int b = base + 128 * u + 4 * lane;
-            if (b < e_end) {
-                float4 *wp = reinterpret_cast<float4 *>(wt + b);
-                const float4 w = *wp;
-                const float gg[4] = {gv[u].x, gv[u].y, gv[u].z, gv[u].w};
-                const float ww[4] = {w.x, w.y, w.z, w.w};
-                float o[4];
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const float z = __fsub_rn(ww[j], __fmul_rn(eta, gg[j]));
-                    const bool k = fabsf(z) > thr;
-                    nonfinite |= z != z;
-                    // z - sgn(z)*thr: z - thr for z > 0, z + thr for z < 0 (same rounding)
-                    o[j] = k ? __fsub_rn(z, copysignf(thr, z)) : __int_as_float(0x7fc00000);
-                    cnt += k;
-                }
-                *wp = make_float4(o[0], o[1], o[2], o[3]);
+            for (int j = 0; j < 4; ++j) {
+                // off the pattern w = +0: z = fl(0 - fl(eta*G)) (its sign is irrelevant: zero is dropped)
+                const float z = ((on >> j) & 1u) ? tv[j] : -__fmul_rn(eta, tv[j]);
+                const bool k = fabsf(z) > thr;
+                nonfinite |= z != z;
+                o[j] = k ? __fsub_rn(z, copysignf(thr, z)) : __int_as_float(0x7fc00000);
+                cnt += k;
             }
+            *vp = make_float4(o[0], o[1], o[2], o[3]);
         }
     }
 #pragma unroll
@@ -615,7 +679,7 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
     for (int base = e_beg; base < e_end; base += 128) {
         const int b = base + 4 * lane;
         const bool in = b < e_end;
-        const float4 v = in ? *reinterpret_cast<const float4 *>(wt + b) : make_float4(__int_as_float(0x7fc00000),
+        const float4 v = in ? *reinterpret_cast<const float4 *>(tile_v + b) : make_float4(__int_as_float(0x7fc00000),
                                                                                    __int_as_float(0x7fc00000),
                                                                                    __int_as_float(0x7fc00000),
                                                                                    __int_as_float(0x7fc00000));
@@ -669,6 +733,10 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
         }
     }
     if (__syncthreads_or(nonfinite) && tid == 0) dev_flag(a.hdr, CSRT_DEV_NONFINITE);
+    if (tid == 0 && s_fail) {
+        dev_flag(a.hdr, CSRT_DEV_TIMEOUT);
+        a.hdr->timeout_site = 3;
+    }
 }
 
 // Returns through *bits_done whether the prox kernel emitted the keep bitmask
@@ -708,12 +776,13 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
     a.status = status;
     a.num_tiles = tiles;
     if (row_path) {
-        const size_t smem = prox ? ((size_t)rows_per_tile * cols + rows_per_tile + 1) * sizeof(float) : 0;
+        const size_t tile_cap = (size_t)rows_per_tile * cols;
+        const size_t smem = prox ? (tile_cap + (tile_cap + 31) / 32 + rows_per_tile + 1) * sizeof(float) : 0;
         static bool attr_done[64] = {false};
         int dev = 0;
         cudaGetDevice(&dev);
         if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-            const int max_smem = (int)((size_t)(kRowMaxK + kRowBudget + 1) * sizeof(float));
+            const int max_smem = (int)((size_t)(kRowMaxK + kRowMaxK / 32 + kRowBudget + 1) * sizeof(float));
             CSRT_CHECK_CUDA(cudaFuncSetAttribute(prox_rows_kernel<true>,
                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem));
             CSRT_CHECK_CUDA(cudaFuncSetAttribute(prox_rows_kernel<false>,

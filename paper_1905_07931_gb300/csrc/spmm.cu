@@ -208,26 +208,31 @@ __global__ void __launch_bounds__(kSpThreads) spmm_merge_kernel(SpmmArgs a) {
     }
 }
 
-// Adds the carries of every cut row, in unit order, to that row of Y.
+// Adds the carries of every cut row, in unit order, to that row of Y. One warp
+// per (unit, n-tile): warps whose unit is not the first carry of its row leave
+// at once; the first one sums the row's carries column by column.
 template <int TN>
 __global__ void __launch_bounds__(256) spmm_fixup_kernel(SpmmArgs a) {
-    const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const int64_t per_tile = (int64_t)a.units * TN;
-    if (tid >= per_tile * a.n_tiles) return;
-    const int t = (int)(tid / per_tile);
-    const int u = (int)((tid % per_tile) / TN);
-    const int j = (int)(tid % TN);
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (gw >= (int64_t)a.units * a.n_tiles) return;
+    const int t = (int)(gw / a.units);
+    const int u = (int)(gw % a.units);
     const int r = a.carry_row[u];
     if (r < 0 || (u > 0 && a.carry_row[u - 1] == r)) return;  // not the first carry of its row
-    const int col = t * TN + j;
-    if (col >= a.n) return;
-    float sum = 0.f;
-    for (int v = u; v < a.units && a.carry_row[v] == r; ++v)
-        sum += a.carry[((int64_t)t * a.units + v) * TN + j];
-    float *yp = a.y + (int64_t)r * a.n + col;
-    float out[1] = {*yp + sum};
-    if (a.bias || a.relu || a.mask) spmm_epilogue<1>(a, r, col, out);
-    *yp = out[0];
+    int last = u;
+    while (last + 1 < a.units && a.carry_row[last + 1] == r) ++last;
+    const bool epi = a.bias || a.relu || a.mask;
+    for (int j = lane; j < TN; j += 32) {
+        const int col = t * TN + j;
+        if (col >= a.n) break;
+        float sum = 0.f;
+        for (int v = u; v <= last; ++v) sum += a.carry[((int64_t)t * a.units + v) * TN + j];
+        float *yp = a.y + (int64_t)r * a.n + col;
+        float out[1] = {*yp + sum};
+        if (epi) spmm_epilogue<1>(a, r, col, out);
+        *yp = out[0];
+    }
 }
 
 struct SpmmShape {
@@ -308,7 +313,7 @@ static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *
         spmm_merge_kernel<VW, NV><<<grid, kSpThreads, 0, s>>>(a);                            \
         count_launch();                                                                      \
         if (sh.units > 1) {                                                                  \
-            const int64_t ft = (int64_t)sh.units * sh.n_tiles * (32 * VW * NV);              \
+            const int64_t ft = (int64_t)sh.units * sh.n_tiles * 32;                            \
             spmm_fixup_kernel<32 * VW * NV><<<(unsigned)ceil_div<int64_t>(ft, 256), 256, 0, s>>>(a); \
             count_launch();                                                                  \
         }                                                                                    \
@@ -635,7 +640,7 @@ extern "C" int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, fl
     a.mask = nullptr;
     cudaStream_t s = as_stream(stream);
     const unsigned grid = (unsigned)ceil_div<int64_t>((int64_t)sh.units * sh.n_tiles * 32, kSpThreads);
-    const unsigned fgrid = (unsigned)ceil_div<int64_t>(carry_floats, 256);
+    const unsigned fgrid = (unsigned)ceil_div<int64_t>((int64_t)sh.units * sh.n_tiles * 32, 256);
     if (sh.vw == 4 && sh.nv == 2) {
         spmm_merge_kernel<4, 2><<<grid, kSpThreads, 0, s>>>(a);
         if (sh.units > 1) spmm_fixup_kernel<256><<<fgrid, 256, 0, s>>>(a);
