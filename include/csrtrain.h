@@ -204,6 +204,20 @@ int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_
 int prox_update_compact(const csrt_csr *w_in, const float *g, float eta, float lambda,
                         csrt_csr *w_out, void *ws, size_t ws_bytes, void *stream);
 
+/* weight_grad_prox_update -- weight_grad_dense followed by
+ * prox_update_compact without writing G: the tensor-core GEMM's epilogue forms
+ * z = w - eta*G from the accumulator, applies the soft threshold of Section
+ * 2.2 (Eq. prox, Section 3.3) and stages the kept entries, which a placement
+ * pass compacts into w_out (and its transposed arrays when set). The result is
+ * bit-identical to weight_grad_dense(precision) + prox_update_compact.
+ * The fused path runs for precision CSRT_PREC_TF32 on tcgen05 GPUs with
+ * n % 4 == 0, rows and cols >= 64, cols % 32 == 0, cols <= 16384 and 16-byte
+ * aligned dY and X; otherwise the two calls run unfused through g_scratch
+ * (M x K floats, may be NULL when the fused path applies). */
+int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, const float *x, int32_t n,
+                            float eta, float lambda, int32_t precision, float *g_scratch,
+                            csrt_csr *w_out, void *ws, size_t ws_bytes, void *stream);
+
 /* debias_update -- the retraining step of Section 2.4 / Section 4.3 (zero
  * weights fixed and not updated): val[k] <- fl32(val[k] - fl32(eta*g_nnz[k]))
  * for every stored entry; row_ptr and col_idx are untouched, and a value

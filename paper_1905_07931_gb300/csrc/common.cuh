@@ -64,6 +64,7 @@ size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
 size_t spmm_scratch_bytes(int32_t max_n);
 size_t sddmm_scratch_bytes(int64_t capacity, int32_t max_n);
 size_t gemm_scratch_bytes(int32_t m, int32_t k, int32_t max_n);
+size_t fused_prox_scratch_bytes(int32_t rows, int32_t cols);
 
 // Internal entry used by csr_from_dense / prox_update_compact.
 int transpose_impl(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s);

@@ -1064,15 +1064,14 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
     }
 }
 
-// Transposed copy from the keep bitmask; scratch: [status][keepbits][wordpos][cnt][coltot].
-static int transpose_from_bits(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s) {
+// Transposed copy from a keep bitmask and word positions (cols % 32 == 0);
+// `scratch` holds the per-block column counts and the column totals.
+int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t *wordpos, void *scratch,
+                            size_t scratch_bytes, cudaStream_t s) {
     const int32_t rows = w->rows, cols = w->cols;
     const int32_t wpr = cols / 32;
-    const int64_t elems = (int64_t)rows * cols;
-    char *base = ws_scratch(ws);
-    const uint32_t *keepbits = reinterpret_cast<const uint32_t *>(base + status_bytes(elems));
-    const int32_t *wordpos = reinterpret_cast<const int32_t *>(base + status_bytes(elems) + bits_bytes(rows, cols));
-    int32_t *cnt = reinterpret_cast<int32_t *>(base + status_bytes(elems) + 2 * bits_bytes(rows, cols));
+    CSRT_ARG(scratch_bytes >= transpose_scratch_bytes(rows, cols), "scratch too small for the transposed copy");
+    int32_t *cnt = static_cast<int32_t *>(scratch);
     const int nb = (int)ceil_div<int64_t>(rows, 32);
     int32_t *coltot = cnt + (int64_t)nb * cols;
     const int64_t warps = (int64_t)nb * wpr;
@@ -1084,6 +1083,24 @@ static int transpose_from_bits(csrt_csr *w, void *ws, size_t ws_bytes, cudaStrea
                                           w->t_col_idx, w->t_val, w->t_pos, w->capacity);
     count_launch(4);
     return check_launch("transpose-from-bits kernels");
+}
+
+// Prox-kernel layout of the workspace: [status][keepbits][wordpos][cnt][coltot].
+static int transpose_from_bits(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s) {
+    const int32_t rows = w->rows, cols = w->cols;
+    const int64_t elems = (int64_t)rows * cols;
+    char *base = ws_scratch(ws);
+    const uint32_t *keepbits = reinterpret_cast<const uint32_t *>(base + status_bytes(elems));
+    const int32_t *wordpos = reinterpret_cast<const int32_t *>(base + status_bytes(elems) + bits_bytes(rows, cols));
+    char *scratch = base + status_bytes(elems) + 2 * bits_bytes(rows, cols);
+    return transpose_from_bits_ext(w, keepbits, wordpos, scratch, transpose_scratch_bytes(rows, cols), s);
+}
+
+// Exclusive scan of n int32 values into out[0..n] (out[n] = total), one block.
+int scan_exclusive_i32(const int32_t *in, int32_t n, int32_t *out, cudaStream_t s) {
+    scan_single_block_kernel<<<1, 1024, 0, s>>>(in, n, out);
+    count_launch();
+    return check_launch("scan_single_block_kernel");
 }
 
 int transpose_impl(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s) {

@@ -57,6 +57,8 @@ _SIGS = {
     "prox_update_compact": [POINTER(csrt_csr), c_void_p, c_float, c_float, POINTER(csrt_csr), c_void_p,
                             c_size_t, c_void_p],
     "debias_update": [POINTER(csrt_csr), c_void_p, c_float, c_void_p],
+    "weight_grad_prox_update": [POINTER(csrt_csr), c_void_p, c_void_p, c_int32, c_float, c_float, c_int32, c_void_p,
+                                POINTER(csrt_csr), c_void_p, c_size_t, c_void_p],
     "csrt_bias_act_fwd": [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p],
     "csrt_relu_bwd": [c_void_p, c_void_p, c_int64, c_void_p],
     "csrt_bias_grad_sgd": [c_void_p, c_int32, c_int32, c_void_p, c_float, c_void_p, c_void_p],
@@ -289,6 +291,18 @@ def prox_update_compact(w_in: CSR, g: torch.Tensor, eta: float, lam: float, w_ou
     _f32(g, "G", w_in.rows * w_in.cols)
     _check(lib().prox_update_compact(w_in.struct, _ptr(g), float(eta), float(lam), w_out.struct, ws.ptr,
                                      ws.nbytes, _stream(stream)), "prox_update_compact")
+
+
+def weight_grad_prox_update(w_in: CSR, dy: torch.Tensor, x: torch.Tensor, eta: float, lam: float, w_out: CSR,
+                            ws: Workspace, precision: int = CSRT_PREC_TF32, g_scratch=None, stream=None):
+    n = dy.shape[1]
+    _f32(dy, "dY", w_in.rows * n)
+    _f32(x, "X", w_in.cols * n)
+    if g_scratch is not None:
+        _f32(g_scratch, "g_scratch", w_in.rows * w_in.cols)
+    _check(lib().weight_grad_prox_update(w_in.struct, _ptr(dy), _ptr(x), n, float(eta), float(lam), int(precision),
+                                         _ptr(g_scratch), w_out.struct, ws.ptr, ws.nbytes, _stream(stream)),
+           "weight_grad_prox_update")
 
 
 def debias_update(w: CSR, g: torch.Tensor, eta: float, stream=None):

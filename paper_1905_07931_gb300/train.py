@@ -31,13 +31,17 @@ from . import csrtrain as C
 
 class SparseNet:
     def __init__(self, layers, dense_weights, biases, batch: int, in_shape, *, device="cuda",
-                 precision: int = C.CSRT_PREC_TF32, stream=None, grad_per_layer: bool = False):
+                 precision: int = C.CSRT_PREC_TF32, stream=None, grad_per_layer: bool = False,
+                 fused: bool = True):
         """layers: layer dicts; dense_weights/biases: numpy arrays, one per fc/conv
         layer (weights M x K, zero off the initial pattern); in_shape: (K,) for an
         fc-first net or (C, H, W) for a conv-first net. The dense gradients of
         all layers share one buffer unless grad_per_layer is set (then each
         layer's G stays readable after the step)."""
         self.grad_per_layer = grad_per_layer
+        # the prox phase applies the update in the gradient GEMM's epilogue (G is
+        # not written) unless each layer's G is to stay readable
+        self.fused = fused and not grad_per_layer
         self.layers = [dict(l) for l in layers]
         self.batch = int(batch)
         self.device = device
@@ -175,7 +179,8 @@ class SparseNet:
                 M, K = W.rows, W.cols
                 if phase == "prox":
                     G = L["G"] if self.grad_per_layer else self.G[: M * K].view(M, K)
-                    C.weight_grad_dense(dpre, L["xmat"], G, self.ws, self.precision, s)
+                    if not self.fused:
+                        C.weight_grad_dense(dpre, L["xmat"], G, self.ws, self.precision, s)
                 else:
                     C.weight_grad_sddmm(W, dpre, L["xmat"], L["g"], self.ws, s)
                 C.bias_grad_sgd(dpre, L["b"], eta, None, s)
@@ -193,7 +198,10 @@ class SparseNet:
                         C.col2im(L["dcols"], ci, self.batch, h, w, L["k"], L["dx"], s)
                 if phase == "prox":
                     Wn = L["W"][1 - L["cur"]]
-                    C.prox_update_compact(W, G, eta, lam, Wn, self.ws, s)
+                    if self.fused:
+                        C.weight_grad_prox_update(W, dpre, L["xmat"], eta, lam, Wn, self.ws, self.precision, G, s)
+                    else:
+                        C.prox_update_compact(W, G, eta, lam, Wn, self.ws, s)
                     L["cur"] = 1 - L["cur"]
                 else:
                     C.debias_update(W, L["g"], eta, s)

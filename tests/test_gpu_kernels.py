@@ -323,6 +323,61 @@ def test_prox_chain_of_steps_bit_exact(C, m, k):
         _check_csr_equal(bufs[(step + 1) % 2], ref)
 
 
+@pytest.mark.parametrize("m,k,n,density,lam,transposed", [
+    (300, 512, 64, 0.1, 0.05, True),
+    (129, 320, 36, 0.2, 0.02, False),
+    (200, 800, 128, 0.05, 0.03, True),
+    (1000, 4096, 256, 0.15, 0.01, True),
+    (64, 64, 4, 0.0, 0.0, True),
+])
+def test_fused_gradient_prox_matches_unfused(C, m, k, n, density, lam, transposed):
+    """weight_grad_prox_update (G never written) gives the same bits as
+    weight_grad_dense (TF32) followed by prox_update_compact."""
+    rng = np.random.default_rng(m + k + n)
+    a = _sparse(rng, m, k, density) * F32(0.05)
+    dy = _dev((rng.standard_normal((m, n)) * 0.1).astype(F32))
+    x = _dev(rng.standard_normal((k, n)).astype(F32))
+    ws = _ws(C, m, k, n)
+    w_in = _gpu_csr(C, a, ws, transposed=False)
+    g = torch.zeros(m, k, device="cuda")
+    C.weight_grad_dense(dy, x, g, ws, precision=C.CSRT_PREC_TF32)
+    ref = C.CSR(m, k, transposed=transposed)
+    C.prox_update_compact(w_in, g, 0.5, lam, ref, ws)
+    out = C.CSR(m, k, transposed=transposed)
+    C.weight_grad_prox_update(w_in, dy, x, 0.5, lam, out, ws)
+    assert ws.status()[0] == 0
+    (rp, ci, v), t = out.to_host()
+    (rp2, ci2, v2), t2 = ref.to_host()
+    np.testing.assert_array_equal(rp, rp2)
+    np.testing.assert_array_equal(ci, ci2)
+    np.testing.assert_array_equal(v.view(np.uint32), v2.view(np.uint32))
+    if transposed:
+        for p_, q_ in zip(t, t2):
+            np.testing.assert_array_equal(p_.view(np.uint32), q_.view(np.uint32))
+    # and against the oracle fed the same G
+    refo = O.prox_update_compact(O.csr_from_dense(a), g.cpu().numpy(), 0.5, lam)
+    np.testing.assert_array_equal(rp, refo.row_ptr)
+    np.testing.assert_array_equal(ci, refo.col_idx)
+
+
+def test_fused_gradient_prox_fallback_needs_scratch(C):
+    rng = np.random.default_rng(1)
+    m, k, n = 50, 40, 6                                   # too small for the tensor-core path
+    a = _sparse(rng, m, k, 0.3)
+    dy, x = _dev(rng.standard_normal((m, n)).astype(F32)), _dev(rng.standard_normal((k, n)).astype(F32))
+    ws = _ws(C, m, k, n)
+    w_in = _gpu_csr(C, a, ws)
+    out = C.CSR(m, k)
+    with pytest.raises(C.CsrtError):
+        C.weight_grad_prox_update(w_in, dy, x, 0.1, 0.01, out, ws)
+    g = torch.zeros(m, k, device="cuda")
+    C.weight_grad_prox_update(w_in, dy, x, 0.1, 0.01, out, ws, g_scratch=g)
+    ref = O.prox_update_compact(O.csr_from_dense(a), g.cpu().numpy(), 0.1, 0.01)
+    (rp, ci, v), _ = out.to_host()
+    np.testing.assert_array_equal(ci, ref.col_idx)
+    np.testing.assert_array_equal(v.view(np.uint32), ref.val.view(np.uint32))
+
+
 def test_prox_nan_is_dropped_and_flagged(C):
     a = np.array([[1.0, 0.0, 2.0, 0.0]], dtype=F32)
     g = np.array([[np.nan, 1.0, 0.0, np.nan]], dtype=F32)
