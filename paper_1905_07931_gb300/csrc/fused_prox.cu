@@ -30,9 +30,12 @@ int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t
                             size_t scratch_bytes, cudaStream_t s);
 size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
 
-constexpr int kFpTileCols = kTcBN;             // 256
-constexpr int kFpTileWords = kFpTileCols / 32;  // 8
+// The placement works on 128-column segments: each GEMM tile (256 columns) is
+// two segments, handled by two epilogue warps per TMEM lane quarter.
+constexpr int kFpTileCols = 128;                 // columns per segment
+constexpr int kFpTileWords = kFpTileCols / 32;   // 4
 constexpr int kFpMaxK = 16384;
+constexpr int kFpThreads = 64 + 8 * 32;          // producer, MMA, 8 epilogue warps
 
 struct FpLayout {
     int32_t nt, wpr;
@@ -82,29 +85,23 @@ __global__ void __launch_bounds__(256) fp_oldbits_kernel(const int32_t *__restri
     }
     __syncwarp();
     for (int i = lane; i < wpr; i += 32) obits[r * wpr + i] = w[i];
-    // stored entries per tile, then a warp exclusive scan over the (<= 64) tiles
-    uint32_t c0 = 0, c1 = 0;
-    const int t0 = lane, t1 = lane + 32;
-    if (t0 < nt)
-        for (int q = 0; q < kFpTileWords && t0 * kFpTileWords + q < wpr; ++q) c0 += __popc(w[t0 * kFpTileWords + q]);
-    if (t1 < nt)
-        for (int q = 0; q < kFpTileWords && t1 * kFpTileWords + q < wpr; ++q) c1 += __popc(w[t1 * kFpTileWords + q]);
-    uint32_t i0 = c0;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-        const uint32_t t = __shfl_up_sync(0xffffffffu, i0, off);
-        if (lane >= off) i0 += t;
-    }
-    const uint32_t tot0 = __shfl_sync(0xffffffffu, i0, 31);
-    uint32_t i1 = c1;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-        const uint32_t t = __shfl_up_sync(0xffffffffu, i1, off);
-        if (lane >= off) i1 += t;
-    }
+    // stored entries per segment, then a warp exclusive scan over the segments (32 at a time)
     int32_t *os = ostart + r * (nt + 1);
-    if (t0 < nt) os[t0] = s + (int32_t)(i0 - c0);
-    if (t1 < nt) os[t1] = s + (int32_t)(tot0 + i1 - c1);
+    int32_t run = s;
+    for (int t0 = 0; t0 < nt; t0 += 32) {
+        const int t = t0 + lane;
+        uint32_t c = 0;
+        if (t < nt)
+            for (int q = 0; q < kFpTileWords && t * kFpTileWords + q < wpr; ++q) c += __popc(w[t * kFpTileWords + q]);
+        uint32_t incl = c;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const uint32_t u = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += u;
+        }
+        if (t < nt) os[t] = run + (int32_t)(incl - c);
+        run += (int32_t)__shfl_sync(0xffffffffu, incl, 31);
+    }
     if (lane == 0) os[nt] = e;
 }
 
@@ -121,7 +118,7 @@ struct FpArgs {
 };
 
 // 2. Persistent TF32 GEMM whose epilogue applies the prox step.
-__global__ void __launch_bounds__(kTcThreads, 1)
+__global__ void __launch_bounds__(kFpThreads, 1)
     gemm_prox_tc_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                         FpArgs a, int32_t tiles_n, int32_t num_tiles) {
     extern __shared__ uint8_t smem_raw[];
@@ -149,8 +146,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         mbar_init(accf, 1);
         mbar_init(accf + 1, 1);
-        mbar_init(acce, 4);
-        mbar_init(acce + 1, 4);
+        mbar_init(acce, 8);
+        mbar_init(acce + 1, 8);
         mbar_init(fin, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_a)) : "memory");
@@ -208,44 +205,57 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             mbar_wait(fin, 0);
         }
     } else {
-        const int q = warp & 3;   // TMEM lanes 32q .. 32q+31 = tile rows 32q ..
+        // epilogue: warp w (2..9) reads TMEM lanes 32*(w%4).. (tile rows) and
+        // segment h = (w-2)/4 of the tile (columns 128h .. 128h+127)
+        const int q = warp & 3;
+        const int h = (warp - 2) >> 2;
         bool nonfinite = false;
+        float zsum = 0.f;
         int j = 0;
         for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++j) {
             const int acc = j & 1;
-            const bool ok = __all_sync(0xffffffffu, mbar_wait_or_abort(accf + acc, (j >> 1) & 1, &s_abort));
-            if (!ok) break;
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const int mt = t / tiles_n, nt = t % tiles_n;
+            const int seg = nt * 2 + h;                     // segment index within the row
             const int64_t row = (int64_t)mt * kTcBM + q * 32 + lane;
-            const bool rv = row < a.m;
+            const bool rv = row < a.m && seg < a.nt;
+            // stored-weight bitmask and first stored entry of this segment: known before the MMA ends
             uint32_t ob[kFpTileWords];
             int32_t oidx = 0;
-            const int wbase = nt * kFpTileWords;
+            const int wbase = seg * kFpTileWords;
 #pragma unroll
             for (int c = 0; c < kFpTileWords; ++c)
                 ob[c] = (rv && wbase + c < a.wpr) ? __ldg(a.obits + row * a.wpr + wbase + c) : 0u;
-            if (rv) oidx = __ldg(a.ostart + row * (a.nt + 1) + nt);
-            float *stage = a.stage + (row * a.nt + nt) * kFpTileCols;
+            if (rv) oidx = __ldg(a.ostart + row * (a.nt + 1) + seg);
+            // old weights of word 0 in flight before waiting for the accumulator
+            float wnext[32];
+#pragma unroll
+            for (int jj = 0; jj < 32; ++jj)
+                wnext[jj] = ((ob[0] >> jj) & 1u) ? __ldg(a.old_val + oidx + __popc(ob[0] & ((1u << jj) - 1u))) : 0.f;
+            const bool ok = __all_sync(0xffffffffu, mbar_wait_or_abort(accf + acc, (j >> 1) & 1, &s_abort));
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            float *stage = a.stage + (row * a.nt + seg) * kFpTileCols;
             uint32_t cnt = 0;
-#pragma unroll 1
+#pragma unroll
             for (int c = 0; c < kFpTileWords; ++c) {
                 uint32_t r[32];
-                tmem_ld_32cols(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kTcBN + c * 32), r);
-                const uint32_t ow = ob[c];
-                // stored weights of this word (loads only where the old pattern has an entry)
+                tmem_ld_32cols(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kTcBN + h * kFpTileCols + c * 32),
+                               r);
                 float w[32];
 #pragma unroll
-                for (int jj = 0; jj < 32; ++jj) {
-                    w[jj] = 0.f;
-                    if ((ow >> jj) & 1u) w[jj] = __ldg(a.old_val + oidx + __popc(ow & ((1u << jj) - 1u)));
+                for (int jj = 0; jj < 32; ++jj) w[jj] = wnext[jj];
+                oidx += __popc(ob[c]);
+                if (c + 1 < kFpTileWords) {   // next word's old weights in flight while this one is computed
+                    const uint32_t on = ob[c + 1];
+#pragma unroll
+                    for (int jj = 0; jj < 32; ++jj)
+                        wnext[jj] = ((on >> jj) & 1u) ? __ldg(a.old_val + oidx + __popc(on & ((1u << jj) - 1u))) : 0.f;
                 }
-                oidx += __popc(ow);
                 uint32_t kw = 0;
 #pragma unroll
                 for (int jj = 0; jj < 32; ++jj) {
                     const float z = __fsub_rn(w[jj], __fmul_rn(a.eta, __uint_as_float(r[jj])));
-                    nonfinite |= z != z;
+                    zsum += z;   // a NaN anywhere in z stays NaN in the sum
                     if (fabsf(z) > a.thr) {
                         kw |= 1u << jj;
                         if (rv) stage[cnt] = __fsub_rn(z, copysignf(a.thr, z));
@@ -254,11 +264,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
                 if (rv && wbase + c < a.wpr) a.kbits[row * a.wpr + wbase + c] = kw;
             }
-            if (rv) a.counts[row * a.nt + nt] = (int32_t)cnt;
+            if (rv) a.counts[row * a.nt + seg] = (int32_t)cnt;
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
             if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(acce + acc)) : "memory");
         }
+        nonfinite = zsum != zsum;
         if (__any_sync(0xffffffffu, nonfinite) && lane == 0) s_nonfinite = 1;
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -277,29 +288,27 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
 }
 
-// 3. Per row: exclusive offsets of the tiles (in place) and the row total.
+// 3. Per row: exclusive offsets of the segments (in place) and the row total.
 __global__ void __launch_bounds__(256) fp_rowscan_kernel(int32_t *__restrict__ counts, int32_t m, int32_t nt,
                                                          int32_t *__restrict__ rowtot) {
     const int lane = threadIdx.x & 31;
     const int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     if (r >= m) return;
     int32_t *c = counts + r * nt;
-    const int32_t c0 = lane < nt ? c[lane] : 0, c1 = lane + 32 < nt ? c[lane + 32] : 0;
-    int32_t i0 = c0, i1 = c1;
+    int32_t run = 0;
+    for (int t0 = 0; t0 < nt; t0 += 32) {
+        const int t = t0 + lane;
+        const int32_t v = t < nt ? c[t] : 0;
+        int32_t incl = v;
 #pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-        const int32_t t0 = __shfl_up_sync(0xffffffffu, i0, off);
-        const int32_t t1 = __shfl_up_sync(0xffffffffu, i1, off);
-        if (lane >= off) {
-            i0 += t0;
-            i1 += t1;
+        for (int off = 1; off < 32; off <<= 1) {
+            const int32_t u = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += u;
         }
+        if (t < nt) c[t] = run + incl - v;
+        run += __shfl_sync(0xffffffffu, incl, 31);
     }
-    const int32_t tot0 = __shfl_sync(0xffffffffu, i0, 31);
-    const int32_t tot1 = __shfl_sync(0xffffffffu, i1, 31);
-    if (lane < nt) c[lane] = i0 - c0;
-    if (lane + 32 < nt) c[lane + 32] = tot0 + i1 - c1;
-    if (lane == 0) rowtot[r] = tot0 + tot1;
+    if (lane == 0) rowtot[r] = run;
 }
 
 // 4. One warp per (row, tile): final positions, one coalesced run per word.
@@ -421,9 +430,9 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     a.counts = counts;
     a.stage = stage;
     a.hdr = static_cast<WsHeader *>(ws);
-    const int tiles_m = (int)ceil_div<int64_t>(m, kTcBM), tiles_n = L.nt;
+    const int tiles_m = (int)ceil_div<int64_t>(m, kTcBM), tiles_n = (int)ceil_div<int64_t>(k, kTcBN);
     const int tiles = tiles_m * tiles_n;
-    gemm_prox_tc_kernel<<<imin(tiles, num_sms()), kTcThreads, kTcSmemBytes, s>>>(ma, mb, a, tiles_n, tiles);
+    gemm_prox_tc_kernel<<<imin(tiles, num_sms()), kFpThreads, kTcSmemBytes, s>>>(ma, mb, a, tiles_n, tiles);
     fp_rowscan_kernel<<<(unsigned)ceil_div<int64_t>((int64_t)m * 32, 256), 256, 0, s>>>(counts, m, L.nt, rowtot);
     count_launch(3);
     // new row pointers: exclusive scan of the row totals (int32: nnz <= M*K < 2^31)

@@ -329,6 +329,8 @@ def test_prox_chain_of_steps_bit_exact(C, m, k):
     (200, 800, 128, 0.05, 0.03, True),
     (1000, 4096, 256, 0.15, 0.01, True),
     (64, 64, 4, 0.0, 0.0, True),
+    (260, 9216, 64, 0.05, 0.02, True),
+    (70, 16384, 32, 0.05, 0.02, False),
 ])
 def test_fused_gradient_prox_matches_unfused(C, m, k, n, density, lam, transposed):
     """weight_grad_prox_update (G never written) gives the same bits as
