@@ -56,6 +56,8 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--precision", choices=["tf32", "fp32"], default="tf32")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--prox-path", choices=["fused", "unfused"], default="unfused",
+                   help="fused: weight gradient and prox update in one tensor-core pass (G not written)")
     p.add_argument("--profile-ops", action="store_true", help="print the per-operation breakdown to stderr")
     return p.parse_args()
 
@@ -330,7 +332,8 @@ def main():
     prec = C.CSRT_PREC_TF32 if args.precision == "tf32" else C.CSRT_PREC_FP32
     cfg = synth.fc_head(seed=0)
     layers = mlp_layers(3)
-    net = SparseNet(layers, cfg["W"], cfg["b"], BATCH, (SIZES[0],), precision=prec)
+    net = SparseNet(layers, cfg["W"], cfg["b"], BATCH, (SIZES[0],), precision=prec,
+                    fused=args.prox_path == "fused")
     x_host = torch.from_numpy(cfg["X"]).pin_memory()
     lab_host = torch.from_numpy(cfg["labels"]).pin_memory()
     net.x_in.copy_(x_host)
@@ -447,6 +450,7 @@ def main():
         "config": {"workload": WORKLOAD, "global_batch": BATCH * world, "per_gpu_batch": BATCH,
                    "layers": list(SIZES), "densities": list(DENSITIES),
                    "weight_grad": "tf32 tcgen05" if prec == C.CSRT_PREC_TF32 else "fp32 simt",
+                   "prox_path": args.prox_path,
                    "l2": "flushed between steps (256 MB write, outside the timed region)",
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "step_ops": [r["label"] for r in prof]},
