@@ -56,7 +56,7 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--precision", choices=["tf32", "fp32"], default="tf32")
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--prox-path", choices=["fused", "unfused"], default="unfused",
+    p.add_argument("--prox-path", choices=["fused", "unfused"], default="fused",
                    help="fused: weight gradient and prox update in one tensor-core pass (G not written)")
     p.add_argument("--profile-ops", action="store_true", help="print the per-operation breakdown to stderr")
     return p.parse_args()

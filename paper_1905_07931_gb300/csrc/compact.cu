@@ -998,11 +998,14 @@ __global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict
 //  count: lane r loads row r's word; a 32 x 32 bit transpose (five shuffle
 //         stages) gives lane j the rows present in column 32c + j; its popcount
 //         is the block's count for that column.
-//  write: the block walks its 32 rows in order; lane j handles column 32c + j.
-//         In row r the CSR positions of the kept columns are consecutive
-//         (word position + rank in the word), so the values are gathered and
-//         t_pos is written coalesced; each column's transposed run advances by
-//         one per kept row.
+//  write: first the row pass, lane j = column 32c + j: the warp walks its 32
+//         rows in order. In row r the CSR positions of the kept columns are
+//         consecutive (word position + rank in the word), so the values are
+//         read and t_pos is written coalesced; each column's transposed run
+//         advances by one per kept row; the values go to a 32 x 32 shared
+//         tile. Then the column pass, lane r = row: for each column the rows
+//         kept in it are consecutive positions of its transposed run, so
+//         t_col and t_val are written coalesced as well.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
     const int lane = threadIdx.x & 31;
@@ -1037,29 +1040,44 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
                                                         const float *__restrict__ val, int32_t *__restrict__ t_col,
                                                         float *__restrict__ t_val, int32_t *__restrict__ t_pos,
                                                         int64_t capacity) {
-    const int lane = threadIdx.x & 31;
+    __shared__ float tile[8][32 * 32];   // element (r, j) at r*32 + (j ^ r): rows and columns conflict-free
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nb = ceil_div<int64_t>(rows, 32);
-    if (gw >= nb * wpr) return;
+    if (gw >= nb * wpr) return;   // whole warps
     const int b = (int)(gw / wpr), c = (int)(gw % wpr);
     const int my_row = b * 32 + lane;
     const uint32_t rw_mine = my_row < rows ? __ldg(keepbits + (int64_t)my_row * wpr + c) : 0u;
     const int32_t rp_mine = my_row < rows ? __ldg(wordpos + (int64_t)my_row * wpr + c) : 0;
     const int col = c * 32 + lane;
-    int64_t pc = (int64_t)__ldg(t_row_ptr + col) + __ldg(off + (int64_t)b * cols + col);
+    const int64_t pc0 = (int64_t)__ldg(t_row_ptr + col) + __ldg(off + (int64_t)b * cols + col);
     const unsigned lt = (1u << lane) - 1u;
+    float *tl = tile[warp];
     const int nr = imin(32, rows - b * 32);
-    for (int r = 0; r < nr; ++r) {
+    int64_t pc = pc0;
+    for (int r = 0; r < nr; ++r) {   // row pass
         const uint32_t rw = __shfl_sync(0xffffffffu, rw_mine, r);
+        if (rw == 0u) continue;
         const int32_t rp = __shfl_sync(0xffffffffu, rp_mine, r);
         if ((rw >> lane) & 1u) {
             const int64_t pr = (int64_t)rp + __popc(rw & lt);
-            if (pc < capacity && pr < capacity) {
-                t_col[pc] = b * 32 + r;
-                t_val[pc] = __ldg(val + pr);
-                t_pos[pr] = (int32_t)pc;
-            }
+            tl[r * 32 + (lane ^ r)] = pr < capacity ? __ldg(val + pr) : 0.f;
+            if (pc < capacity && pr < capacity) t_pos[pr] = (int32_t)pc;
             ++pc;
+        }
+    }
+    __syncwarp();
+    const uint32_t colmask = warp_transpose32(rw_mine);   // lane j: the block's rows kept in column 32c + j
+    for (int jj = 0; jj < 32; ++jj) {   // column pass
+        const uint32_t cm = __shfl_sync(0xffffffffu, colmask, jj);
+        if (cm == 0u) continue;
+        const int64_t base = __shfl_sync(0xffffffffu, pc0, jj);
+        if ((cm >> lane) & 1u) {
+            const int64_t p = base + __popc(cm & lt);
+            if (p < capacity) {
+                t_col[p] = b * 32 + lane;
+                t_val[p] = tl[lane * 32 + (jj ^ lane)];
+            }
         }
     }
 }

@@ -4,22 +4,27 @@
 // The prox step (Eq. prox with the soft threshold of Section 2.2, applied to
 // the dense w - eta*G as in Section 3.3, compacted after every update as in
 // Section 4.4) needs G = dY X^T at every entry, but only once: here the
-// tensor-core GEMM's epilogue applies it straight from the accumulator.
+// tensor-core GEMM's epilogue applies it straight from the accumulator. The
+// output position of an entry depends on the kept counts of every earlier row,
+// so the GEMM runs twice; the accumulator of a tile is the same in both passes
+// (same tiles, same MMA order), hence so are the keep decisions.
 //
 //  1. fp_oldbits_kernel: per row of W_in, a bitmask of the stored columns and,
-//     per 256-column tile, the index of the row's first stored entry in it.
-//  2. gemm_prox_tc_kernel: the persistent tcgen05 GEMM of gemm_tc.cu (same
-//     tiles, same MMA order, so the same G bits as weight_grad_dense TF32).
-//     Its epilogue thread owns one row of a 128 x 256 tile; for each entry it
-//     takes w from W_in (through the bitmask: loads only where a weight is
-//     stored), forms z = fl(w - fl(eta*G)), keeps |z| > fl(eta*lambda) and
-//     stages the kept values of (row, tile) contiguously plus the tile's keep
-//     bitmask and its count.
+//     per 128-column segment, the index of the row's first stored entry in it.
+//  2. gemm_prox_tc_kernel<count>: the persistent tcgen05 GEMM of gemm_tc.cu
+//     (same tiles, same MMA order, so the same G bits as weight_grad_dense
+//     TF32). Each epilogue thread owns one row of a 128-column segment of a
+//     128 x 256 tile; per entry it takes w from W_in (through the bitmask:
+//     loads only where a weight is stored), forms z = fl(w - fl(eta*G)), keeps
+//     |z| > fl(eta*lambda), and writes the keep bitmask and the kept count of
+//     the segment.
 //  3. fp_rowscan_kernel + scan_single_block_kernel: per-row offsets of the
-//     tiles and the new row pointers.
-//  4. fp_place_kernel: one warp per (row, tile) writes the tile's kept entries
-//     at their final positions, one coalesced run per 32-column word, and the
-//     word positions used to build the transposed copy from the bitmask.
+//     segments and the new row pointers.
+//  4. gemm_prox_tc_kernel<write>: the same GEMM again; the epilogue recomputes
+//     z, passes each 32 x 32 block through shared memory and writes the kept
+//     entries of one row at a time at their final positions (a coalesced run
+//     per row and 32 columns), plus the word positions from which the
+//     transposed copy is built out of the bitmask.
 // The result is bit-identical to weight_grad_dense (TF32) followed by
 // prox_update_compact.
 #include "tc_common.cuh"
@@ -30,16 +35,41 @@ int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t
                             size_t scratch_bytes, cudaStream_t s);
 size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
 
-// The placement works on 128-column segments: each GEMM tile (256 columns) is
-// two segments, handled by two epilogue warps per TMEM lane quarter.
-constexpr int kFpTileCols = 128;                 // columns per segment
-constexpr int kFpTileWords = kFpTileCols / 32;   // 4
+// Segments (the unit of the per-row offsets) are 64 columns, two 32-column
+// words; a GEMM tile (256 columns) is four of them.
+constexpr int kFpTileCols = 64;                  // columns per segment
+constexpr int kFpTileWords = kFpTileCols / 32;   // 2
 constexpr int kFpMaxK = 16384;
-constexpr int kFpThreads = 64 + 8 * 32;          // producer, MMA, 8 epilogue warps
+constexpr int kFpPre = 8;                        // stored old weights per word prefetched into registers
+
+// Launch shape of each pass: epilogue warps and pipeline stages. The count
+// pass is bound by the MMA (4 stages); the write pass by its epilogue, which
+// also needs a per-row table (3 stages leave room for it).
+#ifndef CSRT_FP_COUNT_EPI
+#define CSRT_FP_COUNT_EPI 8
+#endif
+#ifndef CSRT_FP_WRITE_EPI
+#define CSRT_FP_WRITE_EPI 8
+#endif
+template <bool kWrite> struct FpShape;
+template <> struct FpShape<false> {
+    static constexpr int kEpi = CSRT_FP_COUNT_EPI, kStages = CSRT_FP_COUNT_EPI > 8 ? 3 : 4;
+};
+template <> struct FpShape<true> { static constexpr int kEpi = CSRT_FP_WRITE_EPI, kStages = 3; };
+template <bool kWrite> constexpr int fp_threads() { return 64 + FpShape<kWrite>::kEpi * 32; }
+// Per epilogue warp: a 32 x 32 float buffer, row r's 16-byte chunk c at float
+// offset r*32 + ((c ^ (r & 7)) << 2), so that a row written as eight 16-byte
+// stores and a column read one element per lane are both free of bank
+// conflicts; then (write pass) a table of the 32 rows' keep word and position.
+template <bool kWrite> __host__ __device__ constexpr int fp_xfloats() { return 32 * 32 + (kWrite ? 2 * 32 : 0); }
+template <bool kWrite> constexpr int fp_smem_bytes() {
+    return FpShape<kWrite>::kStages * kTcStageBytes + 1024 + 256 + FpShape<kWrite>::kEpi * fp_xfloats<kWrite>() * 4;
+}
+static_assert(fp_smem_bytes<false>() <= 232448 && fp_smem_bytes<true>() <= 232448, "shared memory per block");
 
 struct FpLayout {
     int32_t nt, wpr;
-    size_t off_obits, off_ostart, off_kbits, off_counts, off_rowtot, off_stage, off_wordpos, off_tr, total;
+    size_t off_obits, off_ostart, off_kbits, off_counts, off_rowtot, off_wordpos, off_tr, total;
 };
 
 static size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -54,7 +84,6 @@ static FpLayout fp_layout(int32_t m, int32_t k) {
     L.off_kbits = o;   o += align256((size_t)m * L.wpr * 4);
     L.off_counts = o;  o += align256((size_t)m * L.nt * 4);
     L.off_rowtot = o;  o += align256((size_t)m * 4);
-    L.off_stage = o;   o += align256((size_t)m * L.nt * kFpTileCols * 4);
     L.off_wordpos = o; o += align256((size_t)m * L.wpr * 4);
     L.off_tr = o;      o += align256(transpose_scratch_bytes(m, k));
     L.total = o;
@@ -111,26 +140,113 @@ struct FpArgs {
     const uint32_t *obits;
     const int32_t *ostart;
     const float *old_val;
-    uint32_t *kbits;
-    int32_t *counts;
-    float *stage;
+    uint32_t *kbits;     // count pass: keep bitmask per 32-column word
+    int32_t *counts;     // count pass: kept entries per (row, segment); write pass: their offsets in the row
+    const int32_t *row_ptr_out;   // write pass: new row pointers (not yet clamped to the capacity)
+    int32_t *out_col;
+    float *out_val;
+    int32_t *wordpos;    // write pass: position of each word's first kept entry (or null)
+    int64_t capacity;
     WsHeader *hdr;
 };
 
-// 2. Persistent TF32 GEMM whose epilogue applies the prox step.
-__global__ void __launch_bounds__(kFpThreads, 1)
+
+// Per-tile inputs of an epilogue thread (its row of the tile's column span):
+// the stored-weight bitmask of each word, the index of the span's first stored
+// weight and, in the write pass, the position of its first kept entry.
+template <int W>
+struct FpMeta {
+    uint32_t ob[W];
+    uint32_t kb[W];   // write pass: the keep bitmask the count pass wrote
+    int32_t o0, pos;
+};
+
+template <bool kWrite, int W>
+__device__ __forceinline__ void fp_load_meta(const FpArgs &a, int t, int num_tiles, int tiles_n, int h, int64_t rowq,
+                                             FpMeta<W> &m) {
+    const int mt = t / tiles_n, nt = t % tiles_n;
+    const int64_t row = (int64_t)mt * kTcBM + rowq;
+    const bool rv = t < num_tiles && row < a.m;
+    const int word0 = nt * (kTcBN / 32) + h * W;
+    const int seg0 = word0 / kFpTileWords;
+    const bool sv = rv && seg0 < a.nt;
+#pragma unroll
+    for (int c = 0; c < W; ++c) m.ob[c] = (rv && word0 + c < a.wpr) ? __ldg(a.obits + row * a.wpr + word0 + c) : 0u;
+#pragma unroll
+    for (int c = 0; c < W; ++c)
+        m.kb[c] = (kWrite && rv && word0 + c < a.wpr) ? __ldg(a.kbits + row * a.wpr + word0 + c) : 0u;
+    m.o0 = sv ? __ldg(a.ostart + row * (a.nt + 1) + seg0) : 0;
+    m.pos = (kWrite && sv) ? __ldg(a.row_ptr_out + row) + __ldg(a.counts + row * a.nt + seg0) : 0;
+}
+
+// The first kFpPre stored weights of a word (its bitmask ob, first index o).
+__device__ __forceinline__ void fp_load_words(const float *__restrict__ old_val, uint32_t ob, int32_t o,
+                                              float (&wv)[kFpPre]) {
+    const int nc = __popc(ob);
+#pragma unroll
+    for (int u = 0; u < kFpPre; ++u) wv[u] = u < nc ? __ldg(old_val + o + u) : 0.f;
+}
+
+// Write pass, column domain: lane = column of the word, the 32 rows in groups
+// of 8 (independent, so their loads overlap). Row i's kept entries go to
+// consecutive positions from the row's position in the table.
+template <bool kCheck>
+__device__ __forceinline__ void fp_write_word(const float *xb, const int2 *tab, const int (&lx)[8], uint32_t lt,
+                                              int32_t col, float thr, int32_t cap32, int32_t *__restrict__ out_col,
+                                              float *__restrict__ out_val) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int i0 = 0; i0 < 32; i0 += 8) {
+        float z[8];
+        int2 tb[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            tb[u] = tab[i0 + u];
+            z[u] = xb[(i0 + u) * 32 + lx[u]];
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const uint32_t kwi = (uint32_t)tb[u].x;
+            const int32_t p = tb[u].y + __popc(kwi & lt);
+            if (((kwi >> lane) & 1u) && (!kCheck || p < cap32)) {
+                out_col[p] = col;
+                out_val[p] = __fsub_rn(z[u], copysignf(thr, z[u]));
+            }
+        }
+    }
+}
+
+// 2./4. Persistent TF32 GEMM whose epilogue applies the prox step: counts and
+// keep bits (kWrite = false) or the compacted entries (kWrite = true).
+//
+// Epilogue warp e reads TMEM lane quarter (e+2) % 4 (tile rows) and column span
+// e / 4 of the tile (128 columns in the count pass, 64 in the write pass).
+// Per 32-column word, in the row domain (thread = row): z = fl(-eta*G) for
+// every entry (exact for an unstored weight: fl(0 - fl(eta*G)) = fl(-eta*G)),
+// staged in the warp's buffer; entries with a stored weight are then fixed up
+// to fl(w + z) = fl(w - fl(eta*G)). The count pass reads back only its own
+// row. The write pass then switches to the column domain (lane = column): for
+// each row of the 32 the kept entries form one run of consecutive positions,
+// written with coalesced stores.
+template <bool kWrite>
+__global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
     gemm_prox_tc_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                         FpArgs a, int32_t tiles_n, int32_t num_tiles) {
+    constexpr int kEpi = FpShape<kWrite>::kEpi, kStages = FpShape<kWrite>::kStages;
+    constexpr int kSpanCols = kTcBN / (kEpi / 4);   // columns per epilogue warp
+    constexpr int kSpanWords = kSpanCols / 32;
+    static_assert(kSpanWords % kFpTileWords == 0, "a span holds whole segments");
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sa = smem;
-    uint8_t *sb = smem + kTcStages * kTcABytes;
-    uint64_t *full = reinterpret_cast<uint64_t *>(smem + kTcStages * kTcStageBytes);
-    uint64_t *empty = full + kTcStages;
-    uint64_t *accf = empty + kTcStages;
+    uint8_t *sb = smem + kStages * kTcABytes;
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + kStages * kTcStageBytes);
+    uint64_t *empty = full + kStages;
+    uint64_t *accf = empty + kStages;
     uint64_t *acce = accf + 2;
     uint64_t *fin = acce + 2;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(fin + 1);
+    float *xbuf = reinterpret_cast<float *>(smem + kStages * kTcStageBytes + 256);
     __shared__ volatile int s_abort;
     __shared__ int s_nonfinite;
 
@@ -140,14 +256,14 @@ __global__ void __launch_bounds__(kFpThreads, 1)
     if (threadIdx.x == 0) {
         s_abort = 0;
         s_nonfinite = 0;
-        for (int s = 0; s < kTcStages; ++s) {
+        for (int s = 0; s < kStages; ++s) {
             mbar_init(full + s, 1);
             mbar_init(empty + s, 1);
         }
         mbar_init(accf, 1);
         mbar_init(accf + 1, 1);
-        mbar_init(acce, 8);
-        mbar_init(acce + 1, 8);
+        mbar_init(acce, kEpi);
+        mbar_init(acce + 1, kEpi);
         mbar_init(fin, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_a)) : "memory");
@@ -170,14 +286,14 @@ __global__ void __launch_bounds__(kFpThreads, 1)
             for (int t = blockIdx.x; t < num_tiles && !s_abort; t += gridDim.x) {
                 const int m0 = (t / tiles_n) * kTcBM, n0 = (t % tiles_n) * kTcBN;
                 for (int kb = 0; kb < num_kb; ++kb, ++it) {
-                    const int s = it % kTcStages;
-                    if (!mbar_wait_or_abort(empty + s, ((it / kTcStages) & 1) ^ 1, &s_abort)) break;
+                    const int s = it % kStages;
+                    if (!mbar_wait_or_abort(empty + s, ((it / kStages) & 1) ^ 1, &s_abort)) break;
                     mbar_expect_tx(full + s, kTcStageBytes);
                     tma_load_2d(sa + s * kTcABytes, &map_a, kb * kTcBK, m0, full + s);
                     tma_load_2d(sb + s * kTcBBytes, &map_b, kb * kTcBK, n0, full + s);
                 }
             }
-            for (int i = imax(0, it - kTcStages); i < it; ++i) mbar_wait(full + i % kTcStages, (i / kTcStages) & 1);
+            for (int i = imax(0, it - kStages); i < it; ++i) mbar_wait(full + i % kStages, (i / kStages) & 1);
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -188,8 +304,8 @@ __global__ void __launch_bounds__(kFpThreads, 1)
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t d = tmem + (uint32_t)(acc * kTcBN);
                 for (int kb = 0; kb < num_kb; ++kb, ++it) {
-                    const int s = it % kTcStages;
-                    if (!mbar_wait_or_abort(full + s, (it / kTcStages) & 1, &s_abort)) break;
+                    const int s = it % kStages;
+                    if (!mbar_wait_or_abort(full + s, (it / kStages) & 1, &s_abort)) break;
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll
                     for (int k = 0; k < kTcBK / 8; ++k) {
@@ -205,79 +321,157 @@ __global__ void __launch_bounds__(kFpThreads, 1)
             mbar_wait(fin, 0);
         }
     } else {
-        // epilogue: warp w (2..9) reads TMEM lanes 32*(w%4).. (tile rows) and
-        // segment h = (w-2)/4 of the tile (columns 128h .. 128h+127)
-        const int q = warp & 3;
-        const int h = (warp - 2) >> 2;
-        bool nonfinite = false;
-        float zsum = 0.f;
+        const int e = warp - 2;
+        const int q = warp & 3;   // the TMEM lane quarter this warp may read
+        const int h = e >> 2;     // column span within the tile
+        const int64_t rowq = q * 32 + lane;
+        float *xb = xbuf + e * fp_xfloats<kWrite>();
+        int2 *tab = reinterpret_cast<int2 *>(xb + 32 * 32);
+        float *xr = xb + lane * 32;   // this thread's row
+        const int sw = (lane & 7) << 2;
+        int lx[8];   // column-domain offsets: element (i, lane) at i*32 + lx[i & 7]
+#pragma unroll
+        for (int u = 0; u < 8; ++u) lx[u] = lane ^ (u << 2);
+        const uint32_t lt = (1u << lane) - 1u;
+        const int32_t cap32 = (int32_t)imin<int64_t>(a.capacity, 0x7fffffff);
+        // every position is below the capacity unless the output overflows
+        const bool fits = !kWrite || (int64_t)__ldg(a.row_ptr_out + a.m) <= a.capacity;
+        float tsum = 0.f;
+        // software pipeline: the next tile's metadata one tile ahead, the
+        // next word's stored weights one word ahead
+        FpMeta<kSpanWords> cur, nxt;
+        fp_load_meta<kWrite>(a, blockIdx.x, num_tiles, tiles_n, h, rowq, cur);
+        fp_load_meta<kWrite>(a, blockIdx.x + gridDim.x, num_tiles, tiles_n, h, rowq, nxt);
+        float wv_n[kFpPre];
+        int32_t ow_n = cur.o0;
+        fp_load_words(a.old_val, cur.ob[0], ow_n, wv_n);
         int j = 0;
         for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++j) {
             const int acc = j & 1;
             const int mt = t / tiles_n, nt = t % tiles_n;
-            const int seg = nt * 2 + h;                     // segment index within the row
-            const int64_t row = (int64_t)mt * kTcBM + q * 32 + lane;
-            const bool rv = row < a.m && seg < a.nt;
-            // stored-weight bitmask and first stored entry of this segment: known before the MMA ends
-            uint32_t ob[kFpTileWords];
-            int32_t oidx = 0;
-            const int wbase = seg * kFpTileWords;
-#pragma unroll
-            for (int c = 0; c < kFpTileWords; ++c)
-                ob[c] = (rv && wbase + c < a.wpr) ? __ldg(a.obits + row * a.wpr + wbase + c) : 0u;
-            if (rv) oidx = __ldg(a.ostart + row * (a.nt + 1) + seg);
-            // old weights of word 0 in flight before waiting for the accumulator
-            float wnext[32];
-#pragma unroll
-            for (int jj = 0; jj < 32; ++jj)
-                wnext[jj] = ((ob[0] >> jj) & 1u) ? __ldg(a.old_val + oidx + __popc(ob[0] & ((1u << jj) - 1u))) : 0.f;
+            const int64_t row = (int64_t)mt * kTcBM + rowq;
+            const bool rv = row < a.m;
+            const int word0 = nt * (kTcBN / 32) + h * kSpanWords;   // first word of the span
             const bool ok = __all_sync(0xffffffffu, mbar_wait_or_abort(accf + acc, (j >> 1) & 1, &s_abort));
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            float *stage = a.stage + (row * a.nt + seg) * kFpTileCols;
+            int32_t pos = cur.pos;   // write pass: position of the row's next kept entry
             uint32_t cnt = 0;
 #pragma unroll
-            for (int c = 0; c < kFpTileWords; ++c) {
-                uint32_t r[32];
-                tmem_ld_32cols(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kTcBN + h * kFpTileCols + c * 32),
-                               r);
-                float w[32];
+            for (int c = 0; c < kSpanWords; ++c) {
+                const int word = word0 + c;
+                const uint32_t obc = cur.ob[c];
+                float wv[kFpPre];
 #pragma unroll
-                for (int jj = 0; jj < 32; ++jj) w[jj] = wnext[jj];
-                oidx += __popc(ob[c]);
-                if (c + 1 < kFpTileWords) {   // next word's old weights in flight while this one is computed
-                    const uint32_t on = ob[c + 1];
-#pragma unroll
-                    for (int jj = 0; jj < 32; ++jj)
-                        wnext[jj] = ((on >> jj) & 1u) ? __ldg(a.old_val + oidx + __popc(on & ((1u << jj) - 1u))) : 0.f;
+                for (int u = 0; u < kFpPre; ++u) wv[u] = wv_n[u];
+                const int32_t ow = ow_n;
+                if (c + 1 < kSpanWords) {
+                    ow_n = ow + __popc(obc);
+                    fp_load_words(a.old_val, cur.ob[c + 1 < kSpanWords ? c + 1 : c], ow_n, wv_n);
+                } else {
+                    ow_n = nxt.o0;
+                    fp_load_words(a.old_val, nxt.ob[0], ow_n, wv_n);
                 }
-                uint32_t kw = 0;
+                uint32_t g[32];
+                tmem_ld_32cols(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kTcBN + h * kSpanCols + c * 32),
+                               g);
+                if (c == kSpanWords - 1) {   // accumulator fully read: hand it back to the MMA warp
+                    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                    __syncwarp();
+                    if (lane == 0)
+                        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(acce + acc)) : "memory");
+                }
+                float zz[32];
 #pragma unroll
-                for (int jj = 0; jj < 32; ++jj) {
-                    const float z = __fsub_rn(w[jj], __fmul_rn(a.eta, __uint_as_float(r[jj])));
-                    zsum += z;   // a NaN anywhere in z stays NaN in the sum
-                    if (fabsf(z) > a.thr) {
-                        kw |= 1u << jj;
-                        if (rv) stage[cnt] = __fsub_rn(z, copysignf(a.thr, z));
-                        ++cnt;
+                for (int jj = 0; jj < 32; ++jj) zz[jj] = __fmul_rn(-a.eta, __uint_as_float(g[jj]));
+                uint32_t kw = 0;
+                if (!kWrite) {
+                    // keep bits of the unstored entries and the NaN probe, as trees
+                    uint32_t k4[4] = {0u, 0u, 0u, 0u};
+                    float s8[8];
+#pragma unroll
+                    for (int jj = 0; jj < 32; ++jj) k4[jj >> 3] |= (fabsf(zz[jj]) > a.thr ? 1u : 0u) << jj;
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) s8[u] = (zz[u] + zz[u + 8]) + (zz[u + 16] + zz[u + 24]);
+                    tsum += ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
+                    kw = (k4[0] | k4[1]) | (k4[2] | k4[3]);
+                }
+                if (kWrite) __syncwarp();   // the previous word's column reads are done
+#pragma unroll
+                for (int cc = 0; cc < 8; ++cc)
+                    *reinterpret_cast<float4 *>(xr + ((cc << 2) ^ sw)) =
+                        make_float4(zz[4 * cc], zz[4 * cc + 1], zz[4 * cc + 2], zz[4 * cc + 3]);
+                // entries with a stored weight: z = fl(w - fl(eta*G)) = fl(w + zz)
+                uint32_t bits = obc;
+                if (__any_sync(0xffffffffu, bits != 0u)) {
+                    // the first kFpPre stored entries, independent of each other
+                    int bpos[kFpPre];
+#pragma unroll
+                    for (int u = 0; u < kFpPre; ++u) {
+                        bpos[u] = bits ? __ffs(bits) - 1 : -1;
+                        bits &= bits - 1u;
+                    }
+                    float zs[kFpPre];
+#pragma unroll
+                    for (int u = 0; u < kFpPre; ++u)
+                        if (bpos[u] >= 0) zs[u] = __fadd_rn(wv[u], xr[bpos[u] ^ sw]);
+#pragma unroll
+                    for (int u = 0; u < kFpPre; ++u) {
+                        if (bpos[u] < 0) continue;
+                        const int b = bpos[u];
+                        if (kWrite) {
+                            xr[b ^ sw] = zs[u];
+                        } else {
+                            tsum += zs[u];
+                            kw = fabsf(zs[u]) > a.thr ? (kw | (1u << b)) : (kw & ~(1u << b));
+                        }
                     }
                 }
-                if (rv && wbase + c < a.wpr) a.kbits[row * a.wpr + wbase + c] = kw;
+                for (int u = kFpPre; bits; ++u) {   // rows with more stored weights in this word
+                    const int b = __ffs(bits) - 1;
+                    bits &= bits - 1u;
+                    float *xe = xr + (b ^ sw);
+                    const float z = __fadd_rn(__ldg(a.old_val + ow + u), *xe);
+                    if (kWrite) {
+                        *xe = z;
+                    } else {
+                        tsum += z;
+                        kw = fabsf(z) > a.thr ? (kw | (1u << b)) : (kw & ~(1u << b));
+                    }
+                }
+                if (!kWrite) {
+                    if (rv && word < a.wpr) a.kbits[row * a.wpr + word] = kw;
+                    cnt += __popc(kw);
+                    if (c % kFpTileWords == kFpTileWords - 1) {   // segment complete
+                        const int seg = word / kFpTileWords;
+                        if (rv && seg < a.nt) a.counts[row * a.nt + seg] = (int32_t)cnt;
+                        cnt = 0;
+                    }
+                } else {
+                    // the keep bits come from the count pass, so the positions
+                    // agree with the row pointers by construction
+                    const uint32_t kb = cur.kb[c];
+                    if (rv && word < a.wpr && a.wordpos) a.wordpos[row * a.wpr + word] = imin(pos, cap32);
+                    tab[lane] = make_int2((int)kb, pos);
+                    __syncwarp();
+                    if (fits)
+                        fp_write_word<false>(xb, tab, lx, lt, word * 32 + lane, a.thr, cap32, a.out_col, a.out_val);
+                    else
+                        fp_write_word<true>(xb, tab, lx, lt, word * 32 + lane, a.thr, cap32, a.out_col, a.out_val);
+                    pos += __popc(kb);
+                }
             }
-            if (rv) a.counts[row * a.nt + seg] = (int32_t)cnt;
-            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-            __syncwarp();
-            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(acce + acc)) : "memory");
+            cur = nxt;
+            fp_load_meta<kWrite>(a, t + 2 * gridDim.x, num_tiles, tiles_n, h, rowq, nxt);
         }
-        nonfinite = zsum != zsum;
-        if (__any_sync(0xffffffffu, nonfinite) && lane == 0) s_nonfinite = 1;
+        if (!kWrite && __any_sync(0xffffffffu, tsum != tsum) && lane == 0) s_nonfinite = 1;
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     if (threadIdx.x == 0) {
         if (s_abort) {
             dev_flag(a.hdr, CSRT_DEV_TIMEOUT);
-            a.hdr->timeout_site = 5;
+            a.hdr->timeout_site = kWrite ? 6 : 5;
         }
         if (s_nonfinite) dev_flag(a.hdr, CSRT_DEV_NONFINITE);
     }
@@ -311,43 +505,9 @@ __global__ void __launch_bounds__(256) fp_rowscan_kernel(int32_t *__restrict__ c
     if (lane == 0) rowtot[r] = run;
 }
 
-// 4. One warp per (row, tile): final positions, one coalesced run per word.
-__global__ void __launch_bounds__(256) fp_place_kernel(int32_t m, int32_t k, int32_t nt, int32_t wpr,
-                                                       const int32_t *__restrict__ row_ptr,
-                                                       const int32_t *__restrict__ toff,
-                                                       const uint32_t *__restrict__ kbits,
-                                                       const float *__restrict__ stage, int32_t *__restrict__ out_col,
-                                                       float *__restrict__ out_val, int32_t *__restrict__ wordpos,
-                                                       int64_t capacity) {
-    const int lane = threadIdx.x & 31;
-    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    if (gw >= (int64_t)m * nt) return;
-    const int64_t r = gw / nt;
-    const int t = (int)(gw % nt);
-    const int64_t base = (int64_t)row_ptr[r] + toff[r * nt + t];
-    const float *sv = stage + (r * nt + t) * kFpTileCols;
-    int32_t pre = 0;
-    const unsigned lt = (1u << lane) - 1u;
-    for (int c = 0; c < kFpTileWords; ++c) {
-        const int wi = t * kFpTileWords + c;
-        if (wi >= wpr) break;
-        const uint32_t kw = __ldg(kbits + r * wpr + wi);
-        if (wordpos && lane == 0) wordpos[r * wpr + wi] = (int32_t)imin<int64_t>(base + pre, capacity);
-        if ((kw >> lane) & 1u) {
-            const int32_t idx = pre + __popc(kw & lt);
-            const int64_t p = base + idx;
-            if (p < capacity) {
-                out_col[p] = t * kFpTileCols + c * 32 + lane;
-                out_val[p] = __ldg(sv + idx);
-            }
-        }
-        pre += __popc(kw);
-    }
-}
-
 __global__ void fp_finish_kernel(const int32_t *__restrict__ row_ptr, int32_t m, int64_t capacity,
                                  int32_t *__restrict__ out_row_ptr, WsHeader *hdr) {
-    // row pointers clamped to the capacity, overflow reported
+    // row pointers clamped to the capacity (a no-op unless the output overflowed), overflow reported
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i <= m; i += (int64_t)gridDim.x * blockDim.x) {
         const int64_t v = row_ptr[i];
         out_row_ptr[i] = (int32_t)imin<int64_t>(v, capacity);
@@ -400,7 +560,6 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     uint32_t *kbits = reinterpret_cast<uint32_t *>(base + L.off_kbits);
     int32_t *counts = reinterpret_cast<int32_t *>(base + L.off_counts);
     int32_t *rowtot = reinterpret_cast<int32_t *>(base + L.off_rowtot);
-    float *stage = reinterpret_cast<float *>(base + L.off_stage);
     int32_t *wordpos = reinterpret_cast<int32_t *>(base + L.off_wordpos);
 
     CUtensorMap ma, mb;
@@ -409,8 +568,10 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        CSRT_CHECK_CUDA(
-            cudaFuncSetAttribute(gemm_prox_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmemBytes));
+        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             fp_smem_bytes<false>()));
+        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             fp_smem_bytes<true>()));
         attr_set[dev] = true;
     }
     fp_oldbits_kernel<<<(unsigned)ceil_div<int64_t>(m, 8), 256, 0, s>>>(w_in->row_ptr, w_in->col_idx, m, L.wpr, L.nt,
@@ -428,20 +589,24 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     a.old_val = w_in->val;
     a.kbits = kbits;
     a.counts = counts;
-    a.stage = stage;
+    a.row_ptr_out = w_out->row_ptr;
+    a.out_col = w_out->col_idx;
+    a.out_val = w_out->val;
+    a.wordpos = want_t ? wordpos : nullptr;
+    a.capacity = w_out->capacity;
     a.hdr = static_cast<WsHeader *>(ws);
     const int tiles_m = (int)ceil_div<int64_t>(m, kTcBM), tiles_n = (int)ceil_div<int64_t>(k, kTcBN);
     const int tiles = tiles_m * tiles_n;
-    gemm_prox_tc_kernel<<<imin(tiles, num_sms()), kFpThreads, kTcSmemBytes, s>>>(ma, mb, a, tiles_n, tiles);
+    const unsigned grid = (unsigned)imin(tiles, num_sms());
+    gemm_prox_tc_kernel<false><<<grid, fp_threads<false>(), fp_smem_bytes<false>(), s>>>(ma, mb, a, tiles_n, tiles);
     fp_rowscan_kernel<<<(unsigned)ceil_div<int64_t>((int64_t)m * 32, 256), 256, 0, s>>>(counts, m, L.nt, rowtot);
     count_launch(3);
     // new row pointers: exclusive scan of the row totals (int32: nnz <= M*K < 2^31)
     int rc = scan_exclusive_i32(rowtot, m, w_out->row_ptr, s);
     if (rc) return rc;
-    fp_place_kernel<<<(unsigned)ceil_div<int64_t>((int64_t)m * L.nt * 32, 256), 256, 0, s>>>(
-        m, k, L.nt, L.wpr, w_out->row_ptr, counts, kbits, stage, w_out->col_idx, w_out->val, want_t ? wordpos : nullptr,
-        w_out->capacity);
-    fp_finish_kernel<<<1, 256, 0, s>>>(w_out->row_ptr, m, w_out->capacity, w_out->row_ptr, static_cast<WsHeader *>(ws));
+    gemm_prox_tc_kernel<true><<<grid, fp_threads<true>(), fp_smem_bytes<true>(), s>>>(ma, mb, a, tiles_n, tiles);
+    fp_finish_kernel<<<(unsigned)ceil_div<int64_t>((int64_t)m + 1, 256), 256, 0, s>>>(
+        w_out->row_ptr, m, w_out->capacity, w_out->row_ptr, static_cast<WsHeader *>(ws));
     count_launch(2);
     rc = check_launch("fused weight-gradient + prox kernels");
     if (rc) return rc;

@@ -9,7 +9,9 @@ L2 flushed before every timed launch):
   spmm_fwd (Y = W X), spmm_bwd_t (dX = W^T dY), weight_grad_sddmm (g at the
   stored entries), prox_update_compact twice: with the workload's lambda
   (1e-4, which makes the layer dense) and with a density-preserving lambda*
-  (the (1 - d) quantile of |w - eta*G| / eta, so nnz' ~ nnz).
+  (the (1 - d) quantile of |w - eta*G| / eta, so nnz' ~ nnz), and the dense
+  weight gradient followed by the prox step, fused (weight_grad_prox_update,
+  G never written) and as two calls (weight_grad_dense + prox_update_compact).
 
 For each it prints the time, the algorithmic bytes (each operand touched
 once) and the achieved GB/s, and the FLOP rate for the products. One
@@ -95,6 +97,25 @@ def run_layer(m: int, k: int, density: float, zipf: bool, batches, ops, reps: in
             rows.append({"op": op, "m": m, "k": k, "density": density, "rows": "zipf" if zipf else "uniform",
                          "n": n, "nnz": nnz, "us": round(ms * 1e3, 2), "bytes": byts,
                          "gbs": round(byts / (ms / 1e3) / 1e9, 1), "tflops": round(flops / (ms / 1e3) / 1e12, 2)})
+    if "fused" in ops:
+        # the dense weight gradient G = dY X^T and the prox step on it: fused
+        # (G never written) and as two library calls (G in HBM)
+        for n in batches:
+            xn = xd[:, :n].contiguous()
+            dyn = dyd[:, :n].contiguous()
+            g_full = torch.empty(m, k, device="cuda")
+            variants = (
+                ("fused", lambda: C.weight_grad_prox_update(W, dyn, xn, eta, lam, W_out, ws, g_scratch=g_full)),
+                ("unfused", lambda: (C.weight_grad_dense(dyn, xn, g_full, ws, precision=C.CSRT_PREC_TF32),
+                                     C.prox_update_compact(W, g_full, eta, lam, W_out, ws))),
+            )
+            for tag, fn in variants:
+                ms = _time(fn, reps, flush)
+                nnz_out = W_out.nnz()
+                byts = 4 * n * (m + k) + 8 * nnz + 4 * (m + 1) + 8 * nnz_out + 4 * (m + 1)
+                rows.append({"op": f"grad+prox ({tag})", "m": m, "k": k, "density": density,
+                             "rows": "zipf" if zipf else "uniform", "n": n, "nnz": nnz, "nnz_out": nnz_out,
+                             "us": round(ms * 1e3, 2), "bytes": byts, "gbs": round(byts / (ms / 1e3) / 1e9, 1)})
     if "prox" in ops:
         for tag, lam_v in (("lambda=1e-4", lam), ("lambda*", density_preserving_lambda(w, g, eta, density))):
             def fn(lam_v=lam_v):
@@ -114,7 +135,7 @@ def run_layer(m: int, k: int, density: float, zipf: bool, batches, ops, reps: in
 
 def main(argv=None):
     p = argparse.ArgumentParser()
-    p.add_argument("--op", choices=["all", "spmm_fwd", "spmm_bwd_t", "sddmm", "prox"], default="all")
+    p.add_argument("--op", choices=["all", "spmm_fwd", "spmm_bwd_t", "sddmm", "prox", "fused"], default="all")
     p.add_argument("--m", type=int, default=4096)
     p.add_argument("--k", type=int, default=4096)
     p.add_argument("--density", type=float, nargs="*", default=list(DENSITIES))
@@ -123,7 +144,7 @@ def main(argv=None):
     p.add_argument("--reps", type=int, default=10)
     p.add_argument("--json", action="store_true")
     a = p.parse_args(argv)
-    ops = {"spmm_fwd", "spmm_bwd_t", "sddmm", "prox"} if a.op == "all" else {a.op}
+    ops = {"spmm_fwd", "spmm_bwd_t", "sddmm", "prox", "fused"} if a.op == "all" else {a.op}
     zipfs = {"both": (False, True), "yes": (True,), "no": (False,)}[a.zipf]
     out = []
     for d in a.density:

@@ -32,7 +32,7 @@ from . import csrtrain as C
 class SparseNet:
     def __init__(self, layers, dense_weights, biases, batch: int, in_shape, *, device="cuda",
                  precision: int = C.CSRT_PREC_TF32, stream=None, grad_per_layer: bool = False,
-                 fused: bool = False):
+                 fused: bool = True):
         """layers: layer dicts; dense_weights/biases: numpy arrays, one per fc/conv
         layer (weights M x K, zero off the initial pattern); in_shape: (K,) for an
         fc-first net or (C, H, W) for a conv-first net. The dense gradients of

@@ -186,3 +186,71 @@ def test_fc_head_full_size_step(C):
     _run_and_compare(C, net, layers, cfg["X"], cfg["labels"], cfg["eta"], cfg["lambda"], "prox", 1)
     net.reset_weights()
     _run_and_compare(C, net, layers, cfg["X"], cfg["labels"], cfg["eta"], cfg["lambda"], "debias", 1)
+
+
+def _assert_prox_within_bound(w_gpu, W_old, d, x, eta, lam, what):
+    """The fused prox step (G never written) against the oracle's fp64 G from
+    the same dL/dpre and layer input. G_gpu is within the TF32 summation bound
+    tol of G, so z = w - eta*G moves by at most dz = eta*tol plus the two fp32
+    roundings: every entry with | |z| - thr | > dz must take the oracle's keep
+    decision, and every kept value must be within dz of z - sign(z)*thr."""
+    got, t = _host_csr(w_gpu)
+    M, K = W_old.rows, W_old.cols
+    n = x.shape[1]
+    G = O.weight_grad_dense(d, x)
+    S = O.weight_grad_dense(np.abs(d), np.abs(x))
+    from tests.parity import TF32_OPERAND, U32, gamma
+    tol = gamma(n + 1) * S + U32 * np.abs(G) + 2 * TF32_OPERAND * S + 1e-30
+    w0 = csr_dense(W_old.row_ptr, W_old.col_idx, W_old.val, M, K).astype(np.float64)
+    thr = float(np.float32(eta) * np.float32(lam))
+    z = w0 - eta * G
+    dz = 2.0 * (eta * tol + U32 * (eta * np.abs(G) + np.abs(z))) + 1e-30
+    keep = np.zeros((M, K), dtype=bool)
+    keep[np.repeat(np.arange(M), np.diff(got.row_ptr.astype(np.int64))), got.col_idx] = True
+    clear = np.abs(np.abs(z) - thr) > dz
+    wrong = clear & (keep != (np.abs(z) > thr))
+    assert not wrong.any(), f"{what}: {int(wrong.sum())} keep decisions outside the bound"
+    vg = csr_dense(got.row_ptr, got.col_idx, got.val, M, K).astype(np.float64)
+    ref = z - np.sign(z) * thr
+    err = np.abs(vg - ref)[keep]
+    assert np.all(err <= dz[keep] + U32 * np.abs(ref[keep])), f"{what}: kept values beyond the bound"
+    assert np.all(np.diff(got.row_ptr) >= 0) and got.row_ptr[0] == 0
+    for r in range(0, M, max(1, M // 64)):   # sorted, unique columns within sampled rows
+        c = got.col_idx[got.row_ptr[r]:got.row_ptr[r + 1]]
+        assert np.all(np.diff(c) > 0), f"{what}: row {r} columns not increasing"
+    if t is not None:   # the transposed copy is exactly the transpose of the GPU's own CSR
+        trp, tci, tv, tpos = O.csr_transpose(got)
+        np.testing.assert_array_equal(t[0], trp)
+        np.testing.assert_array_equal(t[1], tci)
+        np.testing.assert_array_equal(t[2].view(np.uint32), tv.astype(F32).view(np.uint32))
+        np.testing.assert_array_equal(t[3], tpos)
+    return int(keep.sum())
+
+
+@pytest.mark.parametrize("workload", ["mlp", "fc_head"])
+def test_fused_prox_step(C, workload):
+    """The network's default prox phase: weight gradient and prox update in
+    one tensor-core pass per layer (shapes it does not cover take the
+    unfused calls), checked against the oracle on the GPU's own dL/dpre."""
+    from paper_1905_07931_gb300 import synth
+    from paper_1905_07931_gb300.train import SparseNet, mlp_layers
+    # 320-192-100-10: two layers fused, the last (K = 100) on the unfused calls
+    cfg = synth.mlp(seed=1, sizes=(320, 192, 100, 10)) if workload == "mlp" else synth.fc_head(seed=0)
+    layers = mlp_layers(3)
+    in_dim = cfg["X"].shape[0]
+    net = SparseNet(layers, cfg["W"], cfg["b"], cfg["X"].shape[1], (in_dim,), precision=1)
+    assert net.fused
+    net.x_in.copy_(torch.from_numpy(cfg["X"]))
+    net.labels.copy_(torch.from_numpy(cfg["labels"]))
+    onet = _oracle_net(layers, net)
+    loss = net.step("prox", cfg["eta"], cfg["lambda"])
+    torch.cuda.synchronize()
+    assert net.ws.status()[0] == 0
+    logits, _ = O.net_forward(onet, cfg["X"], cfg["X"].shape[1])
+    oloss, _ = O.softmax_xent(logits, cfg["labels"])
+    assert abs(float(loss[0].item()) - oloss) <= 2e-5 * max(1.0, abs(oloss))
+    for pi, L in enumerate(net.params):
+        W = onet.params[[i for i, l in enumerate(layers) if l["kind"] == "fc"][pi]]["W"]
+        d = L["dpre"].cpu().numpy().reshape(W.rows, -1).astype(np.float64)
+        x = L["xmat"].cpu().numpy().reshape(W.cols, -1).astype(np.float64)
+        _assert_prox_within_bound(net.weights(pi), W, d, x, cfg["eta"], cfg["lambda"], f"layer {pi}")
