@@ -223,13 +223,23 @@ __global__ void __launch_bounds__(256) spmm_fixup_kernel(SpmmArgs a) {
     int last = u;
     while (last + 1 < a.units && a.carry_row[last + 1] == r) ++last;
     const bool epi = a.bias || a.relu || a.mask;
-    for (int j = lane; j < TN; j += 32) {
-        const int col = t * TN + j;
+    // lane j holds columns j, j+32, ...: every carry's loads for them are
+    // independent, so they are issued together, carry by carry in unit order
+    constexpr int kPer = TN / 32;
+    float sum[kPer];
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) sum[q] = 0.f;
+    for (int v = u; v <= last; ++v) {
+        const float *cp = a.carry + ((int64_t)t * a.units + v) * TN + lane;
+#pragma unroll
+        for (int q = 0; q < kPer; ++q) sum[q] += __ldg(cp + 32 * q);
+    }
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+        const int col = t * TN + lane + 32 * q;
         if (col >= a.n) break;
-        float sum = 0.f;
-        for (int v = u; v <= last; ++v) sum += a.carry[((int64_t)t * a.units + v) * TN + j];
         float *yp = a.y + (int64_t)r * a.n + col;
-        float out[1] = {*yp + sum};
+        float out[1] = {*yp + sum[q]};
         if (epi) spmm_epilogue<1>(a, r, col, out);
         *yp = out[0];
     }

@@ -154,6 +154,12 @@ SPMM_CASES = [
     (4, 9, 1, 1.0, False),
     (50, 40, 7, 0.0, False),
     (1000, 600, 1024, 0.02, True),
+    # long rows cut by many work units, one float4 per lane, a ragged
+    # second n-tile, and a larger uniform case
+    (300, 5000, 256, 0.1, False),
+    (129, 1000, 128, 0.2, False),
+    (257, 300, 384, 0.3, True),
+    (2048, 1024, 256, 0.05, False),
 ]
 
 
@@ -207,15 +213,16 @@ def test_fused_epilogues_match_unfused(C, m, k, n, zipf):
     np.testing.assert_array_equal(dx.cpu().numpy().view(np.uint32), dx_ref.cpu().numpy().view(np.uint32))
 
 
-def test_spmm_is_deterministic(C):
+@pytest.mark.parametrize("n", [96, 256])
+def test_spmm_is_deterministic(C, n):
     rng = np.random.default_rng(11)
     a = _sparse(rng, 700, 900, 0.08, zipf=True)
-    x = _dev(rng.standard_normal((900, 96)).astype(F32))
-    ws = _ws(C, 900, 900, 96)
+    x = _dev(rng.standard_normal((900, n)).astype(F32))
+    ws = _ws(C, 900, 900, n)
     w = _gpu_csr(C, a, ws)
     ys = []
     for _ in range(3):
-        y = torch.zeros(700, 96, device="cuda")
+        y = torch.zeros(700, n, device="cuda")
         C.spmm_fwd(w, x, y, ws)
         ys.append(y.cpu().numpy())
     np.testing.assert_array_equal(ys[0].view(np.uint32), ys[1].view(np.uint32))
