@@ -44,6 +44,7 @@ __all__ = [
     "CSR", "csr_from_dense", "csr_to_dense", "csr_abs", "csr_transpose",
     "spmm_fwd", "spmm_bwd_t", "weight_grad_dense", "weight_grad_sddmm",
     "soft_threshold", "prox_update_compact", "debias_update",
+    "rmsprop_direction", "adam_direction", "prox_rmsprop_update_compact", "prox_adam_update_compact",
     "dense_times_compressed_t", "dense_times_compressed",
     "compression_rate",
     "im2col", "col2im", "maxpool2_fwd", "maxpool2_bwd", "relu",
@@ -305,6 +306,80 @@ def prox_update_compact(w: CSR, g: np.ndarray, eta: float, lam: float) -> CSR:
     # (Sterbenz), so the kept value is never zero.
     dense_new = np.where(keep, out, F32(0)).astype(F32)
     return csr_from_dense(dense_new)
+
+
+def rmsprop_direction(g: np.ndarray, v: np.ndarray, beta: float, eps: float):
+    """The moment update and search direction of one Prox-RMSProp step
+    (Algorithm 1), on every M x K entry.
+
+    Algorithm 1 keeps v, the running average of g*g (elementwise), and moves
+    along g / (sqrt(v) + eps). Float32 rules, every operation rounded once,
+    in this order (c = fl32(1 - beta)):
+      v' = fl(fl(beta * v) + fl(c * fl(g * g)))
+      d  = fl(g / fl(fl(sqrt(v')) + eps))
+    Returns (v', d). Pinned by exact hand cases, by the beta = 0 reduction
+    shared with Adam, and by a five-step trajectory against the textbook
+    float64 method.
+    """
+    g = np.asarray(g, dtype=F32)
+    v = np.asarray(v, dtype=F32)
+    beta32, eps32 = F32(beta), F32(eps)
+    c = F32(1) - beta32
+    v_new = (beta32 * v + c * (g * g)).astype(F32)
+    d = (g / (np.sqrt(v_new) + eps32)).astype(F32)
+    return v_new, d
+
+
+def adam_direction(g: np.ndarray, m: np.ndarray, v: np.ndarray, t: int, beta1: float, beta2: float,
+                   eps: float):
+    """The moment updates and search direction of step t >= 1 of Prox-ADAM
+    (Algorithm 2), on every M x K entry.
+
+    Algorithm 2 keeps the first moment m and the second moment v of g, divides
+    each by its bias correction 1 - beta^t, and moves along
+    m_hat / (sqrt(v_hat) + eps). Float32 rules, every operation rounded once,
+    in this order (c_i = fl32(1 - beta_i); the corrections bc_i =
+    fl32(1 - beta_i^t) with the power taken in float64):
+      m' = fl(fl(beta1 * m) + fl(c1 * g))
+      v' = fl(fl(beta2 * v) + fl(c2 * fl(g * g)))
+      m_hat = fl(m' / bc1), v_hat = fl(v' / bc2)
+      d = fl(m_hat / fl(fl(sqrt(v_hat)) + eps))
+    Returns (m', v', d). Pinned like rmsprop_direction.
+    """
+    if int(t) < 1:
+        raise ValueError("the step counter t starts at 1")
+    g = np.asarray(g, dtype=F32)
+    m = np.asarray(m, dtype=F32)
+    v = np.asarray(v, dtype=F32)
+    b1, b2, eps32 = F32(beta1), F32(beta2), F32(eps)
+    c1, c2 = F32(1) - b1, F32(1) - b2
+    bc1 = F32(1.0 - float(b1) ** int(t))
+    bc2 = F32(1.0 - float(b2) ** int(t))
+    m_new = (b1 * m + c1 * g).astype(F32)
+    v_new = (b2 * v + c2 * (g * g)).astype(F32)
+    m_hat = (m_new / bc1).astype(F32)
+    v_hat = (v_new / bc2).astype(F32)
+    d = (m_hat / (np.sqrt(v_hat) + eps32)).astype(F32)
+    return m_new, v_new, d
+
+
+def prox_rmsprop_update_compact(w: CSR, g: np.ndarray, v: np.ndarray, eta: float, lam: float, beta: float,
+                                eps: float):
+    """One Prox-RMSProp step (Algorithm 1) followed by CSR re-compaction:
+    w <- prox_{eta*lambda*||.||_1}(w - eta * d) with d from rmsprop_direction,
+    i.e. prox_update_compact applied to d (the threshold stays eta*lambda, not
+    scaled by the adaptive denominator). Returns (w', v')."""
+    v_new, d = rmsprop_direction(g, v, beta, eps)
+    return prox_update_compact(w, d, eta, lam), v_new
+
+
+def prox_adam_update_compact(w: CSR, g: np.ndarray, m: np.ndarray, v: np.ndarray, t: int, eta: float,
+                             lam: float, beta1: float, beta2: float, eps: float):
+    """One Prox-ADAM step (Algorithm 2) followed by CSR re-compaction:
+    w <- prox_{eta*lambda*||.||_1}(w - eta * d) with d from adam_direction.
+    Returns (w', m', v')."""
+    m_new, v_new, d = adam_direction(g, m, v, t, beta1, beta2, eps)
+    return prox_update_compact(w, d, eta, lam), m_new, v_new
 
 
 def debias_update(w: CSR, g: np.ndarray, eta: float) -> CSR:

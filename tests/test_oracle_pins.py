@@ -354,3 +354,123 @@ def test_pins_catch_a_wrong_threshold_sign():
     thr = F32(d["eta"]) * F32(d["lambda"])
     z = F32(c["w"]) - F32(d["eta"]) * F32(c["g"])
     assert F32(z - thr) != F32(c["out"])            # sign mistake is caught
+
+
+# --- Prox-RMSProp (Algorithm 1) and Prox-ADAM (Algorithm 2) -----------------
+
+def _one_entry(w):
+    return O.csr_from_dense(np.array([[w]], dtype=F32))
+
+
+def _dense_value(csr):
+    return None if csr.nnz == 0 else float(O.csr_to_dense(csr)[0, 0])
+
+
+def test_rmsprop_hand_cases():
+    d = _load("adaptive_prox_cases.json")
+    for c in d["rmsprop"]:
+        g = np.array([[c["g"]]], dtype=F32)
+        v = np.array([[c["v"]]], dtype=F32)
+        v_new, dd = O.rmsprop_direction(g, v, c["beta"], c["eps"])
+        assert v_new[0, 0] == F32(c["v_new"]) and dd[0, 0] == F32(c["d"]), c
+        w_new, v2 = O.prox_rmsprop_update_compact(_one_entry(c["w"]), g, v, d["eta"], d["lambda"], c["beta"],
+                                                  c["eps"])
+        assert _dense_value(w_new) == c["w_new"], c
+        assert v2[0, 0] == F32(c["v_new"])
+
+
+def test_adam_hand_cases():
+    d = _load("adaptive_prox_cases.json")
+    for c in d["adam"]:
+        g = np.array([[c["g"]]], dtype=F32)
+        m = np.array([[c["m"]]], dtype=F32)
+        v = np.array([[c["v"]]], dtype=F32)
+        m_new, v_new, dd = O.adam_direction(g, m, v, c["t"], c["beta1"], c["beta2"], c["eps"])
+        assert (m_new[0, 0], v_new[0, 0], dd[0, 0]) == (F32(c["m_new"]), F32(c["v_new"]), F32(c["d"])), c
+        w_new, m2, v2 = O.prox_adam_update_compact(_one_entry(c["w"]), g, m, v, c["t"], d["eta"], d["lambda"],
+                                                   c["beta1"], c["beta2"], c["eps"])
+        assert _dense_value(w_new) == c["w_new"], c
+        assert m2[0, 0] == F32(c["m_new"]) and v2[0, 0] == F32(c["v_new"])
+
+
+def test_adam_without_momentum_is_rmsprop_without_averaging():
+    # beta1 = beta2 = 0: m_hat = g and v_hat = g*g, the bias corrections are 1;
+    # RMSProp with beta = 0 has v = g*g: the two directions agree bit for bit.
+    rng = np.random.default_rng(5)
+    g = rng.standard_normal((7, 9)).astype(F32)
+    m = rng.standard_normal((7, 9)).astype(F32)
+    v = np.abs(rng.standard_normal((7, 9))).astype(F32)
+    _, _, d_adam = O.adam_direction(g, m, v, 3, 0.0, 0.0, 1e-3)
+    _, d_rms = O.rmsprop_direction(g, v, 0.0, 1e-3)
+    np.testing.assert_array_equal(d_adam.view(np.uint32), d_rms.view(np.uint32))
+
+
+def _textbook_adam(w, gs, eta, b1, b2, eps):
+    m = np.zeros_like(w)
+    v = np.zeros_like(w)
+    for t, g in enumerate(gs, start=1):
+        m = b1 * m + (1 - b1) * g
+        v = b2 * v + (1 - b2) * g * g
+        w = w - eta * (m / (1 - b1 ** t)) / (np.sqrt(v / (1 - b2 ** t)) + eps)
+    return w
+
+
+def _textbook_rmsprop(w, gs, eta, beta, eps):
+    v = np.zeros_like(w)
+    for g in gs:
+        v = beta * v + (1 - beta) * g * g
+        w = w - eta * g / (np.sqrt(v) + eps)
+    return w
+
+
+def test_adaptive_trajectories_match_textbook_float64():
+    # lambda = 0: the prox is the identity (only exact zeros drop), so five
+    # steps must follow the float64 textbook method within float32 rounding
+    rng = np.random.default_rng(21)
+    w0 = rng.standard_normal((6, 10)).astype(F32)
+    gs = [rng.standard_normal((6, 10)).astype(F32) for _ in range(5)]
+    eta, b1, b2, eps = 0.01, 0.9, 0.999, 1e-8
+    w = O.csr_from_dense(w0)
+    m = np.zeros_like(w0)
+    v = np.zeros_like(w0)
+    for t, g in enumerate(gs, start=1):
+        w, m, v = O.prox_adam_update_compact(w, g, m, v, t, eta, 0.0, b1, b2, eps)
+    ref = _textbook_adam(w0.astype(np.float64), [g.astype(np.float64) for g in gs], eta, b1, b2, eps)
+    np.testing.assert_allclose(O.csr_to_dense(w), ref, rtol=0, atol=2e-6)
+    w = O.csr_from_dense(w0)
+    v = np.zeros_like(w0)
+    for g in gs:
+        w, v = O.prox_rmsprop_update_compact(w, g, v, eta, 0.0, 0.9, eps)
+    ref = _textbook_rmsprop(w0.astype(np.float64), [g.astype(np.float64) for g in gs], eta, 0.9, eps)
+    np.testing.assert_allclose(O.csr_to_dense(w), ref, rtol=0, atol=2e-6)
+
+
+def test_adaptive_threshold_is_eta_lambda():
+    # the threshold is eta*lambda, not divided by the adaptive denominator:
+    # Adam's first step moves every entry by about eta (|d| ~ 1), so with
+    # eta*lambda above eta everything starting at 0 is dropped, and below it
+    # everything is kept
+    rng = np.random.default_rng(8)
+    g = rng.standard_normal((5, 8)).astype(F32)
+    zero = O.csr_from_dense(np.zeros((5, 8), dtype=F32))
+    z = np.zeros((5, 8), dtype=F32)
+    w_big, _, _ = O.prox_adam_update_compact(zero, g, z, z, 1, 0.1, 1.5, 0.9, 0.999, 1e-8)
+    w_small, _, _ = O.prox_adam_update_compact(zero, g, z, z, 1, 0.1, 0.5, 0.9, 0.999, 1e-8)
+    assert w_big.nnz == 0 and w_small.nnz == 40
+
+
+def test_pins_catch_a_missing_bias_correction():
+    d = _load("adaptive_prox_cases.json")
+    c = d["adam"][0]
+    c1, c2 = F32(1) - F32(c["beta1"]), F32(1) - F32(c["beta2"])
+    m_new = c1 * F32(c["g"])
+    v_new = c2 * F32(c["g"]) * F32(c["g"])
+    wrong = m_new / (np.sqrt(v_new) + F32(c["eps"]))          # no division by 1 - beta^t
+    assert F32(wrong) != F32(c["d"])
+
+
+def test_pins_catch_the_old_second_moment():
+    d = _load("adaptive_prox_cases.json")
+    c = d["rmsprop"][0]
+    wrong = F32(c["g"]) / (np.sqrt(F32(c["v"])) + F32(c["eps"]))   # v_{t-1} instead of v_t
+    assert F32(wrong) != F32(c["d"])
