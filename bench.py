@@ -59,6 +59,9 @@ def parse_args():
     p.add_argument("--prox-path", choices=["fused", "unfused"], default="fused",
                    help="fused: weight gradient and prox update in one tensor-core pass (G not written)")
     p.add_argument("--profile-ops", action="store_true", help="print the per-operation breakdown to stderr")
+    p.add_argument("--optimizer", choices=["sgd", "rmsprop", "adam"], default="sgd",
+                   help="proximal method of the prox phase: SGD, Prox-RMSProp (Algorithm 1) or Prox-ADAM "
+                        "(Algorithm 2); the adaptive ones take the unfused gradient + prox calls")
     return p.parse_args()
 
 
@@ -280,10 +283,12 @@ def op_bytes(name, info):
         if info.get("transposed"):
             b += 8 * nnz_out + 4 * (M + 1) + 12 * nnz_out + 4 * (K + 1)
         return b
-    if name == "prox_update_compact":
+    if name in ("prox_update_compact", "prox_rmsprop_update_compact", "prox_adam_update_compact"):
         b = 4 * M * K + 8 * nnz + 4 * (M + 1) + 8 * nnz_out + 4 * (M + 1)
         if info.get("transposed"):
             b += 8 * nnz_out + 4 * (M + 1) + 12 * nnz_out + 4 * (K + 1)
+        # the dense moments, read and written: v (RMSProp), m and v (Adam)
+        b += {"prox_rmsprop_update_compact": 8, "prox_adam_update_compact": 16}.get(name, 0) * M * K
         return b
     return None
 
@@ -333,7 +338,7 @@ def main():
     cfg = synth.fc_head(seed=0)
     layers = mlp_layers(3)
     net = SparseNet(layers, cfg["W"], cfg["b"], BATCH, (SIZES[0],), precision=prec,
-                    fused=args.prox_path == "fused")
+                    fused=args.prox_path == "fused", optimizer=args.optimizer)
     x_host = torch.from_numpy(cfg["X"]).pin_memory()
     lab_host = torch.from_numpy(cfg["labels"]).pin_memory()
     net.x_in.copy_(x_host)
@@ -343,9 +348,12 @@ def main():
     eta, lam = cfg["eta"], cfg["lambda"]
 
     def restore():
+        # every step starts from the initial weights, biases and (adaptive
+        # methods) zero moments: each timed step is the first step
         for L, b in zip(net.params, b0):
             L["b"].copy_(b)
             L["cur"] = 0
+        net.reset_optimizer()
 
     # warm-up (eager)
     for _ in range(max(args.warmup, 0)):
@@ -450,7 +458,8 @@ def main():
         "config": {"workload": WORKLOAD, "global_batch": BATCH * world, "per_gpu_batch": BATCH,
                    "layers": list(SIZES), "densities": list(DENSITIES),
                    "weight_grad": "tf32 tcgen05" if prec == C.CSRT_PREC_TF32 else "fp32 simt",
-                   "prox_path": args.prox_path,
+                   "prox_path": args.prox_path if args.optimizer == "sgd" else "unfused",
+                   "optimizer": args.optimizer,
                    "l2": "flushed between steps (256 MB write, outside the timed region)",
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "step_ops": [r["label"] for r in prof]},
@@ -486,12 +495,13 @@ def profile_ops(net, C, torch, eta, lam, flush):
     records = []
     wrapped = {}
     names = ["spmm_fwd", "spmm_bwd_t", "spmm_fwd_bias_act", "spmm_bwd_t_relu", "weight_grad_dense",
-             "weight_grad_sddmm", "prox_update_compact", "weight_grad_prox_update", "debias_update", "bias_act_fwd",
-             "relu_bwd", "bias_grad_sgd", "softmax_xent"]
+             "weight_grad_sddmm", "prox_update_compact", "prox_rmsprop_update_compact", "prox_adam_update_compact",
+             "weight_grad_prox_update", "debias_update", "bias_act_fwd", "relu_bwd", "bias_grad_sgd", "softmax_xent"]
     kernel_of = {"spmm_fwd": "spmm_merge_kernel", "spmm_bwd_t": "spmm_merge_kernel",
                  "spmm_fwd_bias_act": "spmm_merge_kernel", "spmm_bwd_t_relu": "spmm_merge_kernel",
                  "weight_grad_dense": "gemm_tf32_tc_persistent_kernel", "weight_grad_sddmm": "sddmm_kernel",
-                 "prox_update_compact": "prox_rows_kernel", "weight_grad_prox_update": "gemm_prox_tc_kernel",
+                 "prox_update_compact": "prox_rows_kernel", "prox_rmsprop_update_compact": "prox_rows_kernel",
+                 "prox_adam_update_compact": "prox_rows_kernel", "weight_grad_prox_update": "gemm_prox_tc_kernel",
                  "debias_update": "debias_kernel"}
     layer_of = {}
     for i, L in enumerate(net.params):
@@ -511,14 +521,15 @@ def profile_ops(net, C, torch, eta, lam, flush):
                 info = {}
                 W = a[0] if a and isinstance(a[0], C.CSR) else None
                 li = layer_of.get(id(W)) if W is not None else None
+                out_arg = {"prox_update_compact": 4, "prox_rmsprop_update_compact": 7, "prox_adam_update_compact": 10}
                 if nm in ("spmm_fwd", "spmm_bwd_t", "spmm_fwd_bias_act", "spmm_bwd_t_relu", "weight_grad_sddmm",
-                          "prox_update_compact", "weight_grad_prox_update", "debias_update"):
+                          "weight_grad_prox_update", "debias_update") or nm in out_arg:
                     info = {"M": W.rows, "K": W.cols, "W": W}
                     if nm in ("spmm_fwd", "spmm_bwd_t", "spmm_fwd_bias_act", "spmm_bwd_t_relu", "weight_grad_sddmm"):
                         info["n"] = a[1].shape[1] if a[1].dim() == 2 else 0
-                    if nm == "prox_update_compact":
-                        info["W_out"] = a[4]
-                        info["transposed"] = a[4].transposed
+                    if nm in out_arg:
+                        info["W_out"] = a[out_arg[nm]]
+                        info["transposed"] = a[out_arg[nm]].transposed
                     if nm == "weight_grad_prox_update":
                         info["n"] = a[1].shape[1]
                         info["W_out"] = a[5]

@@ -204,12 +204,42 @@ int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_
 int prox_update_compact(const csrt_csr *w_in, const float *g, float eta, float lambda,
                         csrt_csr *w_out, void *ws, size_t ws_bytes, void *stream);
 
+/* prox_rmsprop_update_compact -- one step of Prox-RMSProp (Algorithm 1):
+ * the prox step of prox_update_compact taken along the search direction d
+ * instead of G. v (dense row-major M x K float32, the running average of
+ * G*G, zero before the first step) is updated in place. Per entry, every
+ * operation rounded once to float32 in this order, c = fl32(1 - beta):
+ *   v <- fl(fl(beta*v) + fl(c*fl(G*G)));  d = fl(G / fl(fl(sqrt(v)) + eps))
+ * then t = fl32(eta*d), z = fl32(w - t) and the threshold fl32(eta*lambda)
+ * exactly as in prox_update_compact (the threshold is not scaled by the
+ * adaptive denominator). beta in [0, 1), eps finite and > 0; v must not alias
+ * G. A non-finite d drops the entry and sets CSRT_DEV_NONFINITE. */
+int prox_rmsprop_update_compact(const csrt_csr *w_in, const float *g, float *v, float eta, float lambda,
+                                float beta, float eps, csrt_csr *w_out, void *ws, size_t ws_bytes,
+                                void *stream);
+
+/* prox_adam_update_compact -- step t (t >= 1, counted by the caller) of
+ * Prox-ADAM (Algorithm 2): the prox step along the bias-corrected Adam
+ * direction. m and v (dense row-major M x K float32, the first and second
+ * moments of G, zero before step 1) are updated in place. Per entry, with
+ * c_i = fl32(1 - beta_i) and bc_i = fl32(1 - beta_i^t) (power in float64):
+ *   m <- fl(fl(beta1*m) + fl(c1*G));  v <- fl(fl(beta2*v) + fl(c2*fl(G*G)))
+ *   d = fl(fl(m/bc1) / fl(fl(sqrt(fl(v/bc2))) + eps))
+ * then the prox step of prox_update_compact along d. beta1, beta2 in [0, 1),
+ * eps finite and > 0; m, v and G must not alias each other. */
+int prox_adam_update_compact(const csrt_csr *w_in, const float *g, float *m, float *v, int32_t t, float eta,
+                             float lambda, float beta1, float beta2, float eps, csrt_csr *w_out, void *ws,
+                             size_t ws_bytes, void *stream);
+
 /* weight_grad_prox_update -- weight_grad_dense followed by
  * prox_update_compact without writing G: the tensor-core GEMM's epilogue forms
- * z = w - eta*G from the accumulator, applies the soft threshold of Section
- * 2.2 (Eq. prox, Section 3.3) and stages the kept entries, which a placement
- * pass compacts into w_out (and its transposed arrays when set). The result is
- * bit-identical to weight_grad_dense(precision) + prox_update_compact.
+ * z = w - eta*G from the accumulator and applies the soft threshold of Section
+ * 2.2 (Eq. prox, Section 3.3). The GEMM runs twice: a count pass writes the
+ * keep bitmask and per-row counts, and after the row-pointer scan a write pass
+ * recomputes the same accumulator and writes the kept entries of w_out at
+ * their final positions (the transposed arrays, when set, are then built from
+ * the bitmask). The result is bit-identical to weight_grad_dense(precision) +
+ * prox_update_compact.
  * The fused path runs for precision CSRT_PREC_TF32 on tcgen05 GPUs with
  * n % 4 == 0, rows and cols >= 64, cols % 32 == 0, cols <= 16384 and 16-byte
  * aligned dY and X; otherwise the two calls run unfused through g_scratch

@@ -24,6 +24,8 @@
 // kernels: per 32-row block and column a bitmask of the rows present, a scan
 // of the per-block counts down each column, a scan over the columns, and a
 // scatter whose rank inside a block is a popcount of the bitmask.
+#include <cmath>
+
 #include "common.cuh"
 
 namespace csrt {
@@ -67,7 +69,27 @@ struct CompactArgs {
     WsHeader *hdr;
     unsigned long long *status;  // one word per tile
     int64_t num_tiles;
+    // adaptive prox step (Algorithms 1 and 2): the gradient is replaced by a
+    // search direction, the moment arrays (dense, like G) updated in place
+    int32_t opt;                 // kOptSgd, kOptRmsprop, kOptAdam
+    float *m, *v;
+    float beta1, beta2, c1, c2, bc1, bc2, eps;
 };
+
+constexpr int32_t kOptSgd = 0, kOptRmsprop = 1, kOptAdam = 2;
+
+// Moment updates and search direction of one adaptive step, every operation
+// rounded once in the order of the definitions: RMSProp (Algorithm 1)
+//   v' = fl(fl(beta2*v) + fl(c2*fl(g*g))),  d = fl(g / fl(fl(sqrt(v')) + eps));
+// Adam (Algorithm 2) with c_i = fl(1 - beta_i), bc_i = fl(1 - beta_i^t)
+//   m' = fl(fl(beta1*m) + fl(c1*g)),  v' as above,
+//   d = fl(fl(m'/bc1) / fl(fl(sqrt(fl(v'/bc2))) + eps)).
+__device__ __forceinline__ float opt_direction(const CompactArgs &a, float g, float &m, float &v) {
+    v = __fadd_rn(__fmul_rn(a.beta2, v), __fmul_rn(a.c2, __fmul_rn(g, g)));
+    if (a.opt == kOptRmsprop) return __fdiv_rn(g, __fadd_rn(__fsqrt_rn(v), a.eps));
+    m = __fadd_rn(__fmul_rn(a.beta1, m), __fmul_rn(a.c1, g));
+    return __fdiv_rn(__fdiv_rn(m, a.bc1), __fadd_rn(__fsqrt_rn(__fdiv_rn(v, a.bc2)), a.eps));
+}
 
 // Decoupled look-back for tile `tile`, run by one whole warp: publishes the
 // tile's aggregate, sums predecessors' aggregates back to the nearest
@@ -180,6 +202,24 @@ __global__ void __launch_bounds__(kCThreads) compact_kernel(CompactArgs a) {
         } else {
 #pragma unroll
             for (int c = 0; c < 4; ++c) v[q][c] = (e + c < e1) ? a.src[e + c] : 0.f;
+        }
+    }
+
+    // 1b. Adaptive prox: the gradient becomes the search direction, the
+    // moments are updated in place.
+    if (kProx && a.opt != kOptSgd) {
+#pragma unroll
+        for (int q = 0; q < kCQuads; ++q) {
+            const int64_t e = e0 + 4 * (int64_t)(q * kCThreads + tid);
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                if (e + c < e1) {
+                    float mm = a.opt == kOptAdam ? a.m[e + c] : 0.f, vv = a.v[e + c];
+                    v[q][c] = opt_direction(a, v[q][c], mm, vv);
+                    if (a.opt == kOptAdam) a.m[e + c] = mm;
+                    a.v[e + c] = vv;
+                }
+            }
         }
     }
 
@@ -590,10 +630,30 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
     // while G streams in: row pointers, cleared bitmask, this thread's old entries
     for (int i = tid; i <= nrows; i += kCThreads) s_rp[i] = a.in_row_ptr[r0 + i];
     for (int i = tid; i < (n_el + 31) / 32; i += kCThreads) onbits[i] = 0u;
+    bool waited = false;
+    if (a.opt != kOptSgd) {
+        // adaptive prox: the tile's G becomes the search direction (moments
+        // updated in place, 16-byte rows since K % 4 == 0) before the fold
+        if (!row_mbar_wait(&s_bar, 0)) s_fail = 1;
+        waited = true;
+        float *mp = a.m + (int64_t)r0 * K, *vp = a.v + (int64_t)r0 * K;
+        for (int b = 4 * tid; b < n_el; b += 4 * kCThreads) {
+            const float4 g4 = *reinterpret_cast<const float4 *>(tile_v + b);
+            float4 m4 = a.opt == kOptAdam ? *reinterpret_cast<const float4 *>(mp + b) : make_float4(0.f, 0.f, 0.f, 0.f);
+            float4 v4 = *reinterpret_cast<const float4 *>(vp + b);
+            float4 d4;
+            d4.x = opt_direction(a, g4.x, m4.x, v4.x);
+            d4.y = opt_direction(a, g4.y, m4.y, v4.y);
+            d4.z = opt_direction(a, g4.z, m4.z, v4.z);
+            d4.w = opt_direction(a, g4.w, m4.w, v4.w);
+            if (a.opt == kOptAdam) *reinterpret_cast<float4 *>(mp + b) = m4;
+            *reinterpret_cast<float4 *>(vp + b) = v4;
+            *reinterpret_cast<float4 *>(tile_v + b) = d4;
+        }
+    }
     __syncthreads();
     const int32_t s0 = s_rp[0], s1 = s_rp[nrows];
     constexpr int kOld = 4;   // old entries held per thread per pass
-    bool waited = false;
     for (int32_t kb = s0; kb < s1; kb += kOld * kCThreads) {
         int32_t pos_e[kOld];
         float wv[kOld];
@@ -741,16 +801,28 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
 
 // Returns through *bits_done whether the prox kernel emitted the keep bitmask
 // (then the transposed copy is built from it).
+struct OptParams {
+    int32_t opt;
+    float *m, *v;
+    float beta1, beta2, eps;
+    int32_t t;
+};
+
 static int compact_launch(bool prox, const float *src, int32_t rows, int32_t cols, const csrt_csr *in,
                           float eta, float thr, csrt_csr *out, void *ws, size_t ws_bytes,
-                          cudaStream_t s, bool want_bits = false, bool *bits_done = nullptr) {
+                          cudaStream_t s, bool want_bits = false, bool *bits_done = nullptr,
+                          const OptParams *op = nullptr) {
     if (bits_done) *bits_done = false;
     const int64_t elems = (int64_t)rows * cols;
     if (elems == 0) {
         CSRT_CHECK_CUDA(cudaMemsetAsync(out->row_ptr, 0, sizeof(int32_t) * ((size_t)rows + 1), s));
         return CSRT_OK;
     }
-    const bool row_path = cols % 4 == 0 && cols <= kRowMaxK && (reinterpret_cast<uintptr_t>(src) & 15) == 0;
+    const bool opt_aligned =
+        op == nullptr || op->opt == kOptSgd ||
+        ((reinterpret_cast<uintptr_t>(op->v) | reinterpret_cast<uintptr_t>(op->m)) & 15) == 0;
+    const bool row_path = cols % 4 == 0 && cols <= kRowMaxK && (reinterpret_cast<uintptr_t>(src) & 15) == 0 &&
+                          opt_aligned;
     const int32_t rows_per_tile = row_path ? imax<int32_t>(1, kRowBudget / cols) : 0;
     const int64_t tiles = row_path ? ceil_div<int64_t>(rows, rows_per_tile) : ceil_div<int64_t>(elems, kTile);
     CSRT_ARG(ws_bytes >= kWsHeaderBytes + status_bytes(elems), "workspace too small for compaction");
@@ -775,6 +847,19 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
     a.hdr = hdr;
     a.status = status;
     a.num_tiles = tiles;
+    a.opt = op ? op->opt : kOptSgd;
+    a.m = op ? op->m : nullptr;
+    a.v = op ? op->v : nullptr;
+    a.beta1 = a.beta2 = a.c1 = a.c2 = a.bc1 = a.bc2 = a.eps = 0.f;
+    if (op && op->opt != kOptSgd) {
+        a.beta1 = op->beta1;
+        a.beta2 = op->beta2;
+        a.c1 = 1.0f - op->beta1;   // fl32(1 - beta)
+        a.c2 = 1.0f - op->beta2;
+        a.bc1 = (float)(1.0 - pow((double)op->beta1, (double)op->t));   // fl32(1 - beta^t), power in float64
+        a.bc2 = (float)(1.0 - pow((double)op->beta2, (double)op->t));
+        a.eps = op->eps;
+    }
     if (row_path) {
         const size_t tile_cap = (size_t)rows_per_tile * cols;
         const size_t smem = prox ? (tile_cap + (tile_cap + 31) / 32 + rows_per_tile + 1) * sizeof(float) : 0;
@@ -1187,8 +1272,8 @@ int csr_transpose(csrt_csr *w, void *ws, size_t ws_bytes, void *stream) {
     return transpose_impl(w, ws, ws_bytes, as_stream(stream));
 }
 
-int prox_update_compact(const csrt_csr *w_in, const float *g, float eta, float lambda, csrt_csr *w_out,
-                        void *ws, size_t ws_bytes, void *stream) {
+static int prox_impl(const csrt_csr *w_in, const float *g, float eta, float lambda, csrt_csr *w_out, void *ws,
+                     size_t ws_bytes, void *stream, const OptParams *op) {
     int rc = check_csr(w_in, false);
     if (rc) return rc;
     rc = check_csr(w_out, false);
@@ -1205,10 +1290,60 @@ int prox_update_compact(const csrt_csr *w_in, const float *g, float eta, float l
     const bool want_t = w_out->t_row_ptr != nullptr;
     if (want_t) CSRT_ARG(w_out->t_col_idx && w_out->t_val && w_out->t_pos, "transposed arrays partly set");
     bool bits = false;
-    rc = compact_launch(true, g, w_in->rows, w_in->cols, w_in, eta, thr, w_out, ws, ws_bytes, s, want_t, &bits);
+    rc = compact_launch(true, g, w_in->rows, w_in->cols, w_in, eta, thr, w_out, ws, ws_bytes, s, want_t, &bits, op);
     if (rc) return rc;
     if (want_t) rc = bits ? transpose_from_bits(w_out, ws, ws_bytes, s) : transpose_impl(w_out, ws, ws_bytes, s);
     return rc;
+}
+
+int prox_update_compact(const csrt_csr *w_in, const float *g, float eta, float lambda, csrt_csr *w_out,
+                        void *ws, size_t ws_bytes, void *stream) {
+    return prox_impl(w_in, g, eta, lambda, w_out, ws, ws_bytes, stream, nullptr);
+}
+
+static int check_moments(const csrt_csr *w, const float *g, const float *m, const float *v, float eps) {
+    const bool empty = w == nullptr || (int64_t)w->rows * w->cols == 0;
+    CSRT_ARG(empty || v != nullptr, "v is NULL");
+    CSRT_ARG(v == nullptr || (v != g && v != m), "v must not alias G or m");
+    CSRT_ARG(m == nullptr || m != g, "m must not alias G");
+    CSRT_ARG(eps > 0.f && eps <= 3.0e38f, "eps must be finite and > 0");
+    return CSRT_OK;
+}
+
+int prox_rmsprop_update_compact(const csrt_csr *w_in, const float *g, float *v, float eta, float lambda,
+                                float beta, float eps, csrt_csr *w_out, void *ws, size_t ws_bytes, void *stream) {
+    int rc = check_moments(w_in, g, nullptr, v, eps);
+    if (rc) return rc;
+    CSRT_ARG(beta >= 0.f && beta < 1.f, "beta must be in [0, 1)");
+    OptParams op;
+    op.opt = kOptRmsprop;
+    op.m = nullptr;
+    op.v = v;
+    op.beta1 = 0.f;
+    op.beta2 = beta;
+    op.eps = eps;
+    op.t = 1;
+    return prox_impl(w_in, g, eta, lambda, w_out, ws, ws_bytes, stream, &op);
+}
+
+int prox_adam_update_compact(const csrt_csr *w_in, const float *g, float *m, float *v, int32_t t, float eta,
+                             float lambda, float beta1, float beta2, float eps, csrt_csr *w_out, void *ws,
+                             size_t ws_bytes, void *stream) {
+    int rc = check_moments(w_in, g, m, v, eps);
+    if (rc) return rc;
+    const bool empty = w_in == nullptr || (int64_t)w_in->rows * w_in->cols == 0;
+    CSRT_ARG(empty || m != nullptr, "m is NULL");
+    CSRT_ARG(t >= 1, "the step counter t starts at 1 (got %d)", t);
+    CSRT_ARG(beta1 >= 0.f && beta1 < 1.f && beta2 >= 0.f && beta2 < 1.f, "beta1 and beta2 must be in [0, 1)");
+    OptParams op;
+    op.opt = kOptAdam;
+    op.m = m;
+    op.v = v;
+    op.beta1 = beta1;
+    op.beta2 = beta2;
+    op.eps = eps;
+    op.t = t;
+    return prox_impl(w_in, g, eta, lambda, w_out, ws, ws_bytes, stream, &op);
 }
 
 }  // extern "C"

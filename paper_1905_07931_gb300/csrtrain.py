@@ -57,6 +57,10 @@ _SIGS = {
     "prox_update_compact": [POINTER(csrt_csr), c_void_p, c_float, c_float, POINTER(csrt_csr), c_void_p,
                             c_size_t, c_void_p],
     "debias_update": [POINTER(csrt_csr), c_void_p, c_float, c_void_p],
+    "prox_rmsprop_update_compact": [POINTER(csrt_csr), c_void_p, c_void_p, c_float, c_float, c_float, c_float,
+                                    POINTER(csrt_csr), c_void_p, c_size_t, c_void_p],
+    "prox_adam_update_compact": [POINTER(csrt_csr), c_void_p, c_void_p, c_void_p, c_int32, c_float, c_float,
+                                 c_float, c_float, c_float, POINTER(csrt_csr), c_void_p, c_size_t, c_void_p],
     "weight_grad_prox_update": [POINTER(csrt_csr), c_void_p, c_void_p, c_int32, c_float, c_float, c_int32, c_void_p,
                                 POINTER(csrt_csr), c_void_p, c_size_t, c_void_p],
     "csrt_bias_act_fwd": [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p],
@@ -291,6 +295,28 @@ def prox_update_compact(w_in: CSR, g: torch.Tensor, eta: float, lam: float, w_ou
     _f32(g, "G", w_in.rows * w_in.cols)
     _check(lib().prox_update_compact(w_in.struct, _ptr(g), float(eta), float(lam), w_out.struct, ws.ptr,
                                      ws.nbytes, _stream(stream)), "prox_update_compact")
+
+
+def prox_rmsprop_update_compact(w_in: CSR, g: torch.Tensor, v: torch.Tensor, eta: float, lam: float, beta: float,
+                                eps: float, w_out: CSR, ws: Workspace, stream=None):
+    """One Prox-RMSProp step (Algorithm 1); v (M x K) is updated in place."""
+    _f32(g, "G", w_in.rows * w_in.cols)
+    _f32(v, "v", w_in.rows * w_in.cols)
+    _check(lib().prox_rmsprop_update_compact(w_in.struct, _ptr(g), _ptr(v), float(eta), float(lam), float(beta),
+                                             float(eps), w_out.struct, ws.ptr, ws.nbytes, _stream(stream)),
+           "prox_rmsprop_update_compact")
+
+
+def prox_adam_update_compact(w_in: CSR, g: torch.Tensor, m: torch.Tensor, v: torch.Tensor, t: int, eta: float,
+                             lam: float, beta1: float, beta2: float, eps: float, w_out: CSR, ws: Workspace,
+                             stream=None):
+    """Step t >= 1 of Prox-ADAM (Algorithm 2); m and v (M x K) are updated in place."""
+    _f32(g, "G", w_in.rows * w_in.cols)
+    _f32(m, "m", w_in.rows * w_in.cols)
+    _f32(v, "v", w_in.rows * w_in.cols)
+    _check(lib().prox_adam_update_compact(w_in.struct, _ptr(g), _ptr(m), _ptr(v), int(t), float(eta), float(lam),
+                                          float(beta1), float(beta2), float(eps), w_out.struct, ws.ptr, ws.nbytes,
+                                          _stream(stream)), "prox_adam_update_compact")
 
 
 def weight_grad_prox_update(w_in: CSR, dy: torch.Tensor, x: torch.Tensor, eta: float, lam: float, w_out: CSR,

@@ -32,16 +32,30 @@ from . import csrtrain as C
 class SparseNet:
     def __init__(self, layers, dense_weights, biases, batch: int, in_shape, *, device="cuda",
                  precision: int = C.CSRT_PREC_TF32, stream=None, grad_per_layer: bool = False,
-                 fused: bool = True):
+                 fused: bool = True, optimizer: str = "sgd", beta1: float = 0.9, beta2: float = 0.999,
+                 rms_beta: float = 0.9, eps: float = 1e-8):
         """layers: layer dicts; dense_weights/biases: numpy arrays, one per fc/conv
         layer (weights M x K, zero off the initial pattern); in_shape: (K,) for an
         fc-first net or (C, H, W) for a conv-first net. The dense gradients of
         all layers share one buffer unless grad_per_layer is set (then each
-        layer's G stays readable after the step)."""
+        layer's G stays readable after the step).
+
+        optimizer selects the proximal method of the prox phase: "sgd" (the
+        proximal gradient step), "rmsprop" (Prox-RMSProp, Algorithm 1, decay
+        rms_beta) or "adam" (Prox-ADAM, Algorithm 2, decays beta1 and beta2);
+        eps is the safeguard of both. The adaptive methods keep dense M x K
+        moment arrays per layer and count their steps on the host (the step
+        number is passed by value, so a captured graph replays the step it was
+        captured at). The debias phase is plain SGD in every case."""
+        if optimizer not in ("sgd", "rmsprop", "adam"):
+            raise ValueError(f"unknown optimizer {optimizer!r}")
+        self.optimizer = optimizer
+        self.beta1, self.beta2, self.rms_beta, self.eps = beta1, beta2, rms_beta, eps
+        self.t = 0
         self.grad_per_layer = grad_per_layer
-        # the prox phase applies the update in the gradient GEMM's epilogue (G is
-        # not written) unless each layer's G is to stay readable
-        self.fused = fused and not grad_per_layer
+        # the SGD prox phase applies the update in the gradient GEMM's epilogue
+        # (G is not written) unless each layer's G is to stay readable
+        self.fused = fused and not grad_per_layer and optimizer == "sgd"
         self.layers = [dict(l) for l in layers]
         self.batch = int(batch)
         self.device = device
@@ -98,6 +112,10 @@ class SparseNet:
                 if L["needs_dx"]:
                     L["dx"] = torch.zeros_like(cur)
                 L["g"] = torch.zeros(M * K, **dev)
+                if optimizer == "adam":
+                    L["m"] = torch.zeros(M, K, **dev)
+                if optimizer != "sgd":
+                    L["v"] = torch.zeros(M, K, **dev)
                 if grad_per_layer:
                     L["G"] = torch.zeros(M, K, **dev)
                 max_rows, max_cols, max_n = max(max_rows, M), max(max_cols, K), max(max_n, n)
@@ -162,6 +180,8 @@ class SparseNet:
         """One training step on the data in ``x_in`` / ``labels``. Returns the
         device tensor whose element 0 is the mean loss (not synchronised)."""
         s = self.stream
+        if phase == "prox":
+            self.t += 1   # step number of the adaptive methods (Algorithms 1 and 2)
         self.forward()
         C.softmax_xent(self.logits, self.labels, self.dlogits, self.loss, s)
         d = self.dlogits
@@ -200,6 +220,11 @@ class SparseNet:
                     Wn = L["W"][1 - L["cur"]]
                     if self.fused:
                         C.weight_grad_prox_update(W, dpre, L["xmat"], eta, lam, Wn, self.ws, self.precision, G, s)
+                    elif self.optimizer == "rmsprop":
+                        C.prox_rmsprop_update_compact(W, G, L["v"], eta, lam, self.rms_beta, self.eps, Wn, self.ws, s)
+                    elif self.optimizer == "adam":
+                        C.prox_adam_update_compact(W, G, L["m"], L["v"], self.t, eta, lam, self.beta1, self.beta2,
+                                                   self.eps, Wn, self.ws, s)
                     else:
                         C.prox_update_compact(W, G, eta, lam, Wn, self.ws, s)
                     L["cur"] = 1 - L["cur"]
@@ -223,6 +248,14 @@ class SparseNet:
         for L in self.params:
             L["cur"] = 0
             C.csr_from_dense(L["W0"], L["W"][0], self.ws, self.stream)
+
+    def reset_optimizer(self):
+        """Zero the adaptive moments and the step counter."""
+        self.t = 0
+        for L in self.params:
+            for key in ("m", "v"):
+                if key in L:
+                    L[key].zero_()
 
 
 def mlp_layers(n_layers: int):

@@ -482,3 +482,121 @@ def test_bias_relu_softmax(C):
         rl, rdz = O.softmax_xent(z, lab)
         assert abs(loss[0].item() - rl) <= 1e-5 * max(1, abs(rl))
         assert_close(dz.cpu().numpy(), rdz, rtol=1e-4, atol=1e-7, what="softmax dz")
+
+
+# --- Prox-RMSProp (Algorithm 1) and Prox-ADAM (Algorithm 2) -----------------
+
+def test_adaptive_hand_cases_on_gpu(C):
+    with open(os.path.join(GOLD, "adaptive_prox_cases.json")) as f:
+        d = json.load(f)
+
+    def run(cases, adam, t=1):
+        k = len(cases)
+        w0 = np.array([[c["w"] for c in cases]], dtype=F32)
+        g = _dev(np.array([[c["g"] for c in cases]], dtype=F32))
+        v = _dev(np.array([[c["v"] for c in cases]], dtype=F32))
+        ws = _ws(C, 1, k, 1)
+        w = _gpu_csr(C, w0, ws)
+        out = C.CSR(1, k)
+        if adam:
+            m = _dev(np.array([[c["m"] for c in cases]], dtype=F32))
+            c0 = cases[0]
+            C.prox_adam_update_compact(w, g, m, v, t, d["eta"], d["lambda"], c0["beta1"], c0["beta2"], c0["eps"],
+                                       out, ws)
+            assert m.cpu().numpy()[0].tolist() == [c["m_new"] for c in cases]
+        else:
+            c0 = cases[0]
+            C.prox_rmsprop_update_compact(w, g, v, d["eta"], d["lambda"], c0["beta"], c0["eps"], out, ws)
+        assert v.cpu().numpy()[0].tolist() == [c["v_new"] for c in cases]
+        (rp, ci, vals), _ = out.to_host()
+        dense = csr_dense(rp, ci, vals, 1, k)[0]
+        for j, c in enumerate(cases):
+            assert (dense[j] if dense[j] != 0 else None) == c["w_new"], c
+        assert ws.status()[0] == 0
+
+    run(d["rmsprop"], adam=False)
+    run([c for c in d["adam"] if c["t"] == 1], adam=True, t=1)
+    run([c for c in d["adam"] if c["t"] == 2], adam=True, t=2)
+
+
+@pytest.mark.parametrize("opt", ["adam", "rmsprop"])
+@pytest.mark.parametrize("m,k,density", [
+    (300, 784, 0.1),        # row tiles
+    (37, 4099, 0.3),        # K % 4 != 0: flat tiles
+    (4097, 3, 0.6),
+    (3, 16384, 0.02),       # the longest row-tile rows
+    (2, 16388, 0.02),       # beyond them: flat tiles
+    (1000, 4096, 0.15),     # the classifier head's last layer
+])
+def test_adaptive_prox_chain_bit_exact(C, opt, m, k, density):
+    """Three adaptive prox steps in a row (double-buffered CSR, moments kept
+    on the GPU), each against the oracle fed the same G and the oracle's own
+    moments: the CSR, its transposed arrays and the moments bit for bit."""
+    rng = np.random.default_rng(m + 3 * k)
+    a = _sparse(rng, m, k, density) * F32(0.1)
+    ws = _ws(C, m, k, 1)
+    bufs = [_gpu_csr(C, a, ws), C.CSR(m, k)]
+    mom = [torch.zeros(m, k, device="cuda"), torch.zeros(m, k, device="cuda")]
+    ref = O.csr_from_dense(a)
+    rm = np.zeros((m, k), dtype=F32)
+    rv = np.zeros((m, k), dtype=F32)
+    eta, lam = 0.01, 0.5
+    for t in range(1, 4):
+        g = (rng.standard_normal((m, k)) * 0.3).astype(F32)
+        if opt == "adam":
+            C.prox_adam_update_compact(bufs[(t - 1) % 2], _dev(g), mom[0], mom[1], t, eta, lam, 0.9, 0.999, 1e-8,
+                                       bufs[t % 2], ws)
+            ref, rm, rv = O.prox_adam_update_compact(ref, g, rm, rv, t, eta, lam, 0.9, 0.999, 1e-8)
+            np.testing.assert_array_equal(mom[0].cpu().numpy().view(np.uint32), rm.view(np.uint32))
+        else:
+            C.prox_rmsprop_update_compact(bufs[(t - 1) % 2], _dev(g), mom[1], eta, lam, 0.9, 1e-8, bufs[t % 2], ws)
+            ref, rv = O.prox_rmsprop_update_compact(ref, g, rv, eta, lam, 0.9, 1e-8)
+        np.testing.assert_array_equal(mom[1].cpu().numpy().view(np.uint32), rv.view(np.uint32))
+        _check_csr_equal(bufs[t % 2], ref)
+        assert ref.nnz > 0
+    assert ws.status()[0] == 0
+
+
+def test_adaptive_prox_unaligned_moments(C):
+    # moments that are not 16-byte aligned take the flat tiles: same result
+    m, k = 64, 256
+    rng = np.random.default_rng(3)
+    a = _sparse(rng, m, k, 0.2)
+    g = (rng.standard_normal((m, k)) * 0.3).astype(F32)
+    ws = _ws(C, m, k, 1)
+    w = _gpu_csr(C, a, ws)
+    store = torch.zeros(2 * m * k + 2, device="cuda")
+    mm, vv = store[1:1 + m * k], store[m * k + 2:]
+    out = C.CSR(m, k)
+    C.prox_adam_update_compact(w, _dev(g), mm, vv, 1, 0.01, 0.5, 0.9, 0.999, 1e-8, out, ws)
+    ref, rm, rv = O.prox_adam_update_compact(O.csr_from_dense(a), g, np.zeros((m, k), F32), np.zeros((m, k), F32),
+                                             1, 0.01, 0.5, 0.9, 0.999, 1e-8)
+    _check_csr_equal(out, ref)
+    np.testing.assert_array_equal(mm.cpu().numpy().view(np.uint32), rm.reshape(-1).view(np.uint32))
+    np.testing.assert_array_equal(vv.cpu().numpy().view(np.uint32), rv.reshape(-1).view(np.uint32))
+
+
+def test_adaptive_prox_nan_and_arguments(C):
+    a = np.array([[1.0, 0.0, 2.0, 0.0]], dtype=F32)
+    g = _dev(np.array([[np.nan, 1.0, 0.0, 1.0]], dtype=F32))
+    ws = _ws(C, 1, 4, 1)
+    w = _gpu_csr(C, a, ws)
+    out = C.CSR(1, 4)
+    m, v = torch.zeros(1, 4, device="cuda"), torch.zeros(1, 4, device="cuda")
+    C.prox_adam_update_compact(w, g, m, v, 1, 0.5, 0.25, 0.9, 0.999, 1e-8, out, ws)
+    (rp, ci, vals), _ = out.to_host()
+    assert 0 not in ci.tolist()                       # the NaN direction drops its entry
+    assert ws.status()[0] & C.CSRT_DEV_NONFINITE
+    lib = C.lib()
+    bad = [
+        lambda: lib.prox_adam_update_compact(w.struct, C._ptr(g), C._ptr(m), C._ptr(v), 0, 0.5, 0.25, 0.9, 0.999,
+                                             1e-8, out.struct, ws.ptr, ws.nbytes, None),          # t = 0
+        lambda: lib.prox_adam_update_compact(w.struct, C._ptr(g), C._ptr(m), C._ptr(v), 1, 0.5, 0.25, 1.0, 0.999,
+                                             1e-8, out.struct, ws.ptr, ws.nbytes, None),          # beta1 = 1
+        lambda: lib.prox_rmsprop_update_compact(w.struct, C._ptr(g), C._ptr(v), 0.5, 0.25, 0.9, 0.0, out.struct,
+                                                ws.ptr, ws.nbytes, None),                         # eps = 0
+        lambda: lib.prox_rmsprop_update_compact(w.struct, C._ptr(g), C._ptr(g), 0.5, 0.25, 0.9, 1e-8, out.struct,
+                                                ws.ptr, ws.nbytes, None),                         # v aliases G
+    ]
+    for call in bad:
+        assert call() == C.CSRT_ERR_ARG

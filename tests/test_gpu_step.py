@@ -254,3 +254,38 @@ def test_fused_prox_step(C, workload):
         d = L["dpre"].cpu().numpy().reshape(W.rows, -1).astype(np.float64)
         x = L["xmat"].cpu().numpy().reshape(W.cols, -1).astype(np.float64)
         _assert_prox_within_bound(net.weights(pi), W, d, x, cfg["eta"], cfg["lambda"], f"layer {pi}")
+
+
+@pytest.mark.parametrize("optimizer", ["adam", "rmsprop"])
+def test_mlp_adaptive_prox_steps(C, optimizer):
+    """The prox phase with Prox-ADAM (Algorithm 2) or Prox-RMSProp
+    (Algorithm 1): three steps; each layer's G against the oracle on the GPU's
+    own dL/dpre and input, and the update (CSR and moments) bit for bit against
+    the oracle's adaptive step fed the GPU's G and the oracle's moments."""
+    from paper_1905_07931_gb300 import synth
+    from paper_1905_07931_gb300.train import SparseNet, mlp_layers
+    cfg = synth.mlp(seed=2)
+    layers = mlp_layers(3)
+    net = SparseNet(layers, cfg["W"], cfg["b"], 256, (784,), precision=1, grad_per_layer=True,
+                    optimizer=optimizer, beta1=0.9, beta2=0.999, rms_beta=0.9, eps=1e-8)
+    net.x_in.copy_(torch.from_numpy(cfg["X"]))
+    net.labels.copy_(torch.from_numpy(cfg["labels"]))
+    moments = [{"m": np.zeros((L["W"][0].rows, L["W"][0].cols), F32),
+                "v": np.zeros((L["W"][0].rows, L["W"][0].cols), F32)} for L in net.params]
+    eta, lam = 1e-3, 0.05
+    for t in range(1, 4):
+        old = [_host_csr(net.weights(pi))[0] for pi in range(len(net.params))]
+        net.step("prox", eta, lam)
+        torch.cuda.synchronize()
+        assert net.ws.status()[0] == 0 and net.t == t
+        for pi, L in enumerate(net.params):
+            G = L["G"].cpu().numpy()
+            st = moments[pi]
+            if optimizer == "adam":
+                ref, st["m"], st["v"] = O.prox_adam_update_compact(old[pi], G, st["m"], st["v"], t, eta, lam, 0.9,
+                                                                   0.999, 1e-8)
+                np.testing.assert_array_equal(L["m"].cpu().numpy().view(np.uint32), st["m"].view(np.uint32))
+            else:
+                ref, st["v"] = O.prox_rmsprop_update_compact(old[pi], G, st["v"], eta, lam, 0.9, 1e-8)
+            np.testing.assert_array_equal(L["v"].cpu().numpy().view(np.uint32), st["v"].view(np.uint32))
+            _assert_csr_bits(net.weights(pi), ref)
