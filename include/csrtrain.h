@@ -289,6 +289,17 @@ int csrt_im2col(const float *x, int32_t c, int32_t b, int32_t h, int32_t w, int3
 int csrt_col2im(const float *dcols, int32_t c, int32_t b, int32_t h, int32_t w, int32_t k,
                 float *dx, void *stream);
 
+/* csrt_conv2d_sparse_fwd -- the forward product of a convolution layer with
+ * compressed filters (Section 3.2: W x the unfolded input, here without
+ * unfolding it): y[m][s*ho*wo + oy*wo + ox] = act(fl32(sum over the stored
+ * taps t = (ci*k + ky)*k + kx of row m of W of val * x[ci][s][oy+ky][ox+kx]
+ * + bias[m])), float32 accumulation in CSR order. x is c x (b*h*w), y is
+ * W->rows x (b*ho*wo), stride 1, no padding; W has c*k*k columns and at most
+ * 65535 rows. bias (W->rows floats) may be NULL; act = ReLU when relu != 0.
+ * The same product as csrt_im2col then spmm_fwd (up to summation order). */
+int csrt_conv2d_sparse_fwd(const csrt_csr *w, const float *x, int32_t c, int32_t b, int32_t h, int32_t wd,
+                           int32_t k, const float *bias, int32_t relu, float *y, void *stream);
+
 /* 2x2 max pooling, stride 2 (h, w even): y is c x (b*(h/2)*(w/2)); idx (int8)
  * records the winning window position dy*2+dx, first maximum in scan order. */
 int csrt_maxpool2_fwd(const float *x, int32_t c, int32_t b, int32_t h, int32_t w,

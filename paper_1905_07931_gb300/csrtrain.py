@@ -69,6 +69,8 @@ _SIGS = {
     "csrt_softmax_xent": [c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p],
     "csrt_im2col": [c_void_p, c_int32, c_int32, c_int32, c_int32, c_int32, c_void_p, c_void_p],
     "csrt_col2im": [c_void_p, c_int32, c_int32, c_int32, c_int32, c_int32, c_void_p, c_void_p],
+    "csrt_conv2d_sparse_fwd": [POINTER(csrt_csr), c_void_p, c_int32, c_int32, c_int32, c_int32, c_int32, c_void_p,
+                               c_int32, c_void_p, c_void_p],
     "csrt_maxpool2_fwd": [c_void_p, c_int32, c_int32, c_int32, c_int32, c_void_p, c_void_p, c_void_p],
     "csrt_maxpool2_bwd": [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_int32, c_void_p, c_void_p],
     "csrt_flatten": [c_void_p, c_int32, c_int32, c_int32, c_void_p, c_void_p],
@@ -374,6 +376,15 @@ def softmax_xent(z, labels, dz, loss, stream=None):
 def im2col(x, c, b, h, w, k, cols, stream=None):
     _check(lib().csrt_im2col(_ptr(_f32(x, "x")), c, b, h, w, k, _ptr(_f32(cols, "cols")), _stream(stream)),
            "csrt_im2col")
+
+
+def conv2d_sparse_fwd(w: CSR, x, c, b, h, wd, k, bias, relu, y, stream=None):
+    """Convolution with CSR filters read straight from the input (no unfolded matrix)."""
+    _f32(x, "x", c * b * h * wd)
+    _f32(y, "y", w.rows * b * (h - k + 1) * (wd - k + 1))
+    bp = _ptr(_f32(bias, "bias", w.rows)) if bias is not None else None
+    _check(lib().csrt_conv2d_sparse_fwd(w.struct, _ptr(x), c, b, h, wd, k, bp, int(bool(relu)), _ptr(y),
+                                        _stream(stream)), "csrt_conv2d_sparse_fwd")
 
 
 def col2im(dcols, c, b, h, w, k, dx, stream=None):

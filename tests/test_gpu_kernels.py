@@ -600,3 +600,30 @@ def test_adaptive_prox_nan_and_arguments(C):
     ]
     for call in bad:
         assert call() == C.CSRT_ERR_ARG
+
+
+# --- convolution with CSR filters, input read in place -----------------------
+
+@pytest.mark.parametrize("cout,cin,b,h,w,k,density,relu", [
+    (20, 1, 3, 28, 28, 5, 158 / 500, False),      # LeNet-5 conv1 at the SpC density of the layer table
+    (50, 20, 2, 12, 12, 5, 2101 / 25000, False),  # conv2
+    (7, 3, 2, 7, 9, 3, 0.5, True),                # ragged shapes, ReLU
+    (4, 2, 1, 5, 5, 5, 0.0, True),                # no stored taps: bias (and ReLU) only
+    (3, 60, 1, 6, 6, 5, 1.0, False),              # 1500 taps per filter: two staging rounds
+])
+def test_conv2d_sparse_fwd_against_oracle(C, cout, cin, b, h, w, k, density, relu):
+    rng = np.random.default_rng(cout * cin + h)
+    wt = _sparse(rng, cout, cin * k * k, density)
+    x = rng.standard_normal((cin, b, h, w)).astype(F32)
+    bias = rng.standard_normal(cout).astype(F32)
+    ws = _ws(C, cout, cin * k * k, 1)
+    W = _gpu_csr(C, wt, ws, transposed=False)
+    ho, wo = h - k + 1, w - k + 1
+    y = torch.full((cout, b * ho * wo), float("nan"), device="cuda")
+    C.conv2d_sparse_fwd(W, _dev(x.reshape(cin, -1)), cin, b, h, w, k, _dev(bias), relu, y)
+    ref_w = O.csr_from_dense(wt)
+    cols = O.im2col(x, k)
+    pre = O.spmm_fwd(ref_w, cols) + bias.astype(np.float64)[:, None]
+    ref = np.maximum(pre, 0.0) if relu else pre
+    bound = O.spmm_fwd(O.csr_abs(ref_w), np.abs(cols)) + np.abs(bias.astype(np.float64))[:, None]
+    assert_close(y.cpu().numpy(), ref, bound, (np.diff(ref_w.row_ptr) + 1)[:, None], what="conv2d_sparse_fwd")
