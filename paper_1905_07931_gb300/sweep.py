@@ -59,7 +59,8 @@ def density_preserving_lambda(w: np.ndarray, g: np.ndarray, eta: float, density:
     return float(np.quantile(z, 1.0 - density))
 
 
-def run_layer(m: int, k: int, density: float, zipf: bool, batches, ops, reps: int, seed: int = 0):
+def run_layer(m: int, k: int, density: float, zipf: bool, batches, ops, reps: int, seed: int = 0,
+              transposed: bool = True):
     rng = synth.rng_for(seed)
     w = synth.masked_weights(rng, m, k, density, zipf=zipf)
     nmax = max(batches)
@@ -70,7 +71,7 @@ def run_layer(m: int, k: int, density: float, zipf: bool, batches, ops, reps: in
     ws = C.Workspace(m, k, nmax)
     W = C.CSR(m, k)
     C.csr_from_dense(torch.from_numpy(w).cuda(), W, ws)
-    W_out = C.CSR(m, k)
+    W_out = C.CSR(m, k, transposed=transposed)
     nnz = W.nnz()
     flush = torch.empty(256 * 1024 * 1024 // 4, device="cuda")
     xd = torch.from_numpy(x).cuda()
@@ -143,13 +144,15 @@ def main(argv=None):
     p.add_argument("--zipf", choices=["both", "yes", "no"], default="both")
     p.add_argument("--reps", type=int, default=10)
     p.add_argument("--json", action="store_true")
+    p.add_argument("--no-transposed", action="store_true",
+                   help="prox outputs without the transposed arrays (a first layer, whose dX is not needed)")
     a = p.parse_args(argv)
     ops = {"spmm_fwd", "spmm_bwd_t", "sddmm", "prox", "fused"} if a.op == "all" else {a.op}
     zipfs = {"both": (False, True), "yes": (True,), "no": (False,)}[a.zipf]
     out = []
     for d in a.density:
         for z in zipfs:
-            out += run_layer(a.m, a.k, d, z, a.n, ops, a.reps)
+            out += run_layer(a.m, a.k, d, z, a.n, ops, a.reps, transposed=not a.no_transposed)
     if a.json:
         print(json.dumps(out))
     else:
