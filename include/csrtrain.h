@@ -100,6 +100,17 @@ typedef struct csrt_csr {
  * `rows` x `cols` and products with at most `max_n` columns. Host only. */
 int csrt_workspace_bytes(int32_t rows, int32_t cols, int32_t max_n, size_t *bytes);
 
+/* csrt_check_bounded_waits -- failure detection, checked without a fault
+ * (the paper has no counterpart). Runs the library's two kinds of bounded
+ * wait against events that never happen: the decoupled look-back of the
+ * compaction kernels waiting on a predecessor tile that never publishes, and
+ * an mbarrier wait (as in the TMA / tensor-core pipelines) on a barrier
+ * nothing arrives on. Each gives up after its iteration limit (well under a
+ * second), sets CSRT_DEV_TIMEOUT in the status word and returns, leaving the
+ * context usable. Clear the status afterwards (csrt_clear_status). Uses the
+ * first 16 bytes of the workspace scratch. */
+int csrt_check_bounded_waits(void *ws, size_t ws_bytes, void *stream);
+
 /* Zero the whole workspace (status word included) on `stream`. */
 int csrt_workspace_init(void *ws, size_t ws_bytes, void *stream);
 

@@ -799,6 +799,28 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
     }
 }
 
+// The library's bounded waits run against events that never happen (failure
+// detection without a fault): (0) the decoupled look-back of tile 1 while
+// tile 0 never publishes, (1) an mbarrier wait on a barrier nothing arrives
+// on. Each gives up after its iteration limit, sets CSRT_DEV_TIMEOUT (with
+// the site of the wait) and the kernel returns normally.
+__global__ void bounded_wait_check_kernel(unsigned long long *__restrict__ status, WsHeader *hdr, int which) {
+    __shared__ __align__(8) uint64_t bar;
+    if (which == 0) {
+        lookback_warp(status, 1, 0u, hdr);   // status[0] is zero and stays zero
+        return;
+    }
+    if (threadIdx.x == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(cvta_smem(&bar)) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncwarp();
+    if (threadIdx.x == 0 && !row_mbar_wait(&bar, 0)) {
+        dev_flag(hdr, CSRT_DEV_TIMEOUT);
+        hdr->timeout_site = 9;
+    }
+}
+
 // Returns through *bits_done whether the prox kernel emitted the keep bitmask
 // (then the transposed copy is built from it).
 struct OptParams {
@@ -1299,6 +1321,17 @@ static int prox_impl(const csrt_csr *w_in, const float *g, float eta, float lamb
 int prox_update_compact(const csrt_csr *w_in, const float *g, float eta, float lambda, csrt_csr *w_out,
                         void *ws, size_t ws_bytes, void *stream) {
     return prox_impl(w_in, g, eta, lambda, w_out, ws, ws_bytes, stream, nullptr);
+}
+
+int csrt_check_bounded_waits(void *ws, size_t ws_bytes, void *stream) {
+    CSRT_ARG(ws != nullptr && ws_bytes >= kWsHeaderBytes + 2 * sizeof(unsigned long long), "workspace too small");
+    cudaStream_t s = as_stream(stream);
+    unsigned long long *status = reinterpret_cast<unsigned long long *>(ws_scratch(ws));
+    CSRT_CHECK_CUDA(cudaMemsetAsync(status, 0, 2 * sizeof(unsigned long long), s));
+    bounded_wait_check_kernel<<<1, 32, 0, s>>>(status, static_cast<WsHeader *>(ws), 0);
+    bounded_wait_check_kernel<<<1, 32, 0, s>>>(status, static_cast<WsHeader *>(ws), 1);
+    count_launch(2);
+    return check_launch("bounded_wait_check_kernel");
 }
 
 static int check_moments(const csrt_csr *w, const float *g, const float *m, const float *v, float eps) {

@@ -69,6 +69,7 @@ _SIGS = {
     "csrt_softmax_xent": [c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_void_p, c_void_p],
     "csrt_im2col": [c_void_p, c_int32, c_int32, c_int32, c_int32, c_int32, c_void_p, c_void_p],
     "csrt_col2im": [c_void_p, c_int32, c_int32, c_int32, c_int32, c_int32, c_void_p, c_void_p],
+    "csrt_check_bounded_waits": [c_void_p, c_size_t, c_void_p],
     "csrt_conv2d_sparse_fwd": [POINTER(csrt_csr), c_void_p, c_int32, c_int32, c_int32, c_int32, c_int32, c_void_p,
                                c_int32, c_void_p, c_void_p],
     "csrt_maxpool2_fwd": [c_void_p, c_int32, c_int32, c_int32, c_int32, c_void_p, c_void_p, c_void_p],
@@ -376,6 +377,12 @@ def softmax_xent(z, labels, dz, loss, stream=None):
 def im2col(x, c, b, h, w, k, cols, stream=None):
     _check(lib().csrt_im2col(_ptr(_f32(x, "x")), c, b, h, w, k, _ptr(_f32(cols, "cols")), _stream(stream)),
            "csrt_im2col")
+
+
+def check_bounded_waits(ws: Workspace, stream=None):
+    """Run the library's bounded waits against events that never happen; they
+    must give up and set CSRT_DEV_TIMEOUT (read it with ws.status())."""
+    _check(lib().csrt_check_bounded_waits(ws.ptr, ws.nbytes, _stream(stream)), "csrt_check_bounded_waits")
 
 
 def conv2d_sparse_fwd(w: CSR, x, c, b, h, wd, k, bias, relu, y, stream=None):

@@ -627,3 +627,31 @@ def test_conv2d_sparse_fwd_against_oracle(C, cout, cin, b, h, w, k, density, rel
     ref = np.maximum(pre, 0.0) if relu else pre
     bound = O.spmm_fwd(O.csr_abs(ref_w), np.abs(cols)) + np.abs(bias.astype(np.float64))[:, None]
     assert_close(y.cpu().numpy(), ref, bound, (np.diff(ref_w.row_ptr) + 1)[:, None], what="conv2d_sparse_fwd")
+
+
+# --- failure detection: bounded waits give up and report ---------------------
+
+def test_bounded_waits_give_up_and_report(C):
+    """The look-back spin and the mbarrier wait, run against a predecessor and
+    a barrier that never arrive, give up, set CSRT_DEV_TIMEOUT and return;
+    the context stays usable for the next product."""
+    import time
+    ws = _ws(C, 64, 64, 64)
+    ws.clear_status()
+    assert ws.status()[0] == 0
+    t0 = time.time()
+    C.check_bounded_waits(ws)
+    flags, _ = ws.status()
+    assert flags & C.CSRT_DEV_TIMEOUT
+    assert time.time() - t0 < 60
+    ws.clear_status()
+    rng = np.random.default_rng(2)
+    a = _sparse(rng, 64, 64, 0.2)
+    x = rng.standard_normal((64, 16)).astype(F32)
+    w = _gpu_csr(C, a, ws)
+    y = torch.zeros(64, 16, device="cuda")
+    C.spmm_fwd(w, _dev(x), y, ws)
+    ref = O.csr_from_dense(a)
+    assert_close(y.cpu().numpy(), O.spmm_fwd(ref, x), O.spmm_fwd(O.csr_abs(ref), np.abs(x)),
+                 np.diff(ref.row_ptr)[:, None], what="spmm after the timed-out waits")
+    assert ws.status()[0] == 0
