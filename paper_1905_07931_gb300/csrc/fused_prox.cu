@@ -40,7 +40,6 @@ size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
 constexpr int kFpTileCols = 64;                  // columns per segment
 constexpr int kFpTileWords = kFpTileCols / 32;   // 2
 constexpr int kFpMaxK = 16384;
-constexpr int kFpPre = 8;                        // stored old weights per word prefetched into registers
 
 // Launch shape of each pass: epilogue warps and pipeline stages. The count
 // pass is bound by the MMA (4 stages); the write pass by its epilogue, which
@@ -51,17 +50,43 @@ constexpr int kFpPre = 8;                        // stored old weights per word 
 #ifndef CSRT_FP_WRITE_EPI
 #define CSRT_FP_WRITE_EPI 8
 #endif
+#ifndef CSRT_FP_WRITE_PRE
+#define CSRT_FP_WRITE_PRE 8
+#endif
+#ifndef CSRT_FP_WRITE_GROUP
+#define CSRT_FP_WRITE_GROUP 8
+#endif
+// kPre: stored old weights per word prefetched into registers; kGroup: rows
+// of a word handled together in the write pass's column domain.
 template <bool kWrite> struct FpShape;
 template <> struct FpShape<false> {
-    static constexpr int kEpi = CSRT_FP_COUNT_EPI, kStages = CSRT_FP_COUNT_EPI > 8 ? 3 : 4;
+    static constexpr int kEpi = CSRT_FP_COUNT_EPI, kStages = CSRT_FP_COUNT_EPI > 8 ? 3 : 4, kPre = 8, kGroup = 8;
 };
-template <> struct FpShape<true> { static constexpr int kEpi = CSRT_FP_WRITE_EPI, kStages = 3; };
+#ifndef CSRT_FP_WRITE_STAGE_WORDS
+#define CSRT_FP_WRITE_STAGE_WORDS 1
+#endif
+template <> struct FpShape<true> {
+    // kStageWords: words of the span staged before they are written row by
+    // row (the shared memory they take leaves 2 pipeline stages at 4 words,
+    // 3 at 1 or 2). Staging 4 words completes each output sector within one
+    // warp's consecutive stores (196 -> 186 us on a dense 4096 x 9216 output)
+    // but costs the classifier-head step 5% (its outputs are 17-25% dense and
+    // its MMA pipeline needs the third stage): 1 is the default.
+    static constexpr int kEpi = CSRT_FP_WRITE_EPI, kPre = CSRT_FP_WRITE_PRE, kGroup = CSRT_FP_WRITE_GROUP,
+                         kStageWords = CSRT_FP_WRITE_STAGE_WORDS, kStages = kStageWords > 2 ? 2 : 3;
+};
 template <bool kWrite> constexpr int fp_threads() { return 64 + FpShape<kWrite>::kEpi * 32; }
-// Per epilogue warp: a 32 x 32 float buffer, row r's 16-byte chunk c at float
+// Per epilogue warp: 32 x 32 float buffers, row r's 16-byte chunk c at float
 // offset r*32 + ((c ^ (r & 7)) << 2), so that a row written as eight 16-byte
 // stores and a column read one element per lane are both free of bank
-// conflicts; then (write pass) a table of the 32 rows' keep word and position.
-template <bool kWrite> __host__ __device__ constexpr int fp_xfloats() { return 32 * 32 + (kWrite ? 2 * 32 : 0); }
+// conflicts. The count pass needs one; the write pass one per word of its
+// span (it stages the whole span before writing).
+template <bool kWrite> __host__ __device__ constexpr int fp_span_words() {
+    return kTcBN / (FpShape<kWrite>::kEpi / 4) / 32;
+}
+template <bool kWrite> __host__ __device__ constexpr int fp_xfloats() {
+    return 32 * 32 * (kWrite ? FpShape<true>::kStageWords : 1);
+}
 template <bool kWrite> constexpr int fp_smem_bytes() {
     return FpShape<kWrite>::kStages * kTcStageBytes + 1024 + 256 + FpShape<kWrite>::kEpi * fp_xfloats<kWrite>() * 4;
 }
@@ -179,38 +204,53 @@ __device__ __forceinline__ void fp_load_meta(const FpArgs &a, int t, int num_til
     m.pos = (kWrite && sv) ? __ldg(a.row_ptr_out + row) + __ldg(a.counts + row * a.nt + seg0) : 0;
 }
 
-// The first kFpPre stored weights of a word (its bitmask ob, first index o).
+// The first N stored weights of a word (its bitmask ob, first index o).
+template <int N>
 __device__ __forceinline__ void fp_load_words(const float *__restrict__ old_val, uint32_t ob, int32_t o,
-                                              float (&wv)[kFpPre]) {
+                                              float (&wv)[N]) {
     const int nc = __popc(ob);
 #pragma unroll
-    for (int u = 0; u < kFpPre; ++u) wv[u] = u < nc ? __ldg(old_val + o + u) : 0.f;
+    for (int u = 0; u < N; ++u) wv[u] = u < nc ? __ldg(old_val + o + u) : 0.f;
 }
 
-// Write pass, column domain: lane = column of the word, the 32 rows in groups
-// of 8 (independent, so their loads overlap). Row i's kept entries go to
-// consecutive positions from the row's position in the table.
-template <bool kCheck>
-__device__ __forceinline__ void fp_write_word(const float *xb, const int2 *tab, const int (&lx)[8], uint32_t lt,
-                                              int32_t col, float thr, int32_t cap32, int32_t *__restrict__ out_col,
+// Write pass, column domain: lane = column within a word. Rows are taken in
+// groups of G (independent, so their loads overlap); each row's kept entries
+// of the W words of the span form one run of consecutive positions, written
+// word after word with no other store in between, so the 32-byte sector shared
+// by two words' runs is completed at once (a sector left half-written while
+// other rows' stores go by is fetched back from DRAM to be merged).
+template <bool kCheck, int G, int W>
+__device__ __forceinline__ void fp_write_span(const float *xb, const int (&lx)[8], uint32_t lt,
+                                              const uint32_t (&kb)[W], int32_t pos, int32_t col0, float thr,
+                                              int32_t cap32, int32_t *__restrict__ out_col,
                                               float *__restrict__ out_val) {
     const int lane = threadIdx.x & 31;
 #pragma unroll
-    for (int i0 = 0; i0 < 32; i0 += 8) {
-        float z[8];
-        int2 tb[8];
+    for (int i0 = 0; i0 < 32; i0 += G) {
+        uint32_t kw[G][W];
+        float z[G][W];
+        int32_t p[G];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-            tb[u] = tab[i0 + u];
-            z[u] = xb[(i0 + u) * 32 + lx[u]];
+        for (int u = 0; u < G; ++u) {
+            p[u] = __shfl_sync(0xffffffffu, pos, i0 + u);
+#pragma unroll
+            for (int c = 0; c < W; ++c) {
+                kw[u][c] = __shfl_sync(0xffffffffu, kb[c], i0 + u);
+                z[u][c] = xb[c * 1024 + (i0 + u) * 32 + lx[(i0 + u) & 7]];
+            }
         }
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-            const uint32_t kwi = (uint32_t)tb[u].x;
-            const int32_t p = tb[u].y + __popc(kwi & lt);
-            if (((kwi >> lane) & 1u) && (!kCheck || p < cap32)) {
-                out_col[p] = col;
-                out_val[p] = __fsub_rn(z[u], copysignf(thr, z[u]));
+        for (int u = 0; u < G; ++u) {
+            int32_t pw = p[u];
+#pragma unroll
+            for (int c = 0; c < W; ++c) {
+                const uint32_t kwi = kw[u][c];
+                const int32_t q = pw + __popc(kwi & lt);
+                if (((kwi >> lane) & 1u) && (!kCheck || q < cap32)) {
+                    out_col[q] = col0 + c * 32 + lane;
+                    out_val[q] = __fsub_rn(z[u][c], copysignf(thr, z[u][c]));
+                }
+                pw += __popc(kwi);
             }
         }
     }
@@ -233,6 +273,7 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
     gemm_prox_tc_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                         FpArgs a, int32_t tiles_n, int32_t num_tiles) {
     constexpr int kEpi = FpShape<kWrite>::kEpi, kStages = FpShape<kWrite>::kStages;
+    constexpr int kFpPre = FpShape<kWrite>::kPre, kGroup = FpShape<kWrite>::kGroup;
     constexpr int kSpanCols = kTcBN / (kEpi / 4);   // columns per epilogue warp
     constexpr int kSpanWords = kSpanCols / 32;
     static_assert(kSpanWords % kFpTileWords == 0, "a span holds whole segments");
@@ -326,8 +367,6 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
         const int h = e >> 2;     // column span within the tile
         const int64_t rowq = q * 32 + lane;
         float *xb = xbuf + e * fp_xfloats<kWrite>();
-        int2 *tab = reinterpret_cast<int2 *>(xb + 32 * 32);
-        float *xr = xb + lane * 32;   // this thread's row
         const int sw = (lane & 7) << 2;
         int lx[8];   // column-domain offsets: element (i, lane) at i*32 + lx[i & 7]
 #pragma unroll
@@ -357,10 +396,14 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             int32_t pos = cur.pos;   // write pass: position of the row's next kept entry
             uint32_t cnt = 0;
+            if (kWrite) __syncwarp();   // the previous tile's column reads are done
 #pragma unroll
             for (int c = 0; c < kSpanWords; ++c) {
                 const int word = word0 + c;
                 const uint32_t obc = cur.ob[c];
+                constexpr int kSW = kWrite ? FpShape<true>::kStageWords : 1;
+                float *xr = xb + (kWrite ? (c % kSW) * 1024 : 0) + lane * 32;   // this thread's row of the word
+                if (kWrite && c % kSW == 0 && c > 0) __syncwarp();   // the previous group's column reads are done
                 float wv[kFpPre];
 #pragma unroll
                 for (int u = 0; u < kFpPre; ++u) wv[u] = wv_n[u];
@@ -396,7 +439,6 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
                     tsum += ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
                     kw = (k4[0] | k4[1]) | (k4[2] | k4[3]);
                 }
-                if (kWrite) __syncwarp();   // the previous word's column reads are done
 #pragma unroll
                 for (int cc = 0; cc < 8; ++cc)
                     *reinterpret_cast<float4 *>(xr + ((cc << 2) ^ sw)) =
@@ -448,17 +490,27 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
                         cnt = 0;
                     }
                 } else {
-                    // the keep bits come from the count pass, so the positions
-                    // agree with the row pointers by construction
-                    const uint32_t kb = cur.kb[c];
                     if (rv && word < a.wpr && a.wordpos) a.wordpos[row * a.wpr + word] = imin(pos, cap32);
-                    tab[lane] = make_int2((int)kb, pos);
-                    __syncwarp();
-                    if (fits)
-                        fp_write_word<false>(xb, tab, lx, lt, word * 32 + lane, a.thr, cap32, a.out_col, a.out_val);
-                    else
-                        fp_write_word<true>(xb, tab, lx, lt, word * 32 + lane, a.thr, cap32, a.out_col, a.out_val);
-                    pos += __popc(kb);
+                    pos += __popc(cur.kb[c]);
+                    if (c % kSW == kSW - 1) {
+                        // a group of words is staged: write it row by row. The
+                        // keep bits come from the count pass, so the positions
+                        // agree with the row pointers by construction.
+                        __syncwarp();
+                        uint32_t kbg[kSW];
+                        int32_t pg = pos;   // position of the group's first entry
+#pragma unroll
+                        for (int u = 0; u < kSW; ++u) {
+                            kbg[u] = cur.kb[c + 1 - kSW + u];
+                            pg -= __popc(kbg[u]);
+                        }
+                        if (fits)
+                            fp_write_span<false, kGroup, kSW>(xb, lx, lt, kbg, pg, (word + 1 - kSW) * 32, a.thr, cap32,
+                                                              a.out_col, a.out_val);
+                        else
+                            fp_write_span<true, kGroup, kSW>(xb, lx, lt, kbg, pg, (word + 1 - kSW) * 32, a.thr, cap32,
+                                                             a.out_col, a.out_val);
+                    }
                 }
             }
             cur = nxt;
