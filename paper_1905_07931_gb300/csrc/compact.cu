@@ -1025,6 +1025,55 @@ __global__ void __launch_bounds__(1024) scan_single_block_kernel(const int32_t *
     if (tid == 0) out[n] = total;
 }
 
+// The same scan, also writing the row pointers clamped to a CSR's capacity
+// (a no-op unless the output overflows, which is then reported with the
+// needed nnz): `out` keeps the unclamped pointers for the kernel that places
+// the entries (whose stores check the capacity themselves).
+__global__ void __launch_bounds__(1024) scan_clamped_kernel(const int32_t *__restrict__ in, int32_t n,
+                                                            int32_t *__restrict__ out,
+                                                            int32_t *__restrict__ out_clamped, int64_t capacity,
+                                                            WsHeader *hdr) {
+    __shared__ int32_t s_warp[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int per = (n + 1023) / 1024;
+    const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+    int32_t local = 0;
+    for (int i = i0; i < i1; ++i) local += in[i];
+    int32_t incl = local;
+    for (int off = 1; off < 32; off <<= 1) {
+        int32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    int32_t wp = 0, total = 0;
+    for (int w = 0; w < 32; ++w) {
+        if (w < warp) wp += s_warp[w];
+        total += s_warp[w];
+    }
+    int32_t run = incl - local + wp;
+    for (int i = i0; i < i1; ++i) {
+        out[i] = run;
+        out_clamped[i] = (int32_t)imin<int64_t>(run, capacity);
+        run += in[i];
+    }
+    if (tid == 0) {
+        out[n] = total;
+        out_clamped[n] = (int32_t)imin<int64_t>(total, capacity);
+        if (total > capacity) {
+            dev_flag(hdr, CSRT_DEV_CAPACITY);
+            atomicMax(&hdr->required, (unsigned long long)total);
+        }
+    }
+}
+
+int scan_exclusive_i32_clamped(const int32_t *in, int32_t n, int32_t *out, int32_t *out_clamped, int64_t capacity,
+                               void *ws, cudaStream_t s) {
+    scan_clamped_kernel<<<1, 1024, 0, s>>>(in, n, out, out_clamped, capacity, static_cast<WsHeader *>(ws));
+    count_launch();
+    return check_launch("scan_clamped_kernel");
+}
+
 // Write kernel: one block per (32-row block, 256-column chunk). Phase A
 // gathers the block's entries into a shared 32 x 256 value tile and the row
 // bitmask of each column; phase B walks the columns one warp each, lane = row,

@@ -18,8 +18,8 @@
 //     loads only where a weight is stored), forms z = fl(w - fl(eta*G)), keeps
 //     |z| > fl(eta*lambda), and writes the keep bitmask and the kept count of
 //     the segment.
-//  3. fp_rowscan_kernel + scan_single_block_kernel: per-row offsets of the
-//     segments and the new row pointers.
+//  3. fp_rowscan_kernel + scan_clamped_kernel: per-row offsets of the
+//     segments and the new row pointers (clamped to the capacity in w_out).
 //  4. gemm_prox_tc_kernel<write>: the same GEMM again; the epilogue recomputes
 //     z, passes each 32 x 32 block through shared memory and writes the kept
 //     entries of one row at a time at their final positions (a coalesced run
@@ -94,7 +94,7 @@ static_assert(fp_smem_bytes<false>() <= 232448 && fp_smem_bytes<true>() <= 23244
 
 struct FpLayout {
     int32_t nt, wpr;
-    size_t off_obits, off_ostart, off_kbits, off_counts, off_rowtot, off_wordpos, off_tr, total;
+    size_t off_obits, off_ostart, off_kbits, off_counts, off_rowtot, off_rawptr, off_wordpos, off_tr, total;
 };
 
 static size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -109,6 +109,7 @@ static FpLayout fp_layout(int32_t m, int32_t k) {
     L.off_kbits = o;   o += align256((size_t)m * L.wpr * 4);
     L.off_counts = o;  o += align256((size_t)m * L.nt * 4);
     L.off_rowtot = o;  o += align256((size_t)m * 4);
+    L.off_rawptr = o;  o += align256((size_t)(m + 1) * 4);
     L.off_wordpos = o; o += align256((size_t)m * L.wpr * 4);
     L.off_tr = o;      o += align256(transpose_scratch_bytes(m, k));
     L.total = o;
@@ -557,20 +558,8 @@ __global__ void __launch_bounds__(256) fp_rowscan_kernel(int32_t *__restrict__ c
     if (lane == 0) rowtot[r] = run;
 }
 
-__global__ void fp_finish_kernel(const int32_t *__restrict__ row_ptr, int32_t m, int64_t capacity,
-                                 int32_t *__restrict__ out_row_ptr, WsHeader *hdr) {
-    // row pointers clamped to the capacity (a no-op unless the output overflowed), overflow reported
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i <= m; i += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t v = row_ptr[i];
-        out_row_ptr[i] = (int32_t)imin<int64_t>(v, capacity);
-        if (i == m && v > capacity) {
-            dev_flag(hdr, CSRT_DEV_CAPACITY);
-            atomicMax(&hdr->required, (unsigned long long)v);
-        }
-    }
-}
-
-int scan_exclusive_i32(const int32_t *in, int32_t n, int32_t *out, cudaStream_t s);
+int scan_exclusive_i32_clamped(const int32_t *in, int32_t n, int32_t *out, int32_t *out_clamped, int64_t capacity,
+                               void *ws, cudaStream_t s);
 
 }  // namespace csrt
 
@@ -612,6 +601,7 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     uint32_t *kbits = reinterpret_cast<uint32_t *>(base + L.off_kbits);
     int32_t *counts = reinterpret_cast<int32_t *>(base + L.off_counts);
     int32_t *rowtot = reinterpret_cast<int32_t *>(base + L.off_rowtot);
+    int32_t *rawptr = reinterpret_cast<int32_t *>(base + L.off_rawptr);
     int32_t *wordpos = reinterpret_cast<int32_t *>(base + L.off_wordpos);
 
     CUtensorMap ma, mb;
@@ -641,7 +631,7 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     a.old_val = w_in->val;
     a.kbits = kbits;
     a.counts = counts;
-    a.row_ptr_out = w_out->row_ptr;
+    a.row_ptr_out = rawptr;
     a.out_col = w_out->col_idx;
     a.out_val = w_out->val;
     a.wordpos = want_t ? wordpos : nullptr;
@@ -653,13 +643,12 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     gemm_prox_tc_kernel<false><<<grid, fp_threads<false>(), fp_smem_bytes<false>(), s>>>(ma, mb, a, tiles_n, tiles);
     fp_rowscan_kernel<<<(unsigned)ceil_div<int64_t>((int64_t)m * 32, 256), 256, 0, s>>>(counts, m, L.nt, rowtot);
     count_launch(3);
-    // new row pointers: exclusive scan of the row totals (int32: nnz <= M*K < 2^31)
-    int rc = scan_exclusive_i32(rowtot, m, w_out->row_ptr, s);
+    // new row pointers: exclusive scan of the row totals (int32: nnz <= M*K < 2^31), unclamped for the write
+    // pass and clamped to the capacity in w_out (overflow reported)
+    int rc = scan_exclusive_i32_clamped(rowtot, m, rawptr, w_out->row_ptr, w_out->capacity, ws, s);
     if (rc) return rc;
     gemm_prox_tc_kernel<true><<<grid, fp_threads<true>(), fp_smem_bytes<true>(), s>>>(ma, mb, a, tiles_n, tiles);
-    fp_finish_kernel<<<(unsigned)ceil_div<int64_t>((int64_t)m + 1, 256), 256, 0, s>>>(
-        w_out->row_ptr, m, w_out->capacity, w_out->row_ptr, static_cast<WsHeader *>(ws));
-    count_launch(2);
+    count_launch(1);
     rc = check_launch("fused weight-gradient + prox kernels");
     if (rc) return rc;
     if (want_t) rc = transpose_from_bits_ext(w_out, kbits, wordpos, base + L.off_tr, L.total - L.off_tr, s);

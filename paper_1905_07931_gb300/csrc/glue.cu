@@ -64,14 +64,25 @@ __global__ void __launch_bounds__(256) softmax_xent_kernel(const float *__restri
     const int64_t col = (int64_t)blockIdx.x * 8 + cl;
     const bool ok = col < n;
     float m = -INFINITY, sum = 0.f;
+    constexpr int kBatch = 8;   // class values loaded together, then folded in order
     if (ok) {
-        for (int c = grp; c < classes; c += 32) {
-            const float x = __ldg(z + (int64_t)c * n + col);
-            if (x > m) {
-                sum = sum * expf(m - x) + 1.f;
-                m = x;
-            } else {
-                sum += expf(x - m);
+        for (int c0 = grp; c0 < classes; c0 += 32 * kBatch) {
+            float xs[kBatch];
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u) {
+                const int c = c0 + 32 * u;
+                xs[u] = c < classes ? __ldg(z + (int64_t)c * n + col) : -INFINITY;
+            }
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u) {
+                if (c0 + 32 * u >= classes) break;
+                const float x = xs[u];
+                if (x > m) {
+                    sum = sum * expf(m - x) + 1.f;
+                    m = x;
+                } else {
+                    sum += expf(x - m);
+                }
             }
         }
     }
@@ -90,9 +101,20 @@ __global__ void __launch_bounds__(256) softmax_xent_kernel(const float *__restri
     const float inv_n = 1.f / (float)n;
     const int lab = __ldg(labels + col);
     const bool lab_ok = lab >= 0 && lab < classes;   // an invalid label gives a NaN loss
-    for (int c = grp; c < classes; c += 32) {
-        const float p = expf(__ldg(z + (int64_t)c * n + col) - mx) * inv;
-        dz[(int64_t)c * n + col] = (p - (c == lab ? 1.f : 0.f)) * inv_n;
+    for (int c0 = grp; c0 < classes; c0 += 32 * kBatch) {
+        float xs[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            const int c = c0 + 32 * u;
+            xs[u] = c < classes ? __ldg(z + (int64_t)c * n + col) : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            const int c = c0 + 32 * u;
+            if (c >= classes) break;
+            const float p = expf(xs[u] - mx) * inv;
+            dz[(int64_t)c * n + col] = (p - (c == lab ? 1.f : 0.f)) * inv_n;
+        }
     }
     if (grp == 0)
         per_sample[col] = lab_ok ? -((__ldg(z + (int64_t)lab * n + col) - mx) - logf(se)) : __int_as_float(0x7fc00000);

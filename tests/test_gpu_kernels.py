@@ -655,3 +655,34 @@ def test_bounded_waits_give_up_and_report(C):
     assert_close(y.cpu().numpy(), O.spmm_fwd(ref, x), O.spmm_fwd(O.csr_abs(ref), np.abs(x)),
                  np.diff(ref.row_ptr)[:, None], what="spmm after the timed-out waits")
     assert ws.status()[0] == 0
+
+
+def test_fused_gradient_prox_capacity_overflow(C):
+    """An output CSR too small for the fused op's result: the overflow and the
+    needed nnz are reported, the row pointers are clamped, and the stored
+    prefix equals the unfused result's."""
+    m, k, n = 256, 512, 64
+    rng = np.random.default_rng(9)
+    a = _sparse(rng, m, k, 0.1) * F32(0.05)
+    dy = _dev((rng.standard_normal((m, n)) * 0.1).astype(F32))
+    x = _dev(rng.standard_normal((k, n)).astype(F32))
+    ws = _ws(C, m, k, n)
+    w_in = _gpu_csr(C, a, ws, transposed=False)
+    g = torch.zeros(m, k, device="cuda")
+    C.weight_grad_dense(dy, x, g, ws, precision=C.CSRT_PREC_TF32)
+    ref = C.CSR(m, k, transposed=False)
+    C.prox_update_compact(w_in, g, 0.5, 0.01, ref, ws)
+    (rp_ref, ci_ref, v_ref), _ = ref.to_host()
+    nnz = int(rp_ref[-1])
+    assert ws.status()[0] == 0
+    cap = nnz // 3
+    out = C.CSR(m, k, capacity=cap, transposed=False)
+    C.weight_grad_prox_update(w_in, dy, x, 0.5, 0.01, out, ws)
+    flags, required = ws.status()
+    assert flags & C.CSRT_DEV_CAPACITY and required == nnz
+    rp = out.row_ptr.cpu().numpy()
+    assert (np.diff(rp) >= 0).all() and rp[-1] == cap
+    np.testing.assert_array_equal(rp, np.minimum(rp_ref, cap))
+    np.testing.assert_array_equal(out.col_idx.cpu().numpy()[:cap], ci_ref[:cap])
+    np.testing.assert_array_equal(out.val.cpu().numpy()[:cap].view(np.uint32), v_ref[:cap].view(np.uint32))
+    ws.clear_status()
