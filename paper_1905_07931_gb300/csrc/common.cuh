@@ -21,8 +21,17 @@ struct WsHeader {
 };
 static_assert(sizeof(WsHeader) == 256, "workspace header is 256 bytes");
 constexpr size_t kWsHeaderBytes = 256;
+// After the header, counters of the SpMM carry protocol (a unit that finishes
+// a row shared with other units counts in; the last one completes the row).
+// Zeroed by csrt_workspace_init and left zero by every call; no call uses
+// them as scratch.
+constexpr size_t kWsCounterInts = 16384;
+constexpr size_t kWsReservedBytes = kWsHeaderBytes + kWsCounterInts * sizeof(int32_t);
 
-inline char *ws_scratch(void *ws) { return static_cast<char *>(ws) + kWsHeaderBytes; }
+inline char *ws_scratch(void *ws) { return static_cast<char *>(ws) + kWsReservedBytes; }
+inline int32_t *ws_counters(void *ws) {
+    return reinterpret_cast<int32_t *>(static_cast<char *>(ws) + kWsHeaderBytes);
+}
 
 // Bounded spin: a wait on another block's flag gives up after this many
 // polls (with nanosleep back-off it is far above any legitimate wait) and

@@ -847,7 +847,7 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
                           opt_aligned;
     const int32_t rows_per_tile = row_path ? imax<int32_t>(1, kRowBudget / cols) : 0;
     const int64_t tiles = row_path ? ceil_div<int64_t>(rows, rows_per_tile) : ceil_div<int64_t>(elems, kTile);
-    CSRT_ARG(ws_bytes >= kWsHeaderBytes + status_bytes(elems), "workspace too small for compaction");
+    CSRT_ARG(ws_bytes >= kWsReservedBytes + status_bytes(elems), "workspace too small for compaction");
     WsHeader *hdr = static_cast<WsHeader *>(ws);
     unsigned long long *status = reinterpret_cast<unsigned long long *>(ws_scratch(ws));
     CSRT_CHECK_CUDA(cudaMemsetAsync(&hdr->ticket, 0, sizeof(unsigned int), s));
@@ -898,7 +898,7 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
         }
         if (prox) {
             const bool bits = want_bits && cols % 32 == 0 &&
-                              ws_bytes >= kWsHeaderBytes + status_bytes(elems) + 2 * bits_bytes(rows, cols) +
+                              ws_bytes >= kWsReservedBytes + status_bytes(elems) + 2 * bits_bytes(rows, cols) +
                                               transpose_scratch_bytes(rows, cols);
             char *base = ws_scratch(ws);
             uint32_t *keepbits = reinterpret_cast<uint32_t *>(base + status_bytes(elems));
@@ -1285,7 +1285,7 @@ int transpose_impl(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s) {
         CSRT_CHECK_CUDA(cudaMemsetAsync(w->t_row_ptr, 0, sizeof(int32_t) * ((size_t)cols + 1), s));
         return CSRT_OK;
     }
-    CSRT_ARG(ws_bytes >= kWsHeaderBytes + transpose_scratch_bytes(rows, cols), "workspace too small for transpose");
+    CSRT_ARG(ws_bytes >= kWsReservedBytes + transpose_scratch_bytes(rows, cols), "workspace too small for transpose");
     const int nb = (int)ceil_div<int64_t>(rows, kTrRows);
     // Enough blocks to fill the GPU: split the columns into chunks of at least
     // 256 (and at most kTrChunk) so that nb * nc reaches ~4 blocks per SM.
@@ -1373,7 +1373,7 @@ int prox_update_compact(const csrt_csr *w_in, const float *g, float eta, float l
 }
 
 int csrt_check_bounded_waits(void *ws, size_t ws_bytes, void *stream) {
-    CSRT_ARG(ws != nullptr && ws_bytes >= kWsHeaderBytes + 2 * sizeof(unsigned long long), "workspace too small");
+    CSRT_ARG(ws != nullptr && ws_bytes >= kWsReservedBytes + 2 * sizeof(unsigned long long), "workspace too small");
     cudaStream_t s = as_stream(stream);
     unsigned long long *status = reinterpret_cast<unsigned long long *>(ws_scratch(ws));
     CSRT_CHECK_CUDA(cudaMemsetAsync(status, 0, 2 * sizeof(unsigned long long), s));

@@ -586,7 +586,7 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     const bool fused = precision == CSRT_PREC_TF32 && device_is_sm10x() && n > 0 && n % 4 == 0 && m >= 64 &&
                        k >= 64 && k % 32 == 0 && k <= kFpMaxK && dy && x &&
                        ((reinterpret_cast<uintptr_t>(dy) | reinterpret_cast<uintptr_t>(x)) & 15) == 0 &&
-                       ws_bytes >= kWsHeaderBytes + fused_prox_scratch_bytes(m, k);
+                       ws_bytes >= kWsReservedBytes + fused_prox_scratch_bytes(m, k);
     if (!fused) {
         CSRT_ARG(g_scratch != nullptr, "this shape/precision needs g_scratch (M x K floats) for the unfused path");
         int rc = weight_grad_dense(dy, x, m, k, n, g_scratch, precision, ws, ws_bytes, stream);

@@ -134,7 +134,7 @@ extern "C" int weight_grad_dense(const float *dy, const float *x, int32_t m, int
     const GemmSplit sp = gemm_split(m, k, n);
     float *out = g;
     if (sp.splits > 1) {
-        const size_t need = kWsHeaderBytes + (size_t)sp.splits * m * k * sizeof(float);
+        const size_t need = kWsReservedBytes + (size_t)sp.splits * m * k * sizeof(float);
         CSRT_ARG(ws != nullptr && ws_bytes >= need, "workspace too small for split gemm (%zu < %zu)", ws_bytes, need);
         out = reinterpret_cast<float *>(ws_scratch(ws));
     }

@@ -61,7 +61,7 @@ int csrt_workspace_bytes(int32_t rows, int32_t cols, int32_t max_n, size_t *byte
     if (t > need) need = t;
     t = fused_prox_scratch_bytes(rows, cols);
     if (t > need) need = t;
-    *bytes = kWsHeaderBytes + ((need + 255) / 256) * 256;
+    *bytes = kWsReservedBytes + ((need + 255) / 256) * 256;
     return CSRT_OK;
 }
 

@@ -68,6 +68,7 @@ struct SpmmArgs {
     int32_t n_tiles;
     float *carry;     // [n_tiles][units][TN]
     int32_t *carry_row;  // [units]
+    int32_t *cnt;     // [n_tiles][units] counters of the shared rows (zero between calls), or null: fix-up kernel
     // optional epilogue on each finished row i: + bias[i], then ReLU, then
     // zero where mask[i, c] <= 0 (the ReLU backward of the layer below)
     const float *bias;
@@ -152,8 +153,49 @@ __device__ __forceinline__ void spmm_consume(const SpmmArgs &a, int64_t k, int64
     }
 }
 
+// Row r, cut between units ua..ub of the merge path (its first nonzero lies
+// in unit ua, its end in unit ub): every one of them counts in after writing
+// its part (ub the partial row in Y, the others their carries); the last to
+// arrive adds the carries in unit order to the partial row, applies the
+// epilogue and resets the counter. The sum is the fix-up kernel's, in the
+// same order; no unit waits for another.
 template <int VW, int NV>
-__global__ void __launch_bounds__(kSpThreads) spmm_merge_kernel(SpmmArgs a) {
+__device__ __forceinline__ void spmm_complete_shared_row(const SpmmArgs &a, int r, int64_t per, int t, int n0) {
+    constexpr int TN = 32 * VW * NV;
+    constexpr int kStride = 32 * VW;
+    const int lane = threadIdx.x & 31;
+    const int64_t d0 = (int64_t)__ldg(a.row_ptr + r) + r, d1 = (int64_t)__ldg(a.row_ptr + r + 1) + r;
+    const int ua = (int)(d0 / per), ub = (int)(d1 / per);
+    __threadfence();   // this unit's part is visible before it counts in
+    __syncwarp();
+    int last = 0;
+    if (lane == 0) last = atomicAdd(a.cnt + (int64_t)t * a.units + ua, 1) == ub - ua;
+    if (!__shfl_sync(0xffffffffu, last, 0)) return;
+    __threadfence();   // the others' parts are visible to the last one
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+        const int c = n0 + v * kStride;
+        if (c >= a.n) continue;
+        float sum[VW];
+#pragma unroll
+        for (int e = 0; e < VW; ++e) sum[e] = 0.f;
+        for (int w = ua; w < ub; ++w) {
+            const float *cp = a.carry + ((int64_t)t * a.units + w) * TN + lane * VW + v * kStride;
+#pragma unroll
+            for (int e = 0; e < VW; ++e) sum[e] += __ldcg(cp + e);
+        }
+        float *yp = a.y + (int64_t)r * a.n + c;
+        float out[VW];
+#pragma unroll
+        for (int e = 0; e < VW; ++e) out[e] = __ldcg(yp + e) + sum[e];
+        if (a.bias || a.relu || a.mask) spmm_epilogue<VW>(a, r, c, out);
+        stv<VW>(yp, out);
+    }
+    if (lane == 0) a.cnt[(int64_t)t * a.units + ua] = 0;
+}
+
+template <int VW, int NV>
+__global__ void __launch_bounds__(kSpThreads, 3) spmm_merge_kernel(SpmmArgs a) {
     constexpr int TN = 32 * VW * NV;
     constexpr int kStride = 32 * VW;
     const int lane = threadIdx.x & 31;
@@ -204,6 +246,15 @@ __global__ void __launch_bounds__(kSpThreads) spmm_merge_kernel(SpmmArgs a) {
             float *cp = a.carry + ((int64_t)t * a.units + u) * TN + lane * VW;
 #pragma unroll
             for (int v = 0; v < NV; ++v) stv<VW>(cp + v * kStride, acc[v]);
+        }
+        if (a.cnt) {
+            // the rows this unit shares with others: the first (begun in an
+            // earlier unit) and the last (going on in a later one); one row
+            // when the unit lies inside a single row
+            const int ra = first_row_cut ? i0 : -1;
+            const int rb = (has_carry && i1 != ra) ? i1 : -1;
+            if (ra >= 0) spmm_complete_shared_row<VW, NV>(a, ra, per, t, n0);
+            if (rb >= 0) spmm_complete_shared_row<VW, NV>(a, rb, per, t, n0);
         }
     }
 }
@@ -311,10 +362,14 @@ static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *
     const size_t carry_floats = (size_t)sh.units * sh.n_tiles * sh.tn;
     a.carry = reinterpret_cast<float *>(ws_scratch(ws));
     a.carry_row = reinterpret_cast<int32_t *>(a.carry + ((carry_floats + 63) / 64) * 64);
+    a.cnt = nullptr;
     if (sh.units > 1) {
-        const size_t need = kWsHeaderBytes + ((carry_floats + 63) / 64) * 64 * sizeof(float) +
+        const size_t need = kWsReservedBytes + ((carry_floats + 63) / 64) * 64 * sizeof(float) +
                             (size_t)sh.units * sizeof(int32_t);
         CSRT_ARG(ws != nullptr && ws_bytes >= need, "workspace too small for spmm (%zu < %zu)", ws_bytes, need);
+        // rows shared by units are completed in the kernel by the last unit to
+        // finish its part; more units than counters fall back to the fix-up kernel
+        if ((int64_t)sh.units * sh.n_tiles <= (int64_t)kWsCounterInts) a.cnt = ws_counters(ws);
     }
     const int64_t threads = (int64_t)sh.units * sh.n_tiles * 32;
     const unsigned grid = (unsigned)ceil_div<int64_t>(threads, kSpThreads);
@@ -322,7 +377,7 @@ static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *
     if (sh.vw == VW && sh.nv == NV) {                                                        \
         spmm_merge_kernel<VW, NV><<<grid, kSpThreads, 0, s>>>(a);                            \
         count_launch();                                                                      \
-        if (sh.units > 1) {                                                                  \
+        if (sh.units > 1 && a.cnt == nullptr) {                                              \
             const int64_t ft = (int64_t)sh.units * sh.n_tiles * 32;                            \
             spmm_fixup_kernel<32 * VW * NV><<<(unsigned)ceil_div<int64_t>(ft, 256), 256, 0, s>>>(a); \
             count_launch();                                                                  \
@@ -524,7 +579,7 @@ int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_
     const int64_t target = (int64_t)num_sms() * kWarpsPerSM;
     a.units = (int)imax<int64_t>(1, imin<int64_t>(ceil_div<int64_t>(target, chunks), w->capacity));
     if (chunks > 1) {
-        CSRT_ARG(ws != nullptr && ws_bytes >= kWsHeaderBytes + sddmm_scratch_bytes(w->capacity, n),
+        CSRT_ARG(ws != nullptr && ws_bytes >= kWsReservedBytes + sddmm_scratch_bytes(w->capacity, n),
                  "workspace too small for sddmm");
         a.out = reinterpret_cast<float *>(ws_scratch(ws));
         a.out_stride = w->capacity;
@@ -645,6 +700,7 @@ extern "C" int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, fl
     a.n_tiles = sh.n_tiles;
     a.carry = g_noalloc_carry_addr[dev];
     a.carry_row = g_noalloc_row_addr[dev];
+    a.cnt = nullptr;   // shared rows are completed by the fix-up kernel
     a.bias = nullptr;
     a.relu = 0;
     a.mask = nullptr;
