@@ -28,8 +28,11 @@
  *  - Workspace. Calls that take `ws` need a device scratch buffer of at least
  *    csrt_workspace_bytes(...) bytes, initialised once with
  *    csrt_workspace_init. Its first 256 bytes hold a device status word that
- *    accumulates data-dependent errors (see CSRT_DEV_*). A workspace serves
- *    one stream at a time: calls on two streams need two workspaces.
+ *    accumulates data-dependent errors (see CSRT_DEV_*); the next 64 KiB hold
+ *    counters that the sparse products use and leave at zero (so the
+ *    workspace must start zeroed, as csrt_workspace_init leaves it). A
+ *    workspace serves one stream at a time: calls on two streams need two
+ *    workspaces.
  *  - Errors. Each call returns CSRT_OK or a CSRT_ERR_* code at once for bad
  *    arguments or a failed launch; no work is enqueued in that case.
  *    Data-dependent errors (capacity overflow, a bounded wait that ran out,
