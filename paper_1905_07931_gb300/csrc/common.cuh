@@ -65,6 +65,33 @@ int num_sms();   // SMs of the current device (cached per device)
 
 inline cudaStream_t as_stream(void *s) { return static_cast<cudaStream_t>(s); }
 
+// Programmatic dependent launch. A kernel launched with launch_pdl may be
+// scheduled while the kernel before it on the stream is finishing (its last
+// blocks exiting and its writes being flushed), which hides the launch
+// latency between consecutive kernels of a step. Every kernel therefore
+// starts with pdl_enter(): griddepcontrol.wait returns once the previous
+// kernel has completed and its writes are visible. Launched without the
+// attribute, the instruction does nothing. (An explicit early
+// launch_dependents, which would let the next kernel's blocks wait on the
+// SMs during this kernel's last wave, measured slower on the training step.)
+__device__ __forceinline__ void pdl_enter() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... P, typename... A>
+inline cudaError_t launch_pdl(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              A &&...args) {
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<P>(args)...);
+}
+
 // ---------------------------------------------------------------------------
 // Workspace sizes of the individual operations (bytes after the header).
 // ---------------------------------------------------------------------------

@@ -175,6 +175,7 @@ __device__ __forceinline__ unsigned long long lookback_warp(unsigned long long *
 
 template <bool kProx, bool kVec>
 __global__ void __launch_bounds__(kCThreads) compact_kernel(CompactArgs a) {
+    pdl_enter();
     __shared__ __align__(16) float w_tile[kProx ? kTile : 4];
     __shared__ int32_t s_rowptr[kProx ? kTile + 2 : 2];
     __shared__ unsigned long long s_warp[kCThreads / 32];
@@ -436,6 +437,7 @@ __device__ __forceinline__ Keep4 eval4(const float4 g, const float4 w, float eta
 
 template <bool kProx>
 __global__ void __launch_bounds__(kCThreads, 4) compact_rows_kernel(CompactArgs a, int32_t rows_per_tile) {
+    pdl_enter();
     extern __shared__ __align__(16) float row_smem[];
     float *wt = row_smem;                                                        // old weights (prox)
     int32_t *s_rp = reinterpret_cast<int32_t *>(row_smem + (kProx ? rows_per_tile * a.cols : 0));
@@ -591,6 +593,7 @@ template <bool kBits>
 __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, int32_t rows_per_tile,
                                                                   uint32_t *__restrict__ keepbits,
                                                                   int32_t *__restrict__ wordpos, int32_t wpr) {
+    pdl_enter();
     // shared: the tile's G (bulk-copied), then z in place, then the kept values
     // (NaN = dropped); a bitmask of the positions that hold a stored weight;
     // the tile's row pointers.
@@ -805,6 +808,7 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
 // on. Each gives up after its iteration limit, sets CSRT_DEV_TIMEOUT (with
 // the site of the wait) and the kernel returns normally.
 __global__ void bounded_wait_check_kernel(unsigned long long *__restrict__ status, WsHeader *hdr, int which) {
+    pdl_enter();
     __shared__ __align__(8) uint64_t bar;
     if (which == 0) {
         lookback_warp(status, 1, 0u, hdr);   // status[0] is zero and stays zero
@@ -904,14 +908,14 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
             uint32_t *keepbits = reinterpret_cast<uint32_t *>(base + status_bytes(elems));
             int32_t *wordpos = reinterpret_cast<int32_t *>(base + status_bytes(elems) + bits_bytes(rows, cols));
             if (bits)
-                prox_rows_kernel<true><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile, keepbits, wordpos,
-                                                                                 cols / 32);
+                launch_pdl(prox_rows_kernel<true>, dim3((unsigned)tiles), dim3(kCThreads), smem, s, a,
+                           rows_per_tile, keepbits, wordpos, cols / 32);
             else
-                prox_rows_kernel<false><<<(unsigned)tiles, kCThreads, smem, s>>>(a, rows_per_tile, nullptr, nullptr,
-                                                                                  0);
+                launch_pdl(prox_rows_kernel<false>, dim3((unsigned)tiles), dim3(kCThreads), smem, s, a,
+                           rows_per_tile, nullptr, nullptr, 0);
             if (bits_done) *bits_done = bits;
         } else {
-            compact_rows_kernel<false><<<(unsigned)tiles, kCThreads, 0, s>>>(a, rows_per_tile);
+            launch_pdl(compact_rows_kernel<false>, dim3((unsigned)tiles), dim3(kCThreads), 0, s, a, rows_per_tile);
         }
         count_launch();
         return check_launch("row-tile compaction kernel");
@@ -919,11 +923,11 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
     const bool vec = (reinterpret_cast<uintptr_t>(src) & 15) == 0;
     dim3 grid((unsigned)tiles), block(kCThreads);
     if (prox) {
-        if (vec) compact_kernel<true, true><<<grid, block, 0, s>>>(a);
-        else compact_kernel<true, false><<<grid, block, 0, s>>>(a);
+        if (vec) launch_pdl(compact_kernel<true, true>, dim3(grid), dim3(block), 0, s, a);
+        else launch_pdl(compact_kernel<true, false>, dim3(grid), dim3(block), 0, s, a);
     } else {
-        if (vec) compact_kernel<false, true><<<grid, block, 0, s>>>(a);
-        else compact_kernel<false, false><<<grid, block, 0, s>>>(a);
+        if (vec) launch_pdl(compact_kernel<false, true>, dim3(grid), dim3(block), 0, s, a);
+        else launch_pdl(compact_kernel<false, false>, dim3(grid), dim3(block), 0, s, a);
     }
     count_launch();
     return check_launch("compact_kernel");
@@ -963,6 +967,7 @@ __device__ __forceinline__ void tr_build_bits(unsigned int *bits, const int32_t 
 __global__ void __launch_bounds__(256) tr_count_kernel(const int32_t *__restrict__ row_ptr,
                                                        const int32_t *__restrict__ col, int32_t rows,
                                                        int32_t cols, int32_t chunk, int32_t *__restrict__ cnt) {
+    pdl_enter();
     __shared__ unsigned int bits[kTrChunk];
     const int b = blockIdx.x, c0 = blockIdx.y * chunk;
     const int cw = min(chunk, cols - c0);
@@ -974,6 +979,7 @@ __global__ void __launch_bounds__(256) tr_count_kernel(const int32_t *__restrict
 // Exclusive scan of cnt[b][j] over b for 32 columns per block; column totals.
 __global__ void __launch_bounds__(256) tr_colscan_kernel(int32_t *__restrict__ cnt, int32_t nb,
                                                          int32_t cols, int32_t *__restrict__ coltot) {
+    pdl_enter();
     __shared__ int32_t seg[8][32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int j = blockIdx.x * 32 + lane;
@@ -999,6 +1005,7 @@ __global__ void __launch_bounds__(256) tr_colscan_kernel(int32_t *__restrict__ c
 // Exclusive scan of n values into out[0..n] (out[n] = total); one block.
 __global__ void __launch_bounds__(1024) scan_single_block_kernel(const int32_t *__restrict__ in, int32_t n,
                                                                  int32_t *__restrict__ out) {
+    pdl_enter();
     __shared__ int32_t s_warp[32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int per = (n + 1023) / 1024;
@@ -1033,6 +1040,7 @@ __global__ void __launch_bounds__(1024) scan_clamped_kernel(const int32_t *__res
                                                             int32_t *__restrict__ out,
                                                             int32_t *__restrict__ out_clamped, int64_t capacity,
                                                             WsHeader *hdr) {
+    pdl_enter();
     __shared__ int32_t s_warp[32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int per = (n + 1023) / 1024;
@@ -1069,7 +1077,8 @@ __global__ void __launch_bounds__(1024) scan_clamped_kernel(const int32_t *__res
 
 int scan_exclusive_i32_clamped(const int32_t *in, int32_t n, int32_t *out, int32_t *out_clamped, int64_t capacity,
                                void *ws, cudaStream_t s) {
-    scan_clamped_kernel<<<1, 1024, 0, s>>>(in, n, out, out_clamped, capacity, static_cast<WsHeader *>(ws));
+    launch_pdl(scan_clamped_kernel, dim3(1), dim3(1024), 0, s, in, n, out, out_clamped, capacity,
+               static_cast<WsHeader *>(ws));
     count_launch();
     return check_launch("scan_clamped_kernel");
 }
@@ -1088,6 +1097,7 @@ __global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict
                                                        const int32_t *__restrict__ t_row_ptr,
                                                        int32_t *__restrict__ t_col, float *__restrict__ t_val,
                                                        int32_t *__restrict__ t_pos, int64_t capacity) {
+    pdl_enter();
     __shared__ unsigned int bits[kTwCols];
     __shared__ int32_t base[kTwCols];            // first position of this block's run in each column
     __shared__ float vt[kTrRows][kTwCols + 1];   // values of the block's entries, padded
@@ -1178,6 +1188,7 @@ __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
 
 __global__ void __launch_bounds__(256) trb_count_kernel(const uint32_t *__restrict__ keepbits, int32_t rows,
                                                         int32_t wpr, int32_t cols, int32_t *__restrict__ cnt) {
+    pdl_enter();
     const int lane = threadIdx.x & 31;
     const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nb = ceil_div<int64_t>(rows, 32);
@@ -1196,6 +1207,7 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
                                                         const float *__restrict__ val, int32_t *__restrict__ t_col,
                                                         float *__restrict__ t_val, int32_t *__restrict__ t_pos,
                                                         int64_t capacity) {
+    pdl_enter();
     __shared__ float tile[8][32 * 32];   // element (r, j) at r*32 + (j ^ r): rows and columns conflict-free
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -1250,11 +1262,11 @@ int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t
     int32_t *coltot = cnt + (int64_t)nb * cols;
     const int64_t warps = (int64_t)nb * wpr;
     const unsigned grid = (unsigned)ceil_div<int64_t>(warps * 32, 256);
-    trb_count_kernel<<<grid, 256, 0, s>>>(keepbits, rows, wpr, cols, cnt);
-    tr_colscan_kernel<<<ceil_div(cols, 32), 256, 0, s>>>(cnt, nb, cols, coltot);
-    scan_single_block_kernel<<<1, 1024, 0, s>>>(coltot, cols, w->t_row_ptr);
-    trb_write_kernel<<<grid, 256, 0, s>>>(keepbits, wordpos, rows, wpr, cols, cnt, w->t_row_ptr, w->val,
-                                          w->t_col_idx, w->t_val, w->t_pos, w->capacity);
+    launch_pdl(trb_count_kernel, dim3(grid), dim3(256), 0, s, keepbits, rows, wpr, cols, cnt);
+    launch_pdl(tr_colscan_kernel, dim3(ceil_div(cols, 32)), dim3(256), 0, s, cnt, nb, cols, coltot);
+    launch_pdl(scan_single_block_kernel, dim3(1), dim3(1024), 0, s, coltot, cols, w->t_row_ptr);
+    launch_pdl(trb_write_kernel, dim3(grid), dim3(256), 0, s, keepbits, wordpos, rows, wpr, cols, cnt, w->t_row_ptr,
+               w->val, w->t_col_idx, w->t_val, w->t_pos, w->capacity);
     count_launch(4);
     return check_launch("transpose-from-bits kernels");
 }
@@ -1272,7 +1284,7 @@ static int transpose_from_bits(csrt_csr *w, void *ws, size_t ws_bytes, cudaStrea
 
 // Exclusive scan of n int32 values into out[0..n] (out[n] = total), one block.
 int scan_exclusive_i32(const int32_t *in, int32_t n, int32_t *out, cudaStream_t s) {
-    scan_single_block_kernel<<<1, 1024, 0, s>>>(in, n, out);
+    launch_pdl(scan_single_block_kernel, dim3(1), dim3(1024), 0, s, in, n, out);
     count_launch();
     return check_launch("scan_single_block_kernel");
 }
@@ -1295,10 +1307,10 @@ int transpose_impl(csrt_csr *w, void *ws, size_t ws_bytes, cudaStream_t s) {
     nc = (int)ceil_div<int64_t>(cols, chunk);
     int32_t *cnt = reinterpret_cast<int32_t *>(ws_scratch(ws));
     int32_t *coltot = cnt + (int64_t)nb * cols;
-    tr_count_kernel<<<dim3(nb, nc), 256, 0, s>>>(w->row_ptr, w->col_idx, rows, cols, chunk, cnt);
-    tr_colscan_kernel<<<ceil_div(cols, 32), 256, 0, s>>>(cnt, nb, cols, coltot);
-    scan_single_block_kernel<<<1, 1024, 0, s>>>(coltot, cols, w->t_row_ptr);
-    tr_write_kernel<<<dim3(nb, (unsigned)ceil_div<int64_t>(cols, kTwCols)), 256, 0, s>>>(
+    launch_pdl(tr_count_kernel, dim3(dim3(nb, nc)), dim3(256), 0, s, w->row_ptr, w->col_idx, rows, cols, chunk, cnt);
+    launch_pdl(tr_colscan_kernel, dim3(ceil_div(cols, 32)), dim3(256), 0, s, cnt, nb, cols, coltot);
+    launch_pdl(scan_single_block_kernel, dim3(1), dim3(1024), 0, s, coltot, cols, w->t_row_ptr);
+    launch_pdl(tr_write_kernel, dim3(dim3(nb, (unsigned)ceil_div<int64_t>(cols, kTwCols))), dim3(256), 0, s,
         w->row_ptr, w->col_idx, w->val, rows, cols, cnt, w->t_row_ptr, w->t_col_idx, w->t_val, w->t_pos,
         w->capacity);
     count_launch(4);
@@ -1377,8 +1389,8 @@ int csrt_check_bounded_waits(void *ws, size_t ws_bytes, void *stream) {
     cudaStream_t s = as_stream(stream);
     unsigned long long *status = reinterpret_cast<unsigned long long *>(ws_scratch(ws));
     CSRT_CHECK_CUDA(cudaMemsetAsync(status, 0, 2 * sizeof(unsigned long long), s));
-    bounded_wait_check_kernel<<<1, 32, 0, s>>>(status, static_cast<WsHeader *>(ws), 0);
-    bounded_wait_check_kernel<<<1, 32, 0, s>>>(status, static_cast<WsHeader *>(ws), 1);
+    launch_pdl(bounded_wait_check_kernel, dim3(1), dim3(32), 0, s, status, static_cast<WsHeader *>(ws), 0);
+    launch_pdl(bounded_wait_check_kernel, dim3(1), dim3(32), 0, s, status, static_cast<WsHeader *>(ws), 1);
     count_launch(2);
     return check_launch("bounded_wait_check_kernel");
 }

@@ -28,6 +28,7 @@ __global__ void __launch_bounds__(kConvThreads) conv_sparse_fwd_kernel(
     const int32_t *__restrict__ row_ptr, const int32_t *__restrict__ col, const float *__restrict__ val,
     const float *__restrict__ x, int32_t cin, int32_t b, int32_t h, int32_t w, int32_t k,
     const float *__restrict__ bias, int32_t relu, float *__restrict__ y) {
+    pdl_enter();
     __shared__ float s_w[kConvTaps];
     __shared__ int64_t s_off[kConvTaps];
     const int ho = h - k + 1, wo = w - k + 1;
@@ -99,8 +100,8 @@ extern "C" int csrt_conv2d_sparse_fwd(const csrt_csr *w, const float *x, int32_t
     CSRT_ARG(w->capacity == 0 || (w->col_idx && w->val), "col_idx/val NULL");
     const int64_t blocks = ceil_div<int64_t>(npix, (int64_t)kConvThreads * kConvPer);
     CSRT_ARG(blocks < ((int64_t)1 << 31), "too many output pixels");
-    conv_sparse_fwd_kernel<<<dim3((unsigned)blocks, (unsigned)w->rows), kConvThreads, 0, as_stream(stream)>>>(
-        w->row_ptr, w->col_idx, w->val, x, c, b, h, wd, k, bias, relu, y);
+    launch_pdl(conv_sparse_fwd_kernel, dim3((unsigned)blocks, (unsigned)w->rows), dim3(kConvThreads), 0,
+               as_stream(stream), w->row_ptr, w->col_idx, w->val, x, c, b, h, wd, k, bias, relu, y);
     count_launch();
     return check_launch("conv_sparse_fwd_kernel");
 }

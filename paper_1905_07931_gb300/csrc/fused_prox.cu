@@ -126,6 +126,7 @@ __global__ void __launch_bounds__(256) fp_oldbits_kernel(const int32_t *__restri
                                                          const int32_t *__restrict__ col, int32_t m, int32_t wpr,
                                                          int32_t nt, uint32_t *__restrict__ obits,
                                                          int32_t *__restrict__ ostart) {
+    pdl_enter();
     __shared__ uint32_t sw[8][kFpMaxK / 32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t r = (int64_t)blockIdx.x * 8 + warp;
@@ -273,6 +274,7 @@ template <bool kWrite>
 __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
     gemm_prox_tc_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                         FpArgs a, int32_t tiles_n, int32_t num_tiles) {
+    pdl_enter();
     constexpr int kEpi = FpShape<kWrite>::kEpi, kStages = FpShape<kWrite>::kStages;
     constexpr int kFpPre = FpShape<kWrite>::kPre, kGroup = FpShape<kWrite>::kGroup;
     constexpr int kSpanCols = kTcBN / (kEpi / 4);   // columns per epilogue warp
@@ -538,6 +540,7 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
 // 3. Per row: exclusive offsets of the segments (in place) and the row total.
 __global__ void __launch_bounds__(256) fp_rowscan_kernel(int32_t *__restrict__ counts, int32_t m, int32_t nt,
                                                          int32_t *__restrict__ rowtot) {
+    pdl_enter();
     const int lane = threadIdx.x & 31;
     const int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     if (r >= m) return;
@@ -616,8 +619,8 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
                                              fp_smem_bytes<true>()));
         attr_set[dev] = true;
     }
-    fp_oldbits_kernel<<<(unsigned)ceil_div<int64_t>(m, 8), 256, 0, s>>>(w_in->row_ptr, w_in->col_idx, m, L.wpr, L.nt,
-                                                                        obits, ostart);
+    launch_pdl(fp_oldbits_kernel, dim3((unsigned)ceil_div<int64_t>(m, 8)), dim3(256), 0, s, w_in->row_ptr,
+               w_in->col_idx, m, L.wpr, L.nt, obits, ostart);
     FpArgs a;
     a.m = m;
     a.k = k;
@@ -640,14 +643,17 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     const int tiles_m = (int)ceil_div<int64_t>(m, kTcBM), tiles_n = (int)ceil_div<int64_t>(k, kTcBN);
     const int tiles = tiles_m * tiles_n;
     const unsigned grid = (unsigned)imin(tiles, num_sms());
-    gemm_prox_tc_kernel<false><<<grid, fp_threads<false>(), fp_smem_bytes<false>(), s>>>(ma, mb, a, tiles_n, tiles);
-    fp_rowscan_kernel<<<(unsigned)ceil_div<int64_t>((int64_t)m * 32, 256), 256, 0, s>>>(counts, m, L.nt, rowtot);
+    launch_pdl(gemm_prox_tc_kernel<false>, dim3(grid), dim3(fp_threads<false>()), fp_smem_bytes<false>(), s, ma, mb, a,
+               tiles_n, tiles);
+    launch_pdl(fp_rowscan_kernel, dim3((unsigned)ceil_div<int64_t>((int64_t)m * 32, 256)), dim3(256), 0, s, counts, m,
+               L.nt, rowtot);
     count_launch(3);
     // new row pointers: exclusive scan of the row totals (int32: nnz <= M*K < 2^31), unclamped for the write
     // pass and clamped to the capacity in w_out (overflow reported)
     int rc = scan_exclusive_i32_clamped(rowtot, m, rawptr, w_out->row_ptr, w_out->capacity, ws, s);
     if (rc) return rc;
-    gemm_prox_tc_kernel<true><<<grid, fp_threads<true>(), fp_smem_bytes<true>(), s>>>(ma, mb, a, tiles_n, tiles);
+    launch_pdl(gemm_prox_tc_kernel<true>, dim3(grid), dim3(fp_threads<true>()), fp_smem_bytes<true>(), s, ma, mb, a,
+               tiles_n, tiles);
     count_launch(1);
     rc = check_launch("fused weight-gradient + prox kernels");
     if (rc) return rc;

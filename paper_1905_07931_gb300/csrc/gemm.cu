@@ -50,6 +50,7 @@ size_t gemm_scratch_bytes(int32_t m, int32_t k, int32_t max_n) {
 __global__ void __launch_bounds__(256) gemm_nt_f32_kernel(const float *__restrict__ dy, const float *__restrict__ x,
                                                           int32_t m, int32_t k, int32_t n, int32_t chunk,
                                                           float *__restrict__ out) {
+    pdl_enter();
     __shared__ float as[kGBK][kGBM + 4];
     __shared__ float bs[kGBK][kGBN + 4];
     const int tid = threadIdx.x;
@@ -98,6 +99,7 @@ __global__ void __launch_bounds__(256) gemm_nt_f32_kernel(const float *__restric
 
 __global__ void split_reduce_kernel(const float *__restrict__ part, int64_t count, int32_t splits,
                                     float *__restrict__ out) {
+    pdl_enter();
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < count; e += (int64_t)gridDim.x * blockDim.x) {
         float s = 0.f;
         for (int p = 0; p < splits; ++p) s += part[(int64_t)p * count + e];
@@ -139,12 +141,12 @@ extern "C" int weight_grad_dense(const float *dy, const float *x, int32_t m, int
         out = reinterpret_cast<float *>(ws_scratch(ws));
     }
     dim3 grid((unsigned)ceil_div<int64_t>(k, kGBN), (unsigned)ceil_div<int64_t>(m, kGBM), (unsigned)sp.splits);
-    gemm_nt_f32_kernel<<<grid, 256, 0, s>>>(dy, x, m, k, n, sp.chunk, out);
+    launch_pdl(gemm_nt_f32_kernel, dim3(grid), dim3(256), 0, s, dy, x, m, k, n, sp.chunk, out);
     count_launch();
     if (sp.splits > 1) {
         const int64_t count = (int64_t)m * k;
         const unsigned rg = (unsigned)imin<int64_t>(ceil_div<int64_t>(count, 256), (int64_t)num_sms() * 8);
-        split_reduce_kernel<<<rg, 256, 0, s>>>(out, count, sp.splits, g);
+        launch_pdl(split_reduce_kernel, dim3(rg), dim3(256), 0, s, out, count, sp.splits, g);
         count_launch();
     }
     return check_launch("gemm_nt_f32_kernel");

@@ -33,6 +33,7 @@ struct TcArgs {
 __global__ void __launch_bounds__(kTcThreads, 1)
     gemm_tf32_tc_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                         TcArgs a) {
+    pdl_enter();
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sa = smem;
@@ -167,6 +168,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     gemm_tf32_tc_persistent_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                                    const __grid_constant__ CUtensorMap map_g, TcArgs a, int32_t tiles_n,
                                    int32_t num_tiles) {
+    pdl_enter();
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sa = smem;
@@ -330,13 +332,14 @@ int gemm_tc_tf32(const float *dy, const float *x, int32_t m, int32_t k, int32_t 
     if (tma_out) {
         const int tiles = tiles_m * tiles_n;
         const int grid = imin(tiles, num_sms());
-        gemm_tf32_tc_persistent_kernel<<<grid, kTcThreads, kPSmemBytes, s>>>(ma, mb, mg, a, tiles_n, tiles);
+        launch_pdl(gemm_tf32_tc_persistent_kernel, dim3(grid), dim3(kTcThreads), kPSmemBytes, s, ma, mb, mg, a,
+                   tiles_n, tiles);
         count_launch();
         *handled = true;
         return check_launch("gemm_tf32_tc_persistent_kernel");
     }
     dim3 grid((unsigned)tiles_n, (unsigned)tiles_m);
-    gemm_tf32_tc_kernel<<<grid, kTcThreads, kTcSmemBytes, s>>>(ma, mb, a);
+    launch_pdl(gemm_tf32_tc_kernel, dim3(grid), dim3(kTcThreads), kTcSmemBytes, s, ma, mb, a);
     count_launch();
     *handled = true;
     return check_launch("gemm_tf32_tc_kernel");

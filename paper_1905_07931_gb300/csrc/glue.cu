@@ -17,6 +17,7 @@ static unsigned grid_for(int64_t count, int threads = 256) {
 
 __global__ void bias_act_kernel(float *__restrict__ y, const float *__restrict__ bias, int32_t m, int32_t n,
                                 int relu) {
+    pdl_enter();
     const int64_t total = (int64_t)m * n;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
         float v = y[e];
@@ -27,6 +28,7 @@ __global__ void bias_act_kernel(float *__restrict__ y, const float *__restrict__
 }
 
 __global__ void relu_bwd_kernel(float *__restrict__ dy, const float *__restrict__ y, int64_t count) {
+    pdl_enter();
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < count; e += (int64_t)gridDim.x * blockDim.x)
         if (!(__ldg(y + e) > 0.f)) dy[e] = 0.f;
 }
@@ -34,6 +36,7 @@ __global__ void relu_bwd_kernel(float *__restrict__ dy, const float *__restrict_
 // One warp per row: gb[i] = sum_c dy[i, c] in a fixed order; SGD on the bias.
 __global__ void bias_grad_sgd_kernel(const float *__restrict__ dy, int32_t m, int32_t n, float *__restrict__ bias,
                                      float eta, float *__restrict__ gb_out) {
+    pdl_enter();
     const int lane = threadIdx.x & 31;
     const int64_t row = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     if (row >= m) return;
@@ -57,6 +60,7 @@ __global__ void __launch_bounds__(256) softmax_xent_kernel(const float *__restri
                                                            const int32_t *__restrict__ labels, int32_t classes,
                                                            int32_t n, float *__restrict__ dz,
                                                            float *__restrict__ per_sample) {
+    pdl_enter();
     __shared__ float s_m[32][8], s_s[32][8];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int cl = lane & 7;
@@ -122,6 +126,7 @@ __global__ void __launch_bounds__(256) softmax_xent_kernel(const float *__restri
 
 // Mean of the per-sample losses in a fixed order (one block).
 __global__ void __launch_bounds__(1024) mean_kernel(const float *__restrict__ v, int32_t n, float *__restrict__ out) {
+    pdl_enter();
     __shared__ float s_warp[32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     float s = 0.f;
@@ -140,6 +145,7 @@ __global__ void __launch_bounds__(1024) mean_kernel(const float *__restrict__ v,
 
 __global__ void im2col_kernel(const float *__restrict__ x, int32_t c, int32_t b, int32_t h, int32_t w, int32_t k,
                               float *__restrict__ cols) {
+    pdl_enter();
     const int ho = h - k + 1, wo = w - k + 1;
     const int64_t ncol = (int64_t)b * ho * wo;
     const int64_t total = (int64_t)c * k * k * ncol;
@@ -156,6 +162,7 @@ __global__ void im2col_kernel(const float *__restrict__ x, int32_t c, int32_t b,
 
 __global__ void col2im_kernel(const float *__restrict__ dcols, int32_t c, int32_t b, int32_t h, int32_t w,
                               int32_t k, float *__restrict__ dx) {
+    pdl_enter();
     const int ho = h - k + 1, wo = w - k + 1;
     const int64_t ncol = (int64_t)b * ho * wo;
     const int64_t total = (int64_t)c * b * h * w;
@@ -180,6 +187,7 @@ __global__ void col2im_kernel(const float *__restrict__ dcols, int32_t c, int32_
 
 __global__ void maxpool2_fwd_kernel(const float *__restrict__ x, int32_t c, int32_t b, int32_t h, int32_t w,
                                     float *__restrict__ y, int8_t *__restrict__ idx) {
+    pdl_enter();
     const int ho = h / 2, wo = w / 2;
     const int64_t total = (int64_t)c * b * ho * wo;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
@@ -198,6 +206,7 @@ __global__ void maxpool2_fwd_kernel(const float *__restrict__ x, int32_t c, int3
 
 __global__ void maxpool2_bwd_kernel(const float *__restrict__ dy, const int8_t *__restrict__ idx, int32_t c,
                                     int32_t b, int32_t h, int32_t w, float *__restrict__ dx) {
+    pdl_enter();
     const int ho = h / 2, wo = w / 2;
     const int64_t total = (int64_t)c * b * h * w;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
@@ -213,6 +222,7 @@ __global__ void maxpool2_bwd_kernel(const float *__restrict__ dy, const int8_t *
 // xf[ci*hw + s][bi] = x[ci][bi*hw + s] (forward); inverse if `inverse`.
 __global__ void flatten_kernel(const float *__restrict__ in, int32_t c, int32_t b, int32_t hw, float *__restrict__ out,
                                int inverse) {
+    pdl_enter();
     const int64_t total = (int64_t)c * b * hw;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
         // e indexes the flattened layout: row f = ci*hw + s, column bi
@@ -235,7 +245,7 @@ int csrt_bias_act_fwd(float *y, const float *bias, int32_t m, int32_t n, int32_t
     CSRT_ARG(m >= 0 && n >= 0, "negative size");
     if ((int64_t)m * n == 0) return CSRT_OK;
     CSRT_ARG(y != nullptr, "y is NULL");
-    bias_act_kernel<<<grid_for((int64_t)m * n), 256, 0, as_stream(stream)>>>(y, bias, m, n, relu);
+    launch_pdl(bias_act_kernel, dim3(grid_for((int64_t)m * n)), dim3(256), 0, as_stream(stream), y, bias, m, n, relu);
     count_launch();
     return check_launch("bias_act_kernel");
 }
@@ -244,7 +254,7 @@ int csrt_relu_bwd(float *dy, const float *y, int64_t count, void *stream) {
     CSRT_ARG(count >= 0, "negative count");
     if (count == 0) return CSRT_OK;
     CSRT_ARG(dy && y, "NULL pointer");
-    relu_bwd_kernel<<<grid_for(count), 256, 0, as_stream(stream)>>>(dy, y, count);
+    launch_pdl(relu_bwd_kernel, dim3(grid_for(count)), dim3(256), 0, as_stream(stream), dy, y, count);
     count_launch();
     return check_launch("relu_bwd_kernel");
 }
@@ -253,8 +263,8 @@ int csrt_bias_grad_sgd(const float *dy, int32_t m, int32_t n, float *bias, float
     CSRT_ARG(m >= 0 && n >= 0, "negative size");
     if (m == 0) return CSRT_OK;
     CSRT_ARG(dy != nullptr || n == 0, "dy is NULL");
-    bias_grad_sgd_kernel<<<(unsigned)ceil_div<int64_t>((int64_t)m * 32, 256), 256, 0, as_stream(stream)>>>(
-        dy, m, n, bias, eta, gb_out);
+    launch_pdl(bias_grad_sgd_kernel, dim3((unsigned)ceil_div<int64_t>((int64_t)m * 32, 256)), dim3(256), 0,
+               as_stream(stream), dy, m, n, bias, eta, gb_out);
     count_launch();
     return check_launch("bias_grad_sgd_kernel");
 }
@@ -265,10 +275,11 @@ int csrt_softmax_xent(const float *z, const int32_t *labels, int32_t classes, in
     CSRT_ARG(z && labels && dz && loss, "NULL pointer");
     cudaStream_t s = as_stream(stream);
     if (n > 0) {
-        softmax_xent_kernel<<<(unsigned)ceil_div<int64_t>(n, 8), 256, 0, s>>>(z, labels, classes, n, dz, loss + 1);
+        launch_pdl(softmax_xent_kernel, dim3((unsigned)ceil_div<int64_t>(n, 8)), dim3(256), 0, s, z, labels, classes,
+                   n, dz, loss + 1);
         count_launch();
     }
-    mean_kernel<<<1, 1024, 0, s>>>(loss + 1, n, loss);
+    launch_pdl(mean_kernel, dim3(1), dim3(1024), 0, s, loss + 1, n, loss);
     count_launch();
     return check_launch("softmax_xent_kernel");
 }
@@ -278,7 +289,7 @@ int csrt_im2col(const float *x, int32_t c, int32_t b, int32_t h, int32_t w, int3
     const int64_t total = (int64_t)c * k * k * b * (h - k + 1) * (w - k + 1);
     if (total == 0) return CSRT_OK;
     CSRT_ARG(x && cols, "NULL pointer");
-    im2col_kernel<<<grid_for(total), 256, 0, as_stream(stream)>>>(x, c, b, h, w, k, cols);
+    launch_pdl(im2col_kernel, dim3(grid_for(total)), dim3(256), 0, as_stream(stream), x, c, b, h, w, k, cols);
     count_launch();
     return check_launch("im2col_kernel");
 }
@@ -288,7 +299,7 @@ int csrt_col2im(const float *dcols, int32_t c, int32_t b, int32_t h, int32_t w, 
     const int64_t total = (int64_t)c * b * h * w;
     if (total == 0) return CSRT_OK;
     CSRT_ARG(dcols && dx, "NULL pointer");
-    col2im_kernel<<<grid_for(total), 256, 0, as_stream(stream)>>>(dcols, c, b, h, w, k, dx);
+    launch_pdl(col2im_kernel, dim3(grid_for(total)), dim3(256), 0, as_stream(stream), dcols, c, b, h, w, k, dx);
     count_launch();
     return check_launch("col2im_kernel");
 }
@@ -299,7 +310,7 @@ int csrt_maxpool2_fwd(const float *x, int32_t c, int32_t b, int32_t h, int32_t w
     const int64_t total = (int64_t)c * b * (h / 2) * (w / 2);
     if (total == 0) return CSRT_OK;
     CSRT_ARG(x && y && idx, "NULL pointer");
-    maxpool2_fwd_kernel<<<grid_for(total), 256, 0, as_stream(stream)>>>(x, c, b, h, w, y, idx);
+    launch_pdl(maxpool2_fwd_kernel, dim3(grid_for(total)), dim3(256), 0, as_stream(stream), x, c, b, h, w, y, idx);
     count_launch();
     return check_launch("maxpool2_fwd_kernel");
 }
@@ -310,7 +321,7 @@ int csrt_maxpool2_bwd(const float *dy, const int8_t *idx, int32_t c, int32_t b, 
     const int64_t total = (int64_t)c * b * h * w;
     if (total == 0) return CSRT_OK;
     CSRT_ARG(dy && idx && dx, "NULL pointer");
-    maxpool2_bwd_kernel<<<grid_for(total), 256, 0, as_stream(stream)>>>(dy, idx, c, b, h, w, dx);
+    launch_pdl(maxpool2_bwd_kernel, dim3(grid_for(total)), dim3(256), 0, as_stream(stream), dy, idx, c, b, h, w, dx);
     count_launch();
     return check_launch("maxpool2_bwd_kernel");
 }
@@ -320,7 +331,7 @@ int csrt_flatten(const float *x, int32_t c, int32_t b, int32_t hw, float *xf, vo
     const int64_t total = (int64_t)c * b * hw;
     if (total == 0) return CSRT_OK;
     CSRT_ARG(x && xf, "NULL pointer");
-    flatten_kernel<<<grid_for(total), 256, 0, as_stream(stream)>>>(x, c, b, hw, xf, 0);
+    launch_pdl(flatten_kernel, dim3(grid_for(total)), dim3(256), 0, as_stream(stream), x, c, b, hw, xf, 0);
     count_launch();
     return check_launch("flatten_kernel");
 }
@@ -330,7 +341,7 @@ int csrt_unflatten(const float *xf, int32_t c, int32_t b, int32_t hw, float *x, 
     const int64_t total = (int64_t)c * b * hw;
     if (total == 0) return CSRT_OK;
     CSRT_ARG(x && xf, "NULL pointer");
-    flatten_kernel<<<grid_for(total), 256, 0, as_stream(stream)>>>(xf, c, b, hw, x, 1);
+    launch_pdl(flatten_kernel, dim3(grid_for(total)), dim3(256), 0, as_stream(stream), xf, c, b, hw, x, 1);
     count_launch();
     return check_launch("flatten_kernel");
 }

@@ -196,6 +196,7 @@ __device__ __forceinline__ void spmm_complete_shared_row(const SpmmArgs &a, int 
 
 template <int VW, int NV>
 __global__ void __launch_bounds__(kSpThreads, 3) spmm_merge_kernel(SpmmArgs a) {
+    pdl_enter();
     constexpr int TN = 32 * VW * NV;
     constexpr int kStride = 32 * VW;
     const int lane = threadIdx.x & 31;
@@ -264,6 +265,7 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_merge_kernel(SpmmArgs a) {
 // at once; the first one sums the row's carries column by column.
 template <int TN>
 __global__ void __launch_bounds__(256) spmm_fixup_kernel(SpmmArgs a) {
+    pdl_enter();
     const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     if (gw >= (int64_t)a.units * a.n_tiles) return;
@@ -373,15 +375,16 @@ static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *
     }
     const int64_t threads = (int64_t)sh.units * sh.n_tiles * 32;
     const unsigned grid = (unsigned)ceil_div<int64_t>(threads, kSpThreads);
-#define CSRT_SPMM_CASE(VW, NV)                                                               \
-    if (sh.vw == VW && sh.nv == NV) {                                                        \
-        spmm_merge_kernel<VW, NV><<<grid, kSpThreads, 0, s>>>(a);                            \
-        count_launch();                                                                      \
-        if (sh.units > 1 && a.cnt == nullptr) {                                              \
-            const int64_t ft = (int64_t)sh.units * sh.n_tiles * 32;                            \
-            spmm_fixup_kernel<32 * VW * NV><<<(unsigned)ceil_div<int64_t>(ft, 256), 256, 0, s>>>(a); \
-            count_launch();                                                                  \
-        }                                                                                    \
+#define CSRT_SPMM_CASE(VW, NV)                                                              \
+    if (sh.vw == VW && sh.nv == NV) {                                                       \
+        launch_pdl(spmm_merge_kernel<VW, NV>, dim3(grid), dim3(kSpThreads), 0, s, a);       \
+        count_launch();                                                                     \
+        if (sh.units > 1 && a.cnt == nullptr) {                                             \
+            const int64_t ft = (int64_t)sh.units * sh.n_tiles * 32;                         \
+            const unsigned fg = (unsigned)ceil_div<int64_t>(ft, 256);                      \
+            launch_pdl(spmm_fixup_kernel<32 * VW * NV>, dim3(fg), dim3(256), 0, s, a);      \
+            count_launch();                                                                 \
+        }                                                                                   \
     }
     CSRT_SPMM_CASE(4, 2)
     else CSRT_SPMM_CASE(4, 1)
@@ -417,6 +420,7 @@ __device__ __forceinline__ int row_of_entry(const int32_t *__restrict__ row_ptr,
 
 template <int VW>
 __global__ void __launch_bounds__(kSpThreads) sddmm_kernel(SddmmArgs a) {
+    pdl_enter();
     const int lane = threadIdx.x & 31;
     const int64_t gw = ((int64_t)blockIdx.x * kSpThreads + threadIdx.x) >> 5;
     if (gw >= (int64_t)a.units * a.chunks) return;
@@ -474,6 +478,7 @@ __global__ void __launch_bounds__(kSpThreads) sddmm_kernel(SddmmArgs a) {
 __global__ void sddmm_reduce_kernel(const int32_t *__restrict__ row_ptr, int32_t rows,
                                     const float *__restrict__ partial, int64_t stride, int32_t chunks,
                                     float *__restrict__ g) {
+    pdl_enter();
     const int64_t nnz = __ldg(row_ptr + rows);
     for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < nnz; k += (int64_t)gridDim.x * blockDim.x) {
         float s = 0.f;
@@ -588,12 +593,13 @@ int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_
         a.out_stride = 0;
     }
     const unsigned grid = (unsigned)ceil_div<int64_t>((int64_t)a.units * chunks * 32, kSpThreads);
-    if (v4) sddmm_kernel<4><<<grid, kSpThreads, 0, s>>>(a);
-    else sddmm_kernel<1><<<grid, kSpThreads, 0, s>>>(a);
+    if (v4) launch_pdl(sddmm_kernel<4>, dim3(grid), dim3(kSpThreads), 0, s, a);
+    else launch_pdl(sddmm_kernel<1>, dim3(grid), dim3(kSpThreads), 0, s, a);
     count_launch();
     if (chunks > 1) {
         const unsigned rg = (unsigned)imin<int64_t>(ceil_div<int64_t>(w->capacity, 256), (int64_t)num_sms() * 8);
-        sddmm_reduce_kernel<<<rg, 256, 0, s>>>(w->row_ptr, w->rows, a.out, a.out_stride, chunks, g_nnz);
+        launch_pdl(sddmm_reduce_kernel, dim3(rg), dim3(256), 0, s, w->row_ptr, w->rows, a.out, a.out_stride, chunks,
+                   g_nnz);
         count_launch();
     }
     return check_launch("sddmm_kernel");
@@ -605,6 +611,7 @@ namespace csrt {
 __global__ void debias_kernel(const int32_t *__restrict__ row_ptr, int32_t rows, float *__restrict__ val,
                               const float *__restrict__ g, float eta, float *__restrict__ t_val,
                               const int32_t *__restrict__ t_pos) {
+    pdl_enter();
     const int64_t nnz = __ldg(row_ptr + rows);
     for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < nnz; k += (int64_t)gridDim.x * blockDim.x) {
         const float nv = __fsub_rn(val[k], __fmul_rn(eta, __ldg(g + k)));
@@ -622,7 +629,8 @@ extern "C" int debias_update(csrt_csr *w, const float *g_nnz, float eta, void *s
     CSRT_ARG(g_nnz != nullptr, "g_nnz is NULL");
     CSRT_ARG(w->t_val == nullptr || w->t_pos != nullptr, "t_val set without t_pos");
     const unsigned grid = (unsigned)imax<int64_t>(1, imin<int64_t>(ceil_div<int64_t>(w->capacity, 256), (int64_t)num_sms() * 8));
-    debias_kernel<<<grid, 256, 0, as_stream(stream)>>>(w->row_ptr, w->rows, w->val, g_nnz, eta, w->t_val, w->t_pos);
+    launch_pdl(debias_kernel, dim3(grid), dim3(256), 0, as_stream(stream), w->row_ptr, w->rows, w->val, g_nnz, eta,
+               w->t_val, w->t_pos);
     count_launch();
     return check_launch("debias_kernel");
 }
@@ -708,17 +716,17 @@ extern "C" int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, fl
     const unsigned grid = (unsigned)ceil_div<int64_t>((int64_t)sh.units * sh.n_tiles * 32, kSpThreads);
     const unsigned fgrid = (unsigned)ceil_div<int64_t>((int64_t)sh.units * sh.n_tiles * 32, 256);
     if (sh.vw == 4 && sh.nv == 2) {
-        spmm_merge_kernel<4, 2><<<grid, kSpThreads, 0, s>>>(a);
-        if (sh.units > 1) spmm_fixup_kernel<256><<<fgrid, 256, 0, s>>>(a);
+        launch_pdl(spmm_merge_kernel<4, 2>, dim3(grid), dim3(kSpThreads), 0, s, a);
+        if (sh.units > 1) launch_pdl(spmm_fixup_kernel<256>, dim3(fgrid), dim3(256), 0, s, a);
     } else if (sh.vw == 4) {
-        spmm_merge_kernel<4, 1><<<grid, kSpThreads, 0, s>>>(a);
-        if (sh.units > 1) spmm_fixup_kernel<128><<<fgrid, 256, 0, s>>>(a);
+        launch_pdl(spmm_merge_kernel<4, 1>, dim3(grid), dim3(kSpThreads), 0, s, a);
+        if (sh.units > 1) launch_pdl(spmm_fixup_kernel<128>, dim3(fgrid), dim3(256), 0, s, a);
     } else if (sh.vw == 2) {
-        spmm_merge_kernel<2, 1><<<grid, kSpThreads, 0, s>>>(a);
-        if (sh.units > 1) spmm_fixup_kernel<64><<<fgrid, 256, 0, s>>>(a);
+        launch_pdl(spmm_merge_kernel<2, 1>, dim3(grid), dim3(kSpThreads), 0, s, a);
+        if (sh.units > 1) launch_pdl(spmm_fixup_kernel<64>, dim3(fgrid), dim3(256), 0, s, a);
     } else {
-        spmm_merge_kernel<1, 1><<<grid, kSpThreads, 0, s>>>(a);
-        if (sh.units > 1) spmm_fixup_kernel<32><<<fgrid, 256, 0, s>>>(a);
+        launch_pdl(spmm_merge_kernel<1, 1>, dim3(grid), dim3(kSpThreads), 0, s, a);
+        if (sh.units > 1) launch_pdl(spmm_fixup_kernel<32>, dim3(fgrid), dim3(256), 0, s, a);
     }
     count_launch(sh.units > 1 ? 2 : 1);
     return check_launch("spmm_fwd_noalloc");
