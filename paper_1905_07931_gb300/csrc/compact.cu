@@ -1164,14 +1164,17 @@ __global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict
 //  count: lane r loads row r's word; a 32 x 32 bit transpose (five shuffle
 //         stages) gives lane j the rows present in column 32c + j; its popcount
 //         is the block's count for that column.
-//  write: first the row pass, lane j = column 32c + j: the warp walks its 32
-//         rows in order. In row r the CSR positions of the kept columns are
-//         consecutive (word position + rank in the word), so the values are
-//         read and t_pos is written coalesced; each column's transposed run
-//         advances by one per kept row; the values go to a 32 x 32 shared
-//         tile. Then the column pass, lane r = row: for each column the rows
-//         kept in it are consecutive positions of its transposed run, so
-//         t_col and t_val are written coalesced as well.
+//  write: the block's kept entries are enumerated twice, 32 at a time, one
+//         entry per lane. Row-major order (the CSR order): the entry's row is
+//         found by a binary search over the rows' exclusive kept counts, its
+//         column as the k-th set bit of the row's word; its CSR position is
+//         the word position + k, so the value is read and t_pos written
+//         coalesced, and the value goes to a 32 x 32 shared tile.
+//         Column-major order (the transposed order): the same with the
+//         columns' counts and masks; consecutive entries of a column are
+//         consecutive positions of its transposed run, so t_col and t_val
+//         are written coalesced as well. A pass costs ceil(kept / 32)
+//         iterations instead of one per row (or column) of the block.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
     const int lane = threadIdx.x & 31;
@@ -1200,6 +1203,45 @@ __global__ void __launch_bounds__(256) trb_count_kernel(const uint32_t *__restri
     cnt[(int64_t)b * cols + c * 32 + lane] = __popc(colmask);
 }
 
+// Position of the k-th (from 0) set bit of m, for k < popc(m); always 0..31.
+__device__ __forceinline__ int nth_set_bit(uint32_t m, int k) {
+    int pos = 0;
+#pragma unroll
+    for (int sft = 16; sft >= 1; sft >>= 1) {
+        const int c = __popc(m & ((1u << sft) - 1u));
+        if (k >= c) {
+            k -= c;
+            m >>= sft;
+            pos += sft;
+        }
+    }
+    return pos;
+}
+
+// Largest lane r with pre(r) <= e, for pre nondecreasing over the lanes and
+// pre(0) = 0 <= e. Every lane of the warp must call it.
+__device__ __forceinline__ int warp_last_le(int pre, int e) {
+    int r = 0;
+#pragma unroll
+    for (int sft = 16; sft >= 1; sft >>= 1) {
+        const int v = __shfl_sync(0xffffffffu, pre, r + sft);
+        if (v <= e) r += sft;
+    }
+    return r;
+}
+
+__device__ __forceinline__ int warp_exclusive_sum(int x, int &total) {
+    const int lane = threadIdx.x & 31;
+    int inc = x;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, inc, d);
+        if (lane >= d) inc += y;
+    }
+    total = __shfl_sync(0xffffffffu, inc, 31);
+    return inc - x;
+}
+
 __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restrict__ keepbits,
                                                         const int32_t *__restrict__ wordpos, int32_t rows,
                                                         int32_t wpr, int32_t cols, const int32_t *__restrict__ off,
@@ -1208,7 +1250,7 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
                                                         float *__restrict__ t_val, int32_t *__restrict__ t_pos,
                                                         int64_t capacity) {
     pdl_enter();
-    __shared__ float tile[8][32 * 32];   // element (r, j) at r*32 + (j ^ r): rows and columns conflict-free
+    __shared__ float tile[8][32 * 32];   // element (r, j) at r*32 + (j ^ r)
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nb = ceil_div<int64_t>(rows, 32);
@@ -1218,33 +1260,42 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
     const uint32_t rw_mine = my_row < rows ? __ldg(keepbits + (int64_t)my_row * wpr + c) : 0u;
     const int32_t rp_mine = my_row < rows ? __ldg(wordpos + (int64_t)my_row * wpr + c) : 0;
     const int col = c * 32 + lane;
-    const int64_t pc0 = (int64_t)__ldg(t_row_ptr + col) + __ldg(off + (int64_t)b * cols + col);
-    const unsigned lt = (1u << lane) - 1u;
+    // start of this block's part of column `col`'s transposed run
+    const int64_t cb_mine = (int64_t)__ldg(t_row_ptr + col) + __ldg(off + (int64_t)b * cols + col);
+    const uint32_t cm_mine = warp_transpose32(rw_mine);   // lane j: the block's rows kept in column 32c + j
+    int total;
+    const int rpre = warp_exclusive_sum(__popc(rw_mine), total);
+    const int cpre = warp_exclusive_sum(__popc(cm_mine), total);
     float *tl = tile[warp];
-    const int nr = imin(32, rows - b * 32);
-    int64_t pc = pc0;
-    for (int r = 0; r < nr; ++r) {   // row pass
+    for (int e0 = 0; e0 < total; e0 += 32) {   // row-major (CSR) order
+        const int e = e0 + lane;
+        const int r = warp_last_le(rpre, e);
         const uint32_t rw = __shfl_sync(0xffffffffu, rw_mine, r);
-        if (rw == 0u) continue;
+        const int k = e - __shfl_sync(0xffffffffu, rpre, r);
         const int32_t rp = __shfl_sync(0xffffffffu, rp_mine, r);
-        if ((rw >> lane) & 1u) {
-            const int64_t pr = (int64_t)rp + __popc(rw & lt);
-            tl[r * 32 + (lane ^ r)] = pr < capacity ? __ldg(val + pr) : 0.f;
+        const int j = nth_set_bit(rw, k);
+        const uint32_t cm = __shfl_sync(0xffffffffu, cm_mine, j);
+        const int64_t cb = __shfl_sync(0xffffffffu, cb_mine, j);
+        if (e < total) {
+            const int64_t pr = (int64_t)rp + k;
+            const int64_t pc = cb + __popc(cm & ((1u << r) - 1u));
+            tl[r * 32 + (j ^ r)] = pr < capacity ? __ldg(val + pr) : 0.f;
             if (pc < capacity && pr < capacity) t_pos[pr] = (int32_t)pc;
-            ++pc;
         }
     }
     __syncwarp();
-    const uint32_t colmask = warp_transpose32(rw_mine);   // lane j: the block's rows kept in column 32c + j
-    for (int jj = 0; jj < 32; ++jj) {   // column pass
-        const uint32_t cm = __shfl_sync(0xffffffffu, colmask, jj);
-        if (cm == 0u) continue;
-        const int64_t base = __shfl_sync(0xffffffffu, pc0, jj);
-        if ((cm >> lane) & 1u) {
-            const int64_t p = base + __popc(cm & lt);
+    for (int e0 = 0; e0 < total; e0 += 32) {   // column-major (transposed) order
+        const int e = e0 + lane;
+        const int j = warp_last_le(cpre, e);
+        const uint32_t cm = __shfl_sync(0xffffffffu, cm_mine, j);
+        const int k = e - __shfl_sync(0xffffffffu, cpre, j);
+        const int64_t cb = __shfl_sync(0xffffffffu, cb_mine, j);
+        const int r = nth_set_bit(cm, k);
+        if (e < total) {
+            const int64_t p = cb + k;
             if (p < capacity) {
-                t_col[p] = b * 32 + lane;
-                t_val[p] = tl[lane * 32 + (jj ^ lane)];
+                t_col[p] = b * 32 + r;
+                t_val[p] = tl[r * 32 + (j ^ r)];
             }
         }
     }

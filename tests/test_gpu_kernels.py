@@ -657,10 +657,12 @@ def test_bounded_waits_give_up_and_report(C):
     assert ws.status()[0] == 0
 
 
-def test_fused_gradient_prox_capacity_overflow(C):
+@pytest.mark.parametrize("transposed", [False, True])
+def test_fused_gradient_prox_capacity_overflow(C, transposed):
     """An output CSR too small for the fused op's result: the overflow and the
     needed nnz are reported, the row pointers are clamped, and the stored
-    prefix equals the unfused result's."""
+    prefix equals the unfused result's (the transposed copy, when asked for,
+    writes only inside the capacity)."""
     m, k, n = 256, 512, 64
     rng = np.random.default_rng(9)
     a = _sparse(rng, m, k, 0.1) * F32(0.05)
@@ -676,7 +678,7 @@ def test_fused_gradient_prox_capacity_overflow(C):
     nnz = int(rp_ref[-1])
     assert ws.status()[0] == 0
     cap = nnz // 3
-    out = C.CSR(m, k, capacity=cap, transposed=False)
+    out = C.CSR(m, k, capacity=cap, transposed=transposed)
     C.weight_grad_prox_update(w_in, dy, x, 0.5, 0.01, out, ws)
     flags, required = ws.status()
     assert flags & C.CSRT_DEV_CAPACITY and required == nnz
