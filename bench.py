@@ -51,7 +51,7 @@ WORKLOAD = "fc_head 9216-4096-4096-1000 CSR 5/5/15%, batch 256, prox-SGD step (e
 def parse_args():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--steps", type=int, default=50)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--precision", choices=["tf32", "fp32"], default="tf32")
@@ -464,6 +464,25 @@ def main():
         if len(cands) > 1:
             roof["other"] = {k: cands[1][k] for k in ("bound", "achieved", "peak", "unit", "frac")}
 
+    # the largest sparse product of the step against its own roofs: FP32 FMA
+    # (measured with the library's probe), HBM (algorithmic bytes), and the
+    # rate at which its stored entries gather rows of the dense operand (L2)
+    spmm_names = ("spmm_fwd", "spmm_bwd_t", "spmm_fwd_bias_act", "spmm_bwd_t_relu")
+    sp = max((r for r in prof if r["name"] in spmm_names and r["info"].get("n")), key=lambda r: r["ms"],
+             default=None)
+    spmm_roof = None
+    if sp is not None:
+        t_sp = sp["ms"] / 1e3
+        fl = 2.0 * sp["info"]["nnz"] * sp["info"]["n"]
+        fma_peak = C.fma_peak_tflops()
+        b_sp = op_bytes(sp["name"], sp["info"])
+        spmm_roof = {"op": sp["label"], "kernel": sp["kernel"], "launch_ms": round(sp["ms"], 4),
+                     "fp32_tflops": round(fl / t_sp / 1e12, 2), "fma_peak_tflops": round(fma_peak, 1),
+                     "fma_frac": round(fl / t_sp / 1e12 / fma_peak, 4),
+                     "hbm_gbs": round(b_sp / t_sp / 1e9, 1), "hbm_frac": round(b_sp / t_sp / 1e9 / peaks["hbm_gbs"], 4),
+                     "gather_tbs": round(4.0 * sp["info"]["nnz"] * sp["info"]["n"] / t_sp / 1e12, 2),
+                     "note": "gather = 4*nnz*n bytes of dense-operand rows read per call (from L2)"}
+
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(total_max_ms / args.steps, 4), "higher_is_better": True,
@@ -480,6 +499,7 @@ def main():
                 "h2d_bytes_per_step": int(x_host.numel() * 4 + lab_host.numel() * 4), "d2h_bytes_per_step": 4},
         "gpu_launches": int(launches_per_step * args.steps),
         "roofline": roof,
+        "spmm_roofline": spmm_roof,
         "clocks": clk,
         "wall_s_timed_region": round(wall, 3),
     }

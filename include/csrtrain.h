@@ -114,6 +114,15 @@ int csrt_workspace_bytes(int32_t rows, int32_t cols, int32_t max_n, size_t *byte
  * first 16 bytes of the workspace scratch. */
 int csrt_check_bounded_waits(void *ws, size_t ws_bytes, void *stream);
 
+/* csrt_fma_peak_run -- measurement aid (not part of the training step): a
+ * kernel of `blocks` blocks of 512 threads, each thread running 8 independent
+ * FP32 fused multiply-add chains for `iters` rounds, then storing one float
+ * to out[blocks*512] (device). *flops (host, may be NULL) receives the
+ * floating-point operations it performs (2 per FMA). The caller times it
+ * (e.g. with events on `stream`) to obtain the GPU's FP32 FMA throughput,
+ * the roof of the CUDA-core sparse products. */
+int csrt_fma_peak_run(float *out, int32_t blocks, int32_t iters, double *flops, void *stream);
+
 /* Zero the whole workspace (status word included) on `stream`. */
 int csrt_workspace_init(void *ws, size_t ws_bytes, void *stream);
 

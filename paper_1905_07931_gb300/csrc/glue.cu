@@ -235,11 +235,42 @@ __global__ void flatten_kernel(const float *__restrict__ in, int32_t c, int32_t 
     }
 }
 
+// FP32 FMA throughput probe (the roof of the CUDA-core products): every
+// thread runs kFmaChains independent fused multiply-add chains
+// (x <- x*b + c with |b| < 1, so the values stay finite) for `iters` rounds
+// and stores their sum, so nothing is optimised away.
+constexpr int kFmaChains = 8;
+constexpr int kFmaThreads = 512;
+__global__ void __launch_bounds__(kFmaThreads) fma_peak_kernel(float *__restrict__ out, int32_t iters, float b,
+                                                                float c) {
+    pdl_enter();
+    float x[kFmaChains];
+#pragma unroll
+    for (int k = 0; k < kFmaChains; ++k) x[k] = (float)(threadIdx.x + k) * 1e-3f;
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+        for (int k = 0; k < kFmaChains; ++k) x[k] = fmaf(x[k], b, c);
+    }
+    float sum = 0.f;
+#pragma unroll
+    for (int k = 0; k < kFmaChains; ++k) sum += x[k];
+    out[(int64_t)blockIdx.x * blockDim.x + threadIdx.x] = sum;
+}
+
 }  // namespace csrt
 
 using namespace csrt;
 
 extern "C" {
+
+int csrt_fma_peak_run(float *out, int32_t blocks, int32_t iters, double *flops, void *stream) {
+    CSRT_ARG(out != nullptr && blocks > 0 && iters > 0, "bad probe arguments");
+    if (flops) *flops = 2.0 * (double)blocks * kFmaThreads * kFmaChains * (double)iters;
+    launch_pdl(fma_peak_kernel, dim3((unsigned)blocks), dim3(kFmaThreads), 0, as_stream(stream), out, iters,
+               0.999999f, 1e-6f);
+    count_launch();
+    return check_launch("fma_peak_kernel");
+}
 
 int csrt_bias_act_fwd(float *y, const float *bias, int32_t m, int32_t n, int32_t relu, void *stream) {
     CSRT_ARG(m >= 0 && n >= 0, "negative size");

@@ -70,6 +70,7 @@ _SIGS = {
     "csrt_im2col": [c_void_p, c_int32, c_int32, c_int32, c_int32, c_int32, c_void_p, c_void_p],
     "csrt_col2im": [c_void_p, c_int32, c_int32, c_int32, c_int32, c_int32, c_void_p, c_void_p],
     "csrt_check_bounded_waits": [c_void_p, c_size_t, c_void_p],
+    "csrt_fma_peak_run": [c_void_p, c_int32, c_int32, ctypes.POINTER(ctypes.c_double), c_void_p],
     "csrt_conv2d_sparse_fwd": [POINTER(csrt_csr), c_void_p, c_int32, c_int32, c_int32, c_int32, c_int32, c_void_p,
                                c_int32, c_void_p, c_void_p],
     "csrt_maxpool2_fwd": [c_void_p, c_int32, c_int32, c_int32, c_int32, c_void_p, c_void_p, c_void_p],
@@ -383,6 +384,33 @@ def check_bounded_waits(ws: Workspace, stream=None):
     """Run the library's bounded waits against events that never happen; they
     must give up and set CSRT_DEV_TIMEOUT (read it with ws.status())."""
     _check(lib().csrt_check_bounded_waits(ws.ptr, ws.nbytes, _stream(stream)), "csrt_check_bounded_waits")
+
+
+def fma_peak_tflops(reps: int = 5) -> float:
+    """Measured FP32 FMA throughput of the current GPU (TFLOP/s): the median of
+    `reps` timed runs of the library's FMA probe (two waves of blocks per SM,
+    after a warm-up run), timed with CUDA events on the current stream."""
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    blocks, iters = 4 * sms, 1 << 15
+    out = torch.empty(blocks * 512, dtype=torch.float32, device="cuda")
+    flops = ctypes.c_double(0.0)
+    s = torch.cuda.current_stream()
+
+    def run():
+        _check(lib().csrt_fma_peak_run(_ptr(out), blocks, iters, ctypes.byref(flops), _stream(s)),
+               "csrt_fma_peak_run")
+
+    run()
+    times = []
+    for _ in range(reps):
+        st, en = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        st.record(s)
+        run()
+        en.record(s)
+        en.synchronize()
+        times.append(st.elapsed_time(en) / 1e3)
+    times.sort()
+    return flops.value / times[len(times) // 2] / 1e12
 
 
 def conv2d_sparse_fwd(w: CSR, x, c, b, h, wd, k, bias, relu, y, stream=None):

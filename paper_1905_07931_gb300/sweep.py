@@ -14,7 +14,8 @@ L2 flushed before every timed launch):
   G never written) and as two calls (weight_grad_dense + prox_update_compact).
 
 For each it prints the time, the algorithmic bytes (each operand touched
-once) and the achieved GB/s, and the FLOP rate for the products. One
+once) and the achieved GB/s, and for the products the FLOP rate and its
+fraction of the GPU's FP32 FMA throughput (measured in the same run). One
 operation on one shape can be selected (for profiling one kernel).
 
   python -m paper_1905_07931_gb300.sweep                      # the full sweep
@@ -153,11 +154,19 @@ def main(argv=None):
     for d in a.density:
         for z in zipfs:
             out += run_layer(a.m, a.k, d, z, a.n, ops, a.reps, transposed=not a.no_transposed)
+    if ops & {"spmm_fwd", "spmm_bwd_t", "sddmm"}:
+        # the CUDA-core products against the measured FP32 FMA throughput
+        peak = C.fma_peak_tflops()
+        for r in out:
+            if "tflops" in r:
+                r["fma_peak_tflops"] = round(peak, 1)
+                r["fma_frac"] = round(r["tflops"] / peak, 4)
     if a.json:
         print(json.dumps(out))
     else:
         for r in out:
-            extra = f" nnz'={r['nnz_out']}" if "nnz_out" in r else f" {r['tflops']:6.2f} TFLOP/s"
+            extra = (f" nnz'={r['nnz_out']}" if "nnz_out" in r else
+                     f" {r['tflops']:6.2f} TFLOP/s ({100 * r.get('fma_frac', 0):.1f}% of FP32 FMA)")
             print(f"{r['op']:<20s} d={r['density']:.2f} {r['rows']:<7s} n={r['n']:<5d} nnz={r['nnz']:<8d} "
                   f"{r['us']:9.1f} us {r['gbs']:8.1f} GB/s{extra}")
     return 0

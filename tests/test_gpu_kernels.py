@@ -160,6 +160,11 @@ SPMM_CASES = [
     (129, 1000, 128, 0.2, False),
     (257, 300, 384, 0.3, True),
     (2048, 1024, 256, 0.05, False),
+    # tall products: thousands of rows, power-law rows at n = 128, and a
+    # transposed product with 9000 output rows
+    (4100, 700, 256, 0.05, False),
+    (7400, 257, 128, 0.2, True),
+    (300, 9000, 256, 0.05, False),
 ]
 
 
@@ -188,7 +193,7 @@ def test_spmm_fwd_and_bwd_against_oracle(C, m, k, n, density, zipf):
 
 
 @pytest.mark.parametrize("m,k,n,zipf", [(700, 900, 256, True), (129, 257, 70, False), (50, 40, 1, False),
-                                         (300, 784, 64, False)])
+                                         (300, 784, 64, False), (4100, 4100, 256, False)])
 def test_fused_epilogues_match_unfused(C, m, k, n, zipf):
     rng = np.random.default_rng(m + k + n)
     a = _sparse(rng, m, k, 0.1, zipf)
