@@ -51,15 +51,28 @@ __global__ void bias_grad_sgd_kernel(const float *__restrict__ dy, int32_t m, in
     }
 }
 
-// Softmax cross-entropy: a block of 256 threads takes 8 samples (columns);
-// thread (class group g = 0..31, column c = 0..7) walks classes g, g+32, ...
+// Softmax cross-entropy: a block of 1024 threads takes 8 samples (columns);
+// thread (class group g = 0..127, column c = 0..7) walks classes g, g+128, ...
 // so every warp load covers 4 classes x 8 consecutive columns (32-byte
-// segments). One pass keeps a running maximum and rescaled sum; the groups
-// are combined in a fixed order in shared memory; a second pass writes dz.
-__global__ void __launch_bounds__(256) softmax_xent_kernel(const float *__restrict__ z,
-                                                           const int32_t *__restrict__ labels, int32_t classes,
-                                                           int32_t n, float *__restrict__ dz,
-                                                           float *__restrict__ per_sample) {
+// segments). One pass keeps a running maximum and rescaled sum per thread;
+// the four groups of a warp are combined by shuffles, then the 32 warps in
+// shared memory, always in the same order; a second pass writes dz.
+constexpr int kSmThreads = 1024;
+constexpr int kSmGroups = kSmThreads / 8;   // class groups per block
+
+__device__ __forceinline__ void softmax_merge(float &m, float &s, float m2, float s2) {
+    const float mx = fmaxf(m, m2);
+    float r = 0.f;
+    if (m != -INFINITY) r += s * expf(m - mx);
+    if (m2 != -INFINITY) r += s2 * expf(m2 - mx);
+    m = mx;
+    s = r;
+}
+
+__global__ void __launch_bounds__(kSmThreads) softmax_xent_kernel(const float *__restrict__ z,
+                                                                  const int32_t *__restrict__ labels,
+                                                                  int32_t classes, int32_t n, float *__restrict__ dz,
+                                                                  float *__restrict__ per_sample) {
     pdl_enter();
     __shared__ float s_m[32][8], s_s[32][8];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -70,16 +83,16 @@ __global__ void __launch_bounds__(256) softmax_xent_kernel(const float *__restri
     float m = -INFINITY, sum = 0.f;
     constexpr int kBatch = 8;   // class values loaded together, then folded in order
     if (ok) {
-        for (int c0 = grp; c0 < classes; c0 += 32 * kBatch) {
+        for (int c0 = grp; c0 < classes; c0 += kSmGroups * kBatch) {
             float xs[kBatch];
 #pragma unroll
             for (int u = 0; u < kBatch; ++u) {
-                const int c = c0 + 32 * u;
+                const int c = c0 + kSmGroups * u;
                 xs[u] = c < classes ? __ldg(z + (int64_t)c * n + col) : -INFINITY;
             }
 #pragma unroll
             for (int u = 0; u < kBatch; ++u) {
-                if (c0 + 32 * u >= classes) break;
+                if (c0 + kSmGroups * u >= classes) break;
                 const float x = xs[u];
                 if (x > m) {
                     sum = sum * expf(m - x) + 1.f;
@@ -90,31 +103,46 @@ __global__ void __launch_bounds__(256) softmax_xent_kernel(const float *__restri
             }
         }
     }
-    s_m[grp][cl] = m;
-    s_s[grp][cl] = sum;
+    // the warp's four groups of each column (lanes cl, cl+8, cl+16, cl+24)
+#pragma unroll
+    for (int off = 8; off <= 16; off <<= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+        const float s2 = __shfl_xor_sync(0xffffffffu, sum, off);
+        if (lane & off) softmax_merge(m, sum, m2, s2);   // same operands in both lanes, in a fixed order
+        else {
+            float mm = m2, ss = s2;
+            softmax_merge(mm, ss, m, sum);
+            m = mm;
+            sum = ss;
+        }
+    }
+    if (lane < 8) {
+        s_m[warp][cl] = m;
+        s_s[warp][cl] = sum;
+    }
     __syncthreads();
     float mx = -INFINITY;
-    for (int g = 0; g < 32; ++g) mx = fmaxf(mx, s_m[g][cl]);
+    for (int w = 0; w < 32; ++w) mx = fmaxf(mx, s_m[w][cl]);
     float se = 0.f;
-    for (int g = 0; g < 32; ++g) {
-        const float mg = s_m[g][cl];
-        if (mg != -INFINITY) se += s_s[g][cl] * expf(mg - mx);
+    for (int w = 0; w < 32; ++w) {
+        const float mw = s_m[w][cl];
+        if (mw != -INFINITY) se += s_s[w][cl] * expf(mw - mx);
     }
     if (!ok) return;
     const float inv = 1.f / se;
     const float inv_n = 1.f / (float)n;
     const int lab = __ldg(labels + col);
     const bool lab_ok = lab >= 0 && lab < classes;   // an invalid label gives a NaN loss
-    for (int c0 = grp; c0 < classes; c0 += 32 * kBatch) {
+    for (int c0 = grp; c0 < classes; c0 += kSmGroups * kBatch) {
         float xs[kBatch];
 #pragma unroll
         for (int u = 0; u < kBatch; ++u) {
-            const int c = c0 + 32 * u;
+            const int c = c0 + kSmGroups * u;
             xs[u] = c < classes ? __ldg(z + (int64_t)c * n + col) : 0.f;
         }
 #pragma unroll
         for (int u = 0; u < kBatch; ++u) {
-            const int c = c0 + 32 * u;
+            const int c = c0 + kSmGroups * u;
             if (c >= classes) break;
             const float p = expf(xs[u] - mx) * inv;
             dz[(int64_t)c * n + col] = (p - (c == lab ? 1.f : 0.f)) * inv_n;
@@ -306,8 +334,8 @@ int csrt_softmax_xent(const float *z, const int32_t *labels, int32_t classes, in
     CSRT_ARG(z && labels && dz && loss, "NULL pointer");
     cudaStream_t s = as_stream(stream);
     if (n > 0) {
-        launch_pdl(softmax_xent_kernel, dim3((unsigned)ceil_div<int64_t>(n, 8)), dim3(256), 0, s, z, labels, classes,
-                   n, dz, loss + 1);
+        launch_pdl(softmax_xent_kernel, dim3((unsigned)ceil_div<int64_t>(n, 8)), dim3(kSmThreads), 0, s, z, labels,
+                   classes, n, dz, loss + 1);
         count_launch();
     }
     launch_pdl(mean_kernel, dim3(1), dim3(1024), 0, s, loss + 1, n, loss);
