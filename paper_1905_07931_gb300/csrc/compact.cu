@@ -1174,7 +1174,10 @@ __global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict
 //         columns' counts and masks; consecutive entries of a column are
 //         consecutive positions of its transposed run, so t_col and t_val
 //         are written coalesced as well. A pass costs ceil(kept / 32)
-//         iterations instead of one per row (or column) of the block.
+//         iterations instead of one per row (or column) of the block; a
+//         block with more than kTrbWalkMin kept entries is instead walked
+//         row by row (lane = column) and column by column (lane = row),
+//         which is cheaper once most lanes hold an entry.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
     const int lane = threadIdx.x & 31;
@@ -1242,6 +1245,8 @@ __device__ __forceinline__ int warp_exclusive_sum(int x, int &total) {
     return inc - x;
 }
 
+constexpr int kTrbWalkMin = 384;   // kept entries of a 32 x 32 block above which it is walked
+
 __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restrict__ keepbits,
                                                         const int32_t *__restrict__ wordpos, int32_t rows,
                                                         int32_t wpr, int32_t cols, const int32_t *__restrict__ off,
@@ -1267,6 +1272,38 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
     const int rpre = warp_exclusive_sum(__popc(rw_mine), total);
     const int cpre = warp_exclusive_sum(__popc(cm_mine), total);
     float *tl = tile[warp];
+    if (total > kTrbWalkMin) {
+        // a dense block: walk its rows (lane = column) and then its columns
+        // (lane = row); a step per row or column costs less than the search
+        // of the enumeration once most lanes hold an entry
+        const unsigned lt = (1u << lane) - 1u;
+        int64_t pc = cb_mine;
+        for (int r = 0; r < 32; ++r) {
+            const uint32_t rw = __shfl_sync(0xffffffffu, rw_mine, r);
+            if (rw == 0u) continue;
+            const int32_t rp = __shfl_sync(0xffffffffu, rp_mine, r);
+            if ((rw >> lane) & 1u) {
+                const int64_t pr = (int64_t)rp + __popc(rw & lt);
+                tl[r * 32 + (lane ^ r)] = pr < capacity ? __ldg(val + pr) : 0.f;
+                if (pc < capacity && pr < capacity) t_pos[pr] = (int32_t)pc;
+                ++pc;
+            }
+        }
+        __syncwarp();
+        for (int j = 0; j < 32; ++j) {
+            const uint32_t cm = __shfl_sync(0xffffffffu, cm_mine, j);
+            if (cm == 0u) continue;
+            const int64_t base = __shfl_sync(0xffffffffu, cb_mine, j);
+            if ((cm >> lane) & 1u) {
+                const int64_t p = base + __popc(cm & lt);
+                if (p < capacity) {
+                    t_col[p] = b * 32 + lane;
+                    t_val[p] = tl[lane * 32 + (j ^ lane)];
+                }
+            }
+        }
+        return;
+    }
     for (int e0 = 0; e0 < total; e0 += 32) {   // row-major (CSR) order
         const int e = e0 + lane;
         const int r = warp_last_le(rpre, e);
