@@ -17,7 +17,9 @@
 // nonzeros are in flight per lane. A row cut by a unit boundary leaves a
 // partial sum ("carry") in the workspace; a fix-up kernel adds the carries of
 // each cut row in unit order, so the result is deterministic and no float
-// atomics are used.
+// atomics are used. Narrow products (n <= 16 floats per vector width) put a
+// group of G < 32 lanes on each nonzero instead (spmm_group_kernel), and the
+// SDDMM uses the same grouped layout.
 #include "common.cuh"
 
 namespace csrt {
@@ -159,11 +161,14 @@ __device__ __forceinline__ void spmm_consume(const SpmmArgs &a, int64_t k, int64
 // arrive adds the carries in unit order to the partial row, applies the
 // epilogue and resets the counter. The sum is the fix-up kernel's, in the
 // same order; no unit waits for another.
-template <int VW, int NV>
+// G is the number of lanes that hold one row segment (32, or the group width
+// of the narrow kernel): lane gl < G holds the tile columns gl*VW + v*G*VW.
+template <int VW, int NV, int G = 32>
 __device__ __forceinline__ void spmm_complete_shared_row(const SpmmArgs &a, int r, int64_t per, int t, int n0) {
-    constexpr int TN = 32 * VW * NV;
-    constexpr int kStride = 32 * VW;
+    constexpr int TN = G * VW * NV;
+    constexpr int kStride = G * VW;
     const int lane = threadIdx.x & 31;
+    const int gl = lane % G;
     const int64_t d0 = (int64_t)__ldg(a.row_ptr + r) + r, d1 = (int64_t)__ldg(a.row_ptr + r + 1) + r;
     const int ua = (int)(d0 / per), ub = (int)(d1 / per);
     __threadfence();   // this unit's part is visible before it counts in
@@ -175,12 +180,12 @@ __device__ __forceinline__ void spmm_complete_shared_row(const SpmmArgs &a, int 
 #pragma unroll
     for (int v = 0; v < NV; ++v) {
         const int c = n0 + v * kStride;
-        if (c >= a.n) continue;
+        if (lane >= G || c >= a.n) continue;
         float sum[VW];
 #pragma unroll
         for (int e = 0; e < VW; ++e) sum[e] = 0.f;
         for (int w = ua; w < ub; ++w) {
-            const float *cp = a.carry + ((int64_t)t * a.units + w) * TN + lane * VW + v * kStride;
+            const float *cp = a.carry + ((int64_t)t * a.units + w) * TN + gl * VW + v * kStride;
 #pragma unroll
             for (int e = 0; e < VW; ++e) sum[e] += __ldcg(cp + e);
         }
@@ -260,6 +265,144 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_merge_kernel(SpmmArgs a) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// Narrow products (n <= 16*VW): G lanes per nonzero.
+//
+// With all 32 lanes on one nonzero, a narrow product leaves most lanes idle
+// (n = 1: one lane in 32) and keeps only a few loads in flight, so it runs
+// far below the HBM rate that its CSR stream could reach. Here a group of
+// G lanes (G*VW >= n) takes one nonzero, so a warp step covers E = 32/G
+// nonzeros; every lane loads its group's column index and value itself
+// (one coalesced request per step), the next batch of U steps is requested
+// before the current one is consumed (also across row ends: a row's entries
+// follow the previous row's), and at the end of a row the groups' partial
+// sums are combined by a butterfly over the lane bits above G. The unit
+// split, the row-end window and the shared-row protocol are those of
+// spmm_merge_kernel (carries of TN = G*VW floats).
+// ---------------------------------------------------------------------------
+template <int VW> struct NarrowSteps { static constexpr int value = VW == 1 ? 8 : 4; };
+
+template <int VW, int G>
+__global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
+    pdl_enter();
+    constexpr int E = 32 / G;
+    constexpr int U = NarrowSteps<VW>::value;
+    constexpr int B = U * E;
+    constexpr int TN = G * VW;
+    const int lane = threadIdx.x & 31, grp = lane / G, gl = lane % G;
+    const int64_t gw = ((int64_t)blockIdx.x * kSpThreads + threadIdx.x) >> 5;
+    if (gw >= (int64_t)a.units * a.n_tiles) return;
+    const int u = (int)(gw % a.units);
+    const int t = (int)(gw / a.units);
+    const int64_t nnz = __ldg(a.row_ptr + a.rows);
+    const int64_t items = (int64_t)a.rows + nnz;
+    const int64_t per = ceil_div<int64_t>(items, a.units);
+    const int64_t d0 = min((int64_t)u * per, items), d1 = min(d0 + per, items);
+    const int i0 = merge_rows_before(a.row_ptr, d0, imax<int64_t>(0, d0 - nnz), imin<int64_t>(d0, a.rows));
+    const int i1 = merge_rows_before(a.row_ptr, d1, imax<int64_t>(0, d1 - nnz), imin<int64_t>(d1, a.rows));
+    const int64_t k0 = d0 - i0, k1 = d1 - i1;
+    const int c0 = t * TN + gl * VW;
+    const bool in_n = c0 < a.n;
+    const bool first_row_cut = i0 < a.rows && k0 > __ldg(a.row_ptr + i0);
+    const bool epi = a.bias || a.relu || a.mask;
+
+    // ends of rows wb .. wb+31 (one per lane); rows from i1 on end at k1 here
+    int wb = i0;
+    int64_t rpl = wb + lane < i1 ? (int64_t)__ldg(a.row_ptr + wb + lane + 1) : k1;
+    auto row_end = [&](int r) -> int64_t {
+        if (r >= i1) return k1;
+        if (r - wb >= 32) {
+            wb = r;
+            rpl = wb + lane < i1 ? (int64_t)__ldg(a.row_ptr + wb + lane + 1) : k1;
+        }
+        return __shfl_sync(0xffffffffu, rpl, r - wb);
+    };
+
+    float acc[VW];
+#pragma unroll
+    for (int e = 0; e < VW; ++e) acc[e] = 0.f;
+    int cn[U];
+    float wn[U];
+    auto fetch = [&](int64_t kb) {
+        const int32_t *cp = a.col + kb + grp;
+        const float *vp = a.val + kb + grp;
+        const int lim = (int)imin<int64_t>(k1 - kb - grp, B);
+#pragma unroll
+        for (int s = 0; s < U; ++s) {
+            const bool ok = s * E < lim;
+            cn[s] = ok ? __ldg(cp + s * E) : 0;
+            wn[s] = ok ? __ldg(vp + s * E) : 0.f;
+        }
+    };
+    // the groups' partial sums of one row, summed over the lane bits above G
+    auto combine = [&](float (&v)[VW]) {
+#pragma unroll
+        for (int e = 0; e < VW; ++e) {
+            v[e] = acc[e];
+#pragma unroll
+            for (int off = G; off < 32; off <<= 1) v[e] += __shfl_xor_sync(0xffffffffu, v[e], off);
+            acc[e] = 0.f;
+        }
+    };
+
+    int i = i0;
+    int64_t e_row = row_end(i);
+    int64_t kr = k0;   // first entry of the current row inside this unit
+    int64_t kb = k0;
+    if (kb < k1) fetch(kb);
+    for (;;) {
+        while (i < i1 && e_row <= kb) {   // rows that end here are complete
+            float v[VW];
+            combine(v);
+            if (grp == 0 && in_n) {
+                if (epi && !(i == i0 && first_row_cut)) spmm_epilogue<VW>(a, i, c0, v);
+                stv<VW>(a.y + (int64_t)i * a.n + c0, v);
+            }
+            kr = e_row;
+            ++i;
+            e_row = row_end(i);
+        }
+        if (kb >= k1) break;
+        int c[U];
+        float w[U];
+#pragma unroll
+        for (int s = 0; s < U; ++s) {
+            c[s] = cn[s];
+            w[s] = wn[s];
+        }
+        const int64_t kn = imin<int64_t>(kb + B, e_row);
+        const int rem = in_n ? (int)imin<int64_t>(e_row - kb - grp, B) : 0;
+        if (kn < k1) fetch(kn);
+        typename Vec<VW>::T xv[U];
+#pragma unroll
+        for (int s = 0; s < U; ++s)
+            if (s * E < rem) xv[s] = ldv<VW>(a.x + (int64_t)c[s] * a.n + c0);
+#pragma unroll
+        for (int s = 0; s < U; ++s)
+            if (s * E < rem) {
+                float f[VW];
+                unpack<VW>(xv[s], f);
+#pragma unroll
+                for (int e = 0; e < VW; ++e) acc[e] = fmaf(w[s], f[e], acc[e]);
+            }
+        kb = kn;
+    }
+    // the unit ends inside row i1: its part is a carry
+    const bool has_carry = k1 > kr;
+    float v[VW];
+    combine(v);
+    if (a.units > 1) {
+        if (t == 0 && lane == 0) a.carry_row[u] = has_carry ? i1 : -1;
+        if (has_carry && grp == 0) stv<VW>(a.carry + ((int64_t)t * a.units + u) * TN + gl * VW, v);
+        if (a.cnt) {
+            const int ra = first_row_cut ? i0 : -1;
+            const int rb = (has_carry && i1 != ra) ? i1 : -1;
+            if (ra >= 0) spmm_complete_shared_row<VW, 1, G>(a, ra, per, t, c0);
+            if (rb >= 0) spmm_complete_shared_row<VW, 1, G>(a, rb, per, t, c0);
+        }
+    }
+}
+
 // Adds the carries of every cut row, in unit order, to that row of Y. One warp
 // per (unit, n-tile): warps whose unit is not the first carry of its row leave
 // at once; the first one sums the row's carries column by column.
@@ -278,19 +421,21 @@ __global__ void __launch_bounds__(256) spmm_fixup_kernel(SpmmArgs a) {
     const bool epi = a.bias || a.relu || a.mask;
     // lane j holds columns j, j+32, ...: every carry's loads for them are
     // independent, so they are issued together, carry by carry in unit order
-    constexpr int kPer = TN / 32;
+    // (tiles narrower than a warp use lanes j < TN)
+    constexpr int kPer = (TN + 31) / 32;
     float sum[kPer];
 #pragma unroll
     for (int q = 0; q < kPer; ++q) sum[q] = 0.f;
     for (int v = u; v <= last; ++v) {
         const float *cp = a.carry + ((int64_t)t * a.units + v) * TN + lane;
 #pragma unroll
-        for (int q = 0; q < kPer; ++q) sum[q] += __ldg(cp + 32 * q);
+        for (int q = 0; q < kPer; ++q)
+            if (lane + 32 * q < TN) sum[q] += __ldg(cp + 32 * q);
     }
 #pragma unroll
     for (int q = 0; q < kPer; ++q) {
         const int col = t * TN + lane + 32 * q;
-        if (col >= a.n) break;
+        if (lane + 32 * q >= TN || col >= a.n) break;
         float *yp = a.y + (int64_t)r * a.n + col;
         float out[1] = {*yp + sum[q]};
         if (epi) spmm_epilogue<1>(a, r, col, out);
@@ -299,34 +444,61 @@ __global__ void __launch_bounds__(256) spmm_fixup_kernel(SpmmArgs a) {
 }
 
 struct SpmmShape {
-    int vw, nv, tn, n_tiles, units;
+    int vw, nv, g, tn, n_tiles, units;
 };
 
-template <int VW, int NV>
-static int spmm_warps_per_sm() {
-    static int cache[64] = {0};
+template <typename K>
+static int kernel_warps_per_sm(K kernel, int (&cache)[64], int cap) {
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return kWarpsPerSM;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cap;
     if (cache[dev] == 0) {
         int blocks = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, spmm_merge_kernel<VW, NV>, kSpThreads, 0) !=
-                cudaSuccess || blocks <= 0)
-            blocks = kWarpsPerSM / (kSpThreads / 32);
-        cache[dev] = imin(blocks * (kSpThreads / 32), kWarpsPerSM);
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kernel, kSpThreads, 0) != cudaSuccess ||
+            blocks <= 0)
+            blocks = cap / (kSpThreads / 32);
+        cache[dev] = imin(blocks * (kSpThreads / 32), cap);
     }
     return cache[dev];
 }
 
+template <int VW, int NV, int G>
+static int spmm_warps_per_sm() {
+    static int cache[64] = {0};
+    if constexpr (G == 32) return kernel_warps_per_sm(spmm_merge_kernel<VW, NV>, cache, kWarpsPerSM);
+    else return kernel_warps_per_sm(spmm_group_kernel<VW, G>, cache, kWarpsPerSM);
+}
+
+static int pow2_at_least(int v) {
+    int p = 1;
+    while (p < v) p <<= 1;
+    return p;
+}
+
+// Tile shape of a product with n columns: 32 lanes on one nonzero with NV
+// vectors of VW floats each (n >= 128 for float4, 64 for float2, 32 for
+// scalars), else the narrow kernel with G = the smallest power of two with
+// G*VW >= n lanes per nonzero.
 static SpmmShape spmm_shape(int32_t n, int64_t max_items, bool vec4_ok, bool vec2_ok) {
     SpmmShape s;
+    s.nv = 1;
+    s.g = 32;
     if (vec4_ok && n >= 128) { s.vw = 4; s.nv = n >= 256 ? 2 : 1; }
-    else if (vec2_ok && n >= 64) { s.vw = 2; s.nv = 1; }
-    else { s.vw = 1; s.nv = 1; }
-    s.tn = 32 * s.vw * s.nv;
+    else if (vec4_ok && n <= 64) { s.vw = 4; s.g = pow2_at_least((n + 3) / 4); }
+    else if (vec2_ok && n >= 64) { s.vw = 2; }
+    else if (vec2_ok && n <= 32) { s.vw = 2; s.g = pow2_at_least((n + 1) / 2); }
+    else if (n <= 16) { s.vw = 1; s.g = pow2_at_least(n); }
+    else { s.vw = 1; }
+    s.tn = s.g * s.vw * s.nv;
     s.n_tiles = (int)ceil_div<int64_t>(n, s.tn);
     // one full wave of resident warps (a partial second wave would run at low occupancy)
-    const int wps = s.vw == 4 ? (s.nv == 2 ? spmm_warps_per_sm<4, 2>() : spmm_warps_per_sm<4, 1>())
-                    : s.vw == 2 ? spmm_warps_per_sm<2, 1>() : spmm_warps_per_sm<1, 1>();
+    int wps = kWarpsPerSM;
+#define CSRT_SPMM_WPS(VW, NV, G) \
+    if (s.vw == VW && s.nv == NV && s.g == G) wps = spmm_warps_per_sm<VW, NV, G>();
+    CSRT_SPMM_WPS(4, 2, 32) CSRT_SPMM_WPS(4, 1, 32) CSRT_SPMM_WPS(2, 1, 32) CSRT_SPMM_WPS(1, 1, 32)
+    CSRT_SPMM_WPS(4, 1, 1) CSRT_SPMM_WPS(4, 1, 2) CSRT_SPMM_WPS(4, 1, 4) CSRT_SPMM_WPS(4, 1, 8) CSRT_SPMM_WPS(4, 1, 16)
+    CSRT_SPMM_WPS(2, 1, 1) CSRT_SPMM_WPS(2, 1, 2) CSRT_SPMM_WPS(2, 1, 4) CSRT_SPMM_WPS(2, 1, 8) CSRT_SPMM_WPS(2, 1, 16)
+    CSRT_SPMM_WPS(1, 1, 1) CSRT_SPMM_WPS(1, 1, 2) CSRT_SPMM_WPS(1, 1, 4) CSRT_SPMM_WPS(1, 1, 8) CSRT_SPMM_WPS(1, 1, 16)
+#undef CSRT_SPMM_WPS
     const int64_t target = (int64_t)num_sms() * wps;
     int64_t units = ceil_div<int64_t>(target, s.n_tiles);
     units = imax<int64_t>(1, imin<int64_t>(units, max_items));
@@ -339,6 +511,43 @@ size_t spmm_scratch_bytes(int32_t max_n) {
     const int64_t target = (int64_t)num_sms() * kWarpsPerSM;
     const int64_t floats = (target + 1) * 256 + (int64_t)max_n + 256;
     return (size_t)floats * sizeof(float) + (size_t)(target + 1) * sizeof(int32_t) + 512;
+}
+
+// Launches the product kernel of shape sh (and, for rows cut by units when
+// a.cnt is null, the fix-up kernel); returns the number of launches, or -1
+// for a shape without a kernel.
+static int spmm_dispatch(const SpmmShape &sh, const SpmmArgs &a, cudaStream_t s) {
+    const int64_t threads = (int64_t)sh.units * sh.n_tiles * 32;
+    const unsigned grid = (unsigned)ceil_div<int64_t>(threads, kSpThreads);
+    const bool fix = sh.units > 1 && a.cnt == nullptr;
+    const unsigned fg = (unsigned)ceil_div<int64_t>(threads, 256);
+#define CSRT_SPMM_CASE(VW, NV, G, KERNEL)                                                   \
+    if (sh.vw == VW && sh.nv == NV && sh.g == G) {                                          \
+        launch_pdl(KERNEL, dim3(grid), dim3(kSpThreads), 0, s, a);                          \
+        if (fix) launch_pdl(spmm_fixup_kernel<G * VW * NV>, dim3(fg), dim3(256), 0, s, a); \
+        return fix ? 2 : 1;                                                                 \
+    }
+    CSRT_SPMM_CASE(4, 2, 32, (spmm_merge_kernel<4, 2>))
+    CSRT_SPMM_CASE(4, 1, 32, (spmm_merge_kernel<4, 1>))
+    CSRT_SPMM_CASE(2, 1, 32, (spmm_merge_kernel<2, 1>))
+    CSRT_SPMM_CASE(1, 1, 32, (spmm_merge_kernel<1, 1>))
+    CSRT_SPMM_CASE(4, 1, 1, (spmm_group_kernel<4, 1>))
+    CSRT_SPMM_CASE(4, 1, 2, (spmm_group_kernel<4, 2>))
+    CSRT_SPMM_CASE(4, 1, 4, (spmm_group_kernel<4, 4>))
+    CSRT_SPMM_CASE(4, 1, 8, (spmm_group_kernel<4, 8>))
+    CSRT_SPMM_CASE(4, 1, 16, (spmm_group_kernel<4, 16>))
+    CSRT_SPMM_CASE(2, 1, 1, (spmm_group_kernel<2, 1>))
+    CSRT_SPMM_CASE(2, 1, 2, (spmm_group_kernel<2, 2>))
+    CSRT_SPMM_CASE(2, 1, 4, (spmm_group_kernel<2, 4>))
+    CSRT_SPMM_CASE(2, 1, 8, (spmm_group_kernel<2, 8>))
+    CSRT_SPMM_CASE(2, 1, 16, (spmm_group_kernel<2, 16>))
+    CSRT_SPMM_CASE(1, 1, 1, (spmm_group_kernel<1, 1>))
+    CSRT_SPMM_CASE(1, 1, 2, (spmm_group_kernel<1, 2>))
+    CSRT_SPMM_CASE(1, 1, 4, (spmm_group_kernel<1, 4>))
+    CSRT_SPMM_CASE(1, 1, 8, (spmm_group_kernel<1, 8>))
+    CSRT_SPMM_CASE(1, 1, 16, (spmm_group_kernel<1, 16>))
+#undef CSRT_SPMM_CASE
+    return -1;
 }
 
 static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *val, int32_t rows,
@@ -373,32 +582,28 @@ static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *
         // finish its part; more units than counters fall back to the fix-up kernel
         if ((int64_t)sh.units * sh.n_tiles <= (int64_t)kWsCounterInts) a.cnt = ws_counters(ws);
     }
-    const int64_t threads = (int64_t)sh.units * sh.n_tiles * 32;
-    const unsigned grid = (unsigned)ceil_div<int64_t>(threads, kSpThreads);
-#define CSRT_SPMM_CASE(VW, NV)                                                              \
-    if (sh.vw == VW && sh.nv == NV) {                                                       \
-        launch_pdl(spmm_merge_kernel<VW, NV>, dim3(grid), dim3(kSpThreads), 0, s, a);       \
-        count_launch();                                                                     \
-        if (sh.units > 1 && a.cnt == nullptr) {                                             \
-            const int64_t ft = (int64_t)sh.units * sh.n_tiles * 32;                         \
-            const unsigned fg = (unsigned)ceil_div<int64_t>(ft, 256);                      \
-            launch_pdl(spmm_fixup_kernel<32 * VW * NV>, dim3(fg), dim3(256), 0, s, a);      \
-            count_launch();                                                                 \
-        }                                                                                   \
-    }
-    CSRT_SPMM_CASE(4, 2)
-    else CSRT_SPMM_CASE(4, 1)
-    else CSRT_SPMM_CASE(2, 1)
-    else CSRT_SPMM_CASE(1, 1)
-#undef CSRT_SPMM_CASE
+    const int launched = spmm_dispatch(sh, a, s);
+    CSRT_ARG(launched > 0, "spmm: no kernel for shape vw=%d nv=%d g=%d", sh.vw, sh.nv, sh.g);
+    count_launch(launched);
     return check_launch("spmm_merge_kernel");
 }
 
 // ---------------------------------------------------------------------------
 // SDDMM: g[k] = <dY[i_k, :], X[j_k, :]>
 // ---------------------------------------------------------------------------
-constexpr int kSdChunk = 2048;   // columns of the n range per partial sum
-
+// Layout as in the narrow SpMM kernel: a group of G lanes (G*VW >= n, or
+// G = 32 with NV vectors per lane and the n range walked in tiles of
+// TN = 32*VW*NV) takes one stored entry, a warp step covers E = 32/G entries,
+// and U steps form a batch whose column indices are requested before the
+// previous batch is consumed. Every entry of a batch lies in one row, whose
+// dY slice stays in registers for the whole row when one tile covers n (else
+// it is reloaded once per batch and tile), so per entry only its row of X is
+// read. The U dot products of a lane are finished together: the first
+// log2(min(U, G)) butterfly steps over the group's lanes exchange halves of
+// the U partial sums (a transposed reduction), the remaining steps add one
+// value, and lane r*(G/R) of each group holds entry r's result. No partial
+// buffers: the whole n range of an entry is summed in one warp, so the
+// result does not depend on the unit split.
 struct SddmmArgs {
     const int32_t *row_ptr;
     const int32_t *col;
@@ -406,11 +611,8 @@ struct SddmmArgs {
     const float *dy;
     const float *x;
     int32_t n;
-    float *out;       // g (one chunk) or partial[chunk][capacity]
-    int64_t out_stride;
+    float *out;
     int32_t units;
-    int32_t chunks;
-    int32_t chunk_len;
 };
 
 // The row holding entry k: the largest i in [0, rows) with row_ptr[i] <= k.
@@ -418,87 +620,145 @@ __device__ __forceinline__ int row_of_entry(const int32_t *__restrict__ row_ptr,
     return (int)warp_first_false(1, rows, [&](int64_t i) { return (int64_t)__ldg(row_ptr + i) <= k; }) - 1;
 }
 
-template <int VW>
-__global__ void __launch_bounds__(kSpThreads) sddmm_kernel(SddmmArgs a) {
-    pdl_enter();
-    const int lane = threadIdx.x & 31;
-    const int64_t gw = ((int64_t)blockIdx.x * kSpThreads + threadIdx.x) >> 5;
-    if (gw >= (int64_t)a.units * a.chunks) return;
-    const int u = (int)(gw % a.units);
-    const int ch = (int)(gw / a.units);
-    const int64_t nnz = __ldg(a.row_ptr + a.rows);
-    const int64_t per = ceil_div<int64_t>(nnz, a.units);
-    const int64_t k0 = min((int64_t)u * per, nnz), k1 = min(k0 + per, nnz);
-    if (k0 >= k1) return;
-    const int nb = ch * a.chunk_len, ne = min(a.n, nb + a.chunk_len);
-    int row = row_of_entry(a.row_ptr, a.rows, k0);
-    int64_t next = __ldg(a.row_ptr + row + 1);
-    float *out = a.out + (int64_t)ch * a.out_stride;
-    for (int64_t kb = k0; kb < k1; kb += 32) {
-        const int cnt = (int)imin<int64_t>(32, k1 - kb);
-        const int my_c = lane < cnt ? __ldg(a.col + kb + lane) : 0;
-        for (int q = 0; q < cnt; q += 4) {
-            int c[4], r[4];
-            bool ok[4];
+// Sums each of the U values of a lane over the G lanes of its group. Values
+// are taken in blocks of R = min(U, G): after the call, p[b*R] of lane gl
+// holds the group's sum of value b*R + gl / (G/R).
+template <int U, int G>
+__device__ __forceinline__ void group_reduce_multi(float (&p)[U], int gl) {
+    constexpr int R = U < G ? U : G;
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int64_t k = kb + q + e;
-                ok[e] = q + e < cnt;
-                c[e] = __shfl_sync(0xffffffffu, my_c, min(q + e, cnt - 1));
-                if (ok[e]) {
-                    while (next <= k) { ++row; next = __ldg(a.row_ptr + row + 1); }
-                }
-                r[e] = row;
-            }
-            float part[4] = {0.f, 0.f, 0.f, 0.f};
-            for (int nc = nb + lane * VW; nc < ne; nc += 32 * VW) {
+    for (int b = 0; b < U / R; ++b) {
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    if (!ok[e]) continue;
-                    float xf[VW], df[VW];
-                    unpack<VW>(ldv<VW>(a.x + (int64_t)c[e] * a.n + nc), xf);
-                    unpack<VW>(ldv<VW>(a.dy + (int64_t)r[e] * a.n + nc), df);
+        for (int h = R / 2, off = G / 2; h >= 1; h >>= 1, off >>= 1) {
+            const bool upper = (gl & off) != 0;
 #pragma unroll
-                    for (int j = 0; j < VW; ++j) part[e] = fmaf(df[j], xf[j], part[e]);
-                }
-            }
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) part[e] += __shfl_xor_sync(0xffffffffu, part[e], off);
-            }
-            if (lane < 4 && ok[lane]) {
-                float pv = lane == 0 ? part[0] : lane == 1 ? part[1] : lane == 2 ? part[2] : part[3];
-                out[kb + q + lane] = pv;
+            for (int j = 0; j < h; ++j) {
+                const float lo = p[b * R + j], hi = p[b * R + j + h];
+                const float send = upper ? lo : hi;
+                const float keep = upper ? hi : lo;
+                p[b * R + j] = keep + __shfl_xor_sync(0xffffffffu, send, off);
             }
         }
+#pragma unroll
+        for (int off = G / (2 * R); off >= 1; off >>= 1) p[b * R] += __shfl_xor_sync(0xffffffffu, p[b * R], off);
     }
 }
 
-__global__ void sddmm_reduce_kernel(const int32_t *__restrict__ row_ptr, int32_t rows,
-                                    const float *__restrict__ partial, int64_t stride, int32_t chunks,
-                                    float *__restrict__ g) {
+template <int VW, int NV, int G>
+__global__ void __launch_bounds__(kSpThreads, 3) sddmm_kernel(SddmmArgs a) {
     pdl_enter();
-    const int64_t nnz = __ldg(row_ptr + rows);
-    for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < nnz; k += (int64_t)gridDim.x * blockDim.x) {
-        float s = 0.f;
-        for (int c = 0; c < chunks; ++c) s += partial[(int64_t)c * stride + k];
-        g[k] = s;
+    constexpr int E = 32 / G;
+    constexpr int U = VW * NV >= 4 ? 4 : 8;
+    constexpr int B = U * E;
+    constexpr int TN = G * VW * NV, kStride = G * VW;
+    constexpr int R = U < G ? U : G;
+    const int lane = threadIdx.x & 31, grp = lane / G, gl = lane % G;
+    const int64_t gw = ((int64_t)blockIdx.x * kSpThreads + threadIdx.x) >> 5;
+    if (gw >= (int64_t)a.units) return;
+    const int64_t nnz = __ldg(a.row_ptr + a.rows);
+    const int64_t per = ceil_div<int64_t>(nnz, a.units);
+    const int64_t k0 = min(gw * per, nnz), k1 = min(k0 + per, nnz);
+    if (k0 >= k1) return;
+    const int n_tiles = (int)ceil_div<int64_t>(a.n, TN);
+
+    int row = row_of_entry(a.row_ptr, a.rows, k0);
+    int wb = row;
+    int64_t rpl = wb + lane < a.rows ? (int64_t)__ldg(a.row_ptr + wb + lane + 1) : nnz;
+    auto row_end = [&](int r) -> int64_t {
+        if (r - wb >= 32) {
+            wb = r;
+            rpl = wb + lane < a.rows ? (int64_t)__ldg(a.row_ptr + wb + lane + 1) : nnz;
+        }
+        return __shfl_sync(0xffffffffu, rpl, r - wb);
+    };
+    float dyv[NV][VW];
+    auto load_dy = [&](int r, int tt) {
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int c = tt * TN + gl * VW + v * kStride;
+            if (c < a.n) unpack<VW>(ldv<VW>(a.dy + (int64_t)r * a.n + c), dyv[v]);
+            else {
+#pragma unroll
+                for (int e = 0; e < VW; ++e) dyv[v][e] = 0.f;
+            }
+        }
+    };
+    int cn[U];
+    auto fetch = [&](int64_t kb) {
+        const int32_t *cp = a.col + kb + grp;
+        const int lim = (int)imin<int64_t>(k1 - kb - grp, B);
+#pragma unroll
+        for (int s = 0; s < U; ++s) cn[s] = s * E < lim ? __ldg(cp + s * E) : 0;
+    };
+
+    int64_t e_row = row_end(row);
+    if (n_tiles == 1) load_dy(row, 0);
+    int64_t kb = k0;
+    fetch(kb);
+    while (kb < k1) {
+        while (e_row <= kb) {   // the row holding entry kb (empty rows are passed over)
+            ++row;
+            e_row = row_end(row);
+            if (n_tiles == 1) load_dy(row, 0);
+        }
+        int c[U];
+#pragma unroll
+        for (int s = 0; s < U; ++s) c[s] = cn[s];
+        // the batch ends at the row's end or at the unit's, whichever is first
+        const int64_t e_cur = imin<int64_t>(e_row, k1);
+        const int64_t kn = imin<int64_t>(kb + B, e_cur);
+        if (kn < k1) fetch(kn);
+        const int rem = (int)imin<int64_t>(e_cur - kb - grp, B);
+        bool ok[U];
+#pragma unroll
+        for (int s = 0; s < U; ++s) ok[s] = s * E < rem;
+        float p[U];
+#pragma unroll
+        for (int s = 0; s < U; ++s) p[s] = 0.f;
+        for (int tt = 0; tt < n_tiles; ++tt) {
+            if (n_tiles > 1) load_dy(row, tt);
+            typename Vec<VW>::T xv[U][NV];
+#pragma unroll
+            for (int s = 0; s < U; ++s)
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    const int col = tt * TN + gl * VW + v * kStride;
+                    if (ok[s] && col < a.n) xv[s][v] = ldv<VW>(a.x + (int64_t)c[s] * a.n + col);
+                }
+#pragma unroll
+            for (int s = 0; s < U; ++s)
+#pragma unroll
+                for (int v = 0; v < NV; ++v) {
+                    const int col = tt * TN + gl * VW + v * kStride;
+                    if (ok[s] && col < a.n) {
+                        float f[VW];
+                        unpack<VW>(xv[s][v], f);
+#pragma unroll
+                        for (int e = 0; e < VW; ++e) p[s] = fmaf(dyv[v][e], f[e], p[s]);
+                    }
+                }
+        }
+        float *op = a.out + kb + grp;
+        if constexpr (G == 1) {
+#pragma unroll
+            for (int s = 0; s < U; ++s)
+                if (ok[s]) op[s * E] = p[s];
+        } else {
+            group_reduce_multi<U, G>(p, gl);
+            if (gl % (G / R) == 0) {
+                const int r = gl / (G / R);
+#pragma unroll
+                for (int b = 0; b < U / R; ++b) {
+                    const int s = b * R + r;
+                    if (s * E < rem) op[s * E] = p[b * R];
+                }
+            }
+        }
+        kb = kn;
     }
 }
 
-static int sddmm_chunks(int64_t capacity, int32_t n) {
-    if (n <= kSdChunk) return 1;
-    const int64_t want = ceil_div<int64_t>(n, kSdChunk);
-    const int64_t room = imax<int64_t>(1, ((int64_t)1 << 22) / imax<int64_t>(1, capacity));
-    return (int)min(want, room);
-}
-
-size_t sddmm_scratch_bytes(int64_t capacity, int32_t max_n) {
-    const int chunks = sddmm_chunks(capacity, max_n);
-    if (chunks <= 1) return 0;
-    return (size_t)chunks * (size_t)capacity * sizeof(float) + 256;
-}
+size_t sddmm_scratch_bytes(int64_t, int32_t) { return 0; }
 
 }  // namespace csrt
 
@@ -570,7 +830,10 @@ int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_
     }
     CSRT_ARG(dy && x, "dY or X is NULL");
     const bool v4 = (n % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(dy)) & 15) == 0;
-    const int chunks = sddmm_chunks(w->capacity, n);
+    const bool v2 = (n % 2 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(dy)) & 7) == 0;
+    const int vw = v4 ? 4 : v2 ? 2 : 1;
+    const int g = imin(32, pow2_at_least((n + vw - 1) / vw));
+    const int nv = g == 32 && n > 32 * vw ? 2 : 1;
     SddmmArgs a;
     a.row_ptr = w->row_ptr;
     a.col = w->col_idx;
@@ -578,30 +841,35 @@ int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_
     a.dy = dy;
     a.x = x;
     a.n = n;
-    a.chunks = chunks;
-    a.chunk_len = chunks > 1 ? (int)ceil_div<int64_t>(n, chunks) : n;
-    if (v4 && chunks > 1) a.chunk_len = (a.chunk_len + 3) / 4 * 4;
-    const int64_t target = (int64_t)num_sms() * kWarpsPerSM;
-    a.units = (int)imax<int64_t>(1, imin<int64_t>(ceil_div<int64_t>(target, chunks), w->capacity));
-    if (chunks > 1) {
-        CSRT_ARG(ws != nullptr && ws_bytes >= kWsReservedBytes + sddmm_scratch_bytes(w->capacity, n),
-                 "workspace too small for sddmm");
-        a.out = reinterpret_cast<float *>(ws_scratch(ws));
-        a.out_stride = w->capacity;
-    } else {
-        a.out = g_nnz;
-        a.out_stride = 0;
+    a.out = g_nnz;
+    static int cache[64][3][6][2];
+    int dev = 0;
+    CSRT_CHECK_CUDA(cudaGetDevice(&dev));
+    CSRT_ARG(dev >= 0 && dev < 64, "device ordinal %d out of range", dev);
+    int lg = 0;
+    while ((1 << lg) < g) ++lg;
+    int &wps = cache[dev][vw == 4 ? 2 : vw - 1][lg][nv - 1];
+    void (*kern)(SddmmArgs) = nullptr;
+#define CSRT_SDDMM_CASE(VW, NV, G) \
+    if (vw == VW && nv == NV && g == G) kern = sddmm_kernel<VW, NV, G>;
+    CSRT_SDDMM_CASE(4, 1, 1) CSRT_SDDMM_CASE(4, 1, 2) CSRT_SDDMM_CASE(4, 1, 4) CSRT_SDDMM_CASE(4, 1, 8)
+    CSRT_SDDMM_CASE(4, 1, 16) CSRT_SDDMM_CASE(4, 1, 32) CSRT_SDDMM_CASE(4, 2, 32)
+    CSRT_SDDMM_CASE(2, 1, 1) CSRT_SDDMM_CASE(2, 1, 2) CSRT_SDDMM_CASE(2, 1, 4) CSRT_SDDMM_CASE(2, 1, 8)
+    CSRT_SDDMM_CASE(2, 1, 16) CSRT_SDDMM_CASE(2, 1, 32) CSRT_SDDMM_CASE(2, 2, 32)
+    CSRT_SDDMM_CASE(1, 1, 1) CSRT_SDDMM_CASE(1, 1, 2) CSRT_SDDMM_CASE(1, 1, 4) CSRT_SDDMM_CASE(1, 1, 8)
+    CSRT_SDDMM_CASE(1, 1, 16) CSRT_SDDMM_CASE(1, 1, 32) CSRT_SDDMM_CASE(1, 2, 32)
+#undef CSRT_SDDMM_CASE
+    CSRT_ARG(kern != nullptr, "sddmm: no kernel for vw=%d nv=%d g=%d", vw, nv, g);
+    if (wps == 0) {
+        int blocks = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kern, kSpThreads, 0) != cudaSuccess || blocks <= 0)
+            blocks = kWarpsPerSM / (kSpThreads / 32);
+        wps = imin(blocks * (kSpThreads / 32), kWarpsPerSM);
     }
-    const unsigned grid = (unsigned)ceil_div<int64_t>((int64_t)a.units * chunks * 32, kSpThreads);
-    if (v4) launch_pdl(sddmm_kernel<4>, dim3(grid), dim3(kSpThreads), 0, s, a);
-    else launch_pdl(sddmm_kernel<1>, dim3(grid), dim3(kSpThreads), 0, s, a);
+    a.units = (int)imax<int64_t>(1, imin<int64_t>((int64_t)num_sms() * wps, w->capacity));
+    const unsigned grid = (unsigned)ceil_div<int64_t>((int64_t)a.units * 32, kSpThreads);
+    launch_pdl(kern, dim3(grid), dim3(kSpThreads), 0, s, a);
     count_launch();
-    if (chunks > 1) {
-        const unsigned rg = (unsigned)imin<int64_t>(ceil_div<int64_t>(w->capacity, 256), (int64_t)num_sms() * 8);
-        launch_pdl(sddmm_reduce_kernel, dim3(rg), dim3(256), 0, s, w->row_ptr, w->rows, a.out, a.out_stride, chunks,
-                   g_nnz);
-        count_launch();
-    }
     return check_launch("sddmm_kernel");
 }
 
@@ -712,22 +980,8 @@ extern "C" int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, fl
     a.bias = nullptr;
     a.relu = 0;
     a.mask = nullptr;
-    cudaStream_t s = as_stream(stream);
-    const unsigned grid = (unsigned)ceil_div<int64_t>((int64_t)sh.units * sh.n_tiles * 32, kSpThreads);
-    const unsigned fgrid = (unsigned)ceil_div<int64_t>((int64_t)sh.units * sh.n_tiles * 32, 256);
-    if (sh.vw == 4 && sh.nv == 2) {
-        launch_pdl(spmm_merge_kernel<4, 2>, dim3(grid), dim3(kSpThreads), 0, s, a);
-        if (sh.units > 1) launch_pdl(spmm_fixup_kernel<256>, dim3(fgrid), dim3(256), 0, s, a);
-    } else if (sh.vw == 4) {
-        launch_pdl(spmm_merge_kernel<4, 1>, dim3(grid), dim3(kSpThreads), 0, s, a);
-        if (sh.units > 1) launch_pdl(spmm_fixup_kernel<128>, dim3(fgrid), dim3(256), 0, s, a);
-    } else if (sh.vw == 2) {
-        launch_pdl(spmm_merge_kernel<2, 1>, dim3(grid), dim3(kSpThreads), 0, s, a);
-        if (sh.units > 1) launch_pdl(spmm_fixup_kernel<64>, dim3(fgrid), dim3(256), 0, s, a);
-    } else {
-        launch_pdl(spmm_merge_kernel<1, 1>, dim3(grid), dim3(kSpThreads), 0, s, a);
-        if (sh.units > 1) launch_pdl(spmm_fixup_kernel<32>, dim3(fgrid), dim3(256), 0, s, a);
-    }
-    count_launch(sh.units > 1 ? 2 : 1);
+    const int launched = spmm_dispatch(sh, a, as_stream(stream));
+    CSRT_ARG(launched > 0, "spmm_fwd_noalloc: no kernel for shape vw=%d nv=%d g=%d", sh.vw, sh.nv, sh.g);
+    count_launch(launched);
     return check_launch("spmm_fwd_noalloc");
 }

@@ -165,6 +165,23 @@ SPMM_CASES = [
     (4100, 700, 256, 0.05, False),
     (7400, 257, 128, 0.2, True),
     (300, 9000, 256, 0.05, False),
+    # narrow products (G lanes per nonzero, G*VW >= n): every group width and
+    # vector width, rows of thousands of entries cut by many units, power-law
+    # rows, empty rows, and tails shorter than one batch
+    (64, 20000, 1, 0.5, False),
+    (2000, 3000, 1, 0.05, True),
+    (1500, 1100, 2, 0.2, False),
+    (700, 900, 3, 0.1, True),
+    (300, 5000, 4, 0.3, False),
+    (257, 700, 5, 0.2, False),
+    (400, 2500, 8, 0.4, True),
+    (129, 257, 12, 0.2, False),
+    (600, 4000, 16, 0.1, False),
+    (300, 800, 24, 0.3, True),
+    (129, 4000, 32, 0.5, False),
+    (1000, 600, 48, 0.1, True),
+    (300, 2000, 64, 0.2, False),
+    (90, 70, 9, 0.0, False),
 ]
 
 
@@ -218,7 +235,7 @@ def test_fused_epilogues_match_unfused(C, m, k, n, zipf):
     np.testing.assert_array_equal(dx.cpu().numpy().view(np.uint32), dx_ref.cpu().numpy().view(np.uint32))
 
 
-@pytest.mark.parametrize("n", [96, 256])
+@pytest.mark.parametrize("n", [1, 8, 32, 96, 256])
 def test_spmm_is_deterministic(C, n):
     rng = np.random.default_rng(11)
     a = _sparse(rng, 700, 900, 0.08, zipf=True)
@@ -254,7 +271,15 @@ def test_weight_grad_dense(C, m, k, n, prec):
 
 @pytest.mark.parametrize("m,k,n,density,zipf", [(300, 784, 64, 0.1, False), (100, 300, 256, 0.09, True),
                                                 (20, 25, 9000, 0.3, False), (50, 40, 1, 0.5, False),
-                                                (33, 17, 5, 0.0, False)])
+                                                (33, 17, 5, 0.0, False),
+                                                # every group width, float4 / float2 / scalar rows of X,
+                                                # long and power-law rows, n walked in several tiles
+                                                (64, 20000, 1, 0.5, False), (2000, 3000, 1, 0.05, True),
+                                                (700, 900, 2, 0.1, True), (300, 5000, 3, 0.2, False),
+                                                (400, 2500, 8, 0.3, True), (129, 4000, 32, 0.5, False),
+                                                (300, 900, 33, 0.2, False), (257, 700, 64, 0.2, True),
+                                                (300, 800, 130, 0.1, False), (500, 3000, 256, 0.05, True),
+                                                (100, 300, 1024, 0.2, False), (60, 90, 1030, 0.3, True)])
 def test_weight_grad_sddmm(C, m, k, n, density, zipf):
     rng = np.random.default_rng(m * k + n)
     a = _sparse(rng, m, k, density, zipf)

@@ -28,7 +28,8 @@ def test_noalloc_matches_spmm_fwd_on_two_calls():
 
     lib = C.lib()
     stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
-    for (m, k, n, zipf) in [(700, 900, 96, True), (300, 784, 256, False)]:
+    for (m, k, n, zipf) in [(700, 900, 96, True), (300, 784, 256, False), (64, 20000, 1, False),
+                            (700, 900, 32, True)]:
         rng = np.random.default_rng(m + n)
         w = synth.masked_weights(rng, m, k, 0.1, zipf=zipf)
         ws = C.Workspace(m, k, n)
