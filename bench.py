@@ -59,6 +59,9 @@ def parse_args():
     p.add_argument("--prox-path", choices=["fused", "unfused"], default="fused",
                    help="fused: weight gradient and prox update in one tensor-core pass (G not written)")
     p.add_argument("--profile-ops", action="store_true", help="print the per-operation breakdown to stderr")
+    p.add_argument("--record-traffic", metavar="CSV",
+                   help="write profiles/traffic.json from an ncu CSV of this bench (dram__bytes_read.sum, "
+                        "dram__bytes_write.sum, gpu__time_duration.sum; --steps 1 --warmup 1) and exit")
     p.add_argument("--optimizer", choices=["sgd", "rmsprop", "adam"], default="sgd",
                    help="proximal method of the prox phase: SGD, Prox-RMSProp (Algorithm 1) or Prox-ADAM "
                         "(Algorithm 2); the adaptive ones take the unfused gradient + prox calls")
@@ -300,6 +303,69 @@ def op_bytes(name, info):
     return None
 
 
+# Kernels of one weight_grad_prox_update call: it starts with fp_oldbits_kernel
+# and runs on through these (the transposed copy included when built).
+FUSED_OP_KERNELS = ("fp_oldbits_kernel", "gemm_prox_tc_kernel", "fp_rowscan_kernel", "scan_clamped_kernel",
+                    "scan_single_block_kernel", "fp_finish_kernel", "trb_count_kernel", "tr_colscan_kernel",
+                    "trb_write_kernel")
+FUSED_OP_SOURCES = ["fused_prox.cu", "compact.cu", "tc_common.cuh", "common.cuh"]
+
+
+def record_traffic(csv_path: str, out_path: str) -> dict:
+    """profiles/traffic.json from an ncu CSV of `bench.py --steps 1 --warmup 1`:
+    per fused gradient + prox call of the second eager step (the instrumented
+    one), the DRAM bytes and serialised time summed over its kernels. The
+    step's calls run layer 2, layer 1, layer 0."""
+    import csv
+    launches = {}
+    with open(csv_path) as f:
+        rows = [r for r in csv.reader(f)]
+    hdr = next(i for i, r in enumerate(rows) if r and r[0] == "ID")
+    cols = rows[hdr]
+    for r in rows[hdr + 1:]:
+        if len(r) != len(cols):
+            continue
+        d = dict(zip(cols, r))
+        k = launches.setdefault(int(d["ID"]), {"name": d["Kernel Name"]})
+        try:
+            k[d["Metric Name"]] = float(d["Metric Value"].replace(",", ""))
+        except ValueError:
+            pass
+    seq = [launches[i] for i in sorted(launches)]
+    calls, i = [], 0
+    while i < len(seq):
+        if seq[i]["name"].split("(")[0].split("::")[-1].startswith("fp_oldbits_kernel"):
+            j = i + 1
+            while j < len(seq) and any(n in seq[j]["name"] for n in FUSED_OP_KERNELS[1:]):
+                j += 1
+            calls.append(seq[i:j])
+            i = j
+        else:
+            i += 1
+    if len(calls) < 6:
+        raise SystemExit(f"record-traffic: found {len(calls)} fused calls, need the 3 of two eager steps")
+    rec = {"_about": "DRAM bytes (read + write) of one call of each fused weight-gradient + prox op of the "
+                     "classifier-head step, summed over the op's kernels (second eager step of the run), from: ncu "
+                     "--metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum --clock-control "
+                     "none --csv --log-file bench_dram.csv python bench.py --steps 1 --warmup 1 --no-cpu-baseline, "
+                     "then python bench.py --record-traffic bench_dram.csv. ncu flushes the caches between kernels, "
+                     "so output lines still dirty in L2 when a kernel ends are not counted: an op whose output fits "
+                     "in L2 shows fewer bytes than it writes."}
+    for layer, call in zip((2, 1, 0), calls[3:6]):
+        rd = sum(k.get("dram__bytes_read.sum", 0.0) for k in call)
+        wr = sum(k.get("dram__bytes_write.sum", 0.0) for k in call)
+        us = sum(k.get("gpu__time_duration.sum", 0.0) for k in call) / 1e3
+        rec[f"weight_grad_prox_update[layer {layer}]"] = {
+            "dram_bytes_per_call": int(rd + wr), "dram_read": int(rd), "dram_write": int(wr),
+            "ncu_us_serialised": round(us, 1),
+            "kernels": [k["name"].split("(")[0].replace("csrt::", "").replace("void ", "") for k in call],
+            "sources": FUSED_OP_SOURCES, "sha256_16": source_digest(FUSED_OP_SOURCES)}
+    with open(out_path, "w") as f:
+        json.dump(rec, f, indent=1)
+        f.write("\n")
+    return rec
+
+
 # ---------------------------------------------------------------------------
 # Multi-rank bookkeeping (replicas: no collective on the data path)
 # ---------------------------------------------------------------------------
@@ -325,6 +391,10 @@ def whole_job_rate(units_per_rank_per_step: int, steps: int, world: int, max_tot
 
 def main():
     args = parse_args()
+    if args.record_traffic:
+        rec = record_traffic(args.record_traffic, os.path.join(ROOT, "profiles", "traffic.json"))
+        print(json.dumps({k: v["dram_bytes_per_call"] for k, v in rec.items() if k != "_about"}))
+        return 0
     if args.impl == "reference":
         return run_reference(args)
     rank, world, local_rank = dist_env()

@@ -331,6 +331,9 @@ def test_prox_hand_cases_on_gpu(C):
     (333, 64, 0.4, 1.0, 0.1, 1.0),
     (3, 16384, 0.02, 1.0, 0.01, 0.5),
     (2, 16388, 0.02, 1.0, 0.01, 0.5),
+    (2, 20000, 0.3, 1.0, 0.01, 0.5),
+    (4100, 512, 0.05, 1.0, 0.01, 1e-4),
+    (700, 900, 0.5, 0.1, 0.1, 1.0),
 ])
 def test_prox_bit_exact(C, m, k, density, gscale, eta, lam):
     rng = np.random.default_rng(m + k)
@@ -415,6 +418,30 @@ def test_fused_gradient_prox_fallback_needs_scratch(C):
     (rp, ci, v), _ = out.to_host()
     np.testing.assert_array_equal(ci, ref.col_idx)
     np.testing.assert_array_equal(v.view(np.uint32), ref.val.view(np.uint32))
+
+
+@pytest.mark.parametrize("m,k,transposed", [(256, 512, False), (256, 512, True), (300, 300, False),
+                                            (129, 4100, True)])
+def test_prox_capacity_overflow(C, m, k, transposed):
+    """An output CSR too small for the prox result: the overflow and the needed
+    nnz are reported, the row pointers are clamped and the stored prefix is the
+    oracle's."""
+    rng = np.random.default_rng(m + k + transposed)
+    a = _sparse(rng, m, k, 0.2)
+    g = rng.standard_normal((m, k)).astype(F32)
+    ws = _ws(C, m, k, 1)
+    w = _gpu_csr(C, a, ws, transposed=False)
+    ref = O.prox_update_compact(O.csr_from_dense(a), g, 0.5, 0.5)
+    cap = ref.nnz // 3
+    out = C.CSR(m, k, capacity=cap, transposed=transposed)
+    C.prox_update_compact(w, _dev(g), 0.5, 0.5, out, ws)
+    flags, required = ws.status()
+    assert flags & C.CSRT_DEV_CAPACITY and required == ref.nnz
+    rp = out.row_ptr.cpu().numpy()
+    np.testing.assert_array_equal(rp, np.minimum(ref.row_ptr, cap))
+    np.testing.assert_array_equal(out.col_idx.cpu().numpy()[:cap], ref.col_idx[:cap])
+    np.testing.assert_array_equal(out.val.cpu().numpy()[:cap].view(np.uint32), ref.val[:cap].view(np.uint32))
+    ws.clear_status()
 
 
 def test_prox_nan_is_dropped_and_flagged(C):
