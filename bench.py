@@ -344,13 +344,28 @@ def record_traffic(csv_path: str, out_path: str) -> dict:
             i += 1
     if len(calls) < 6:
         raise SystemExit(f"record-traffic: found {len(calls)} fused calls, need the 3 of two eager steps")
-    rec = {"_about": "DRAM bytes (read + write) of one call of each fused weight-gradient + prox op of the "
-                     "classifier-head step, summed over the op's kernels (second eager step of the run), from: ncu "
+    pending = {}
+    rec = {"_about": "DRAM bytes (read + write) of one call of each fused weight-gradient + prox op and each "
+                     "sparse product of the classifier-head step, summed over the op's kernels (second eager step "
+                     "of the run), from: ncu "
                      "--metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum --clock-control "
                      "none --csv --log-file bench_dram.csv python bench.py --steps 1 --warmup 1 --no-cpu-baseline, "
                      "then python bench.py --record-traffic bench_dram.csv. ncu flushes the caches between kernels, "
                      "so output lines still dirty in L2 when a kernel ends are not counted: an op whose output fits "
                      "in L2 shows fewer bytes than it writes."}
+    # the step's sparse products, in call order: forward layers 0, 1, 2, then
+    # the backward products of layers 2 and 1 (second eager step)
+    sp = [k for k in seq if "spmm_merge_kernel" in k["name"] or "spmm_group_kernel" in k["name"]]
+    if len(sp) >= 10:
+        labels = ["spmm_fwd_bias_act[layer 0]", "spmm_fwd_bias_act[layer 1]", "spmm_fwd_bias_act[layer 2]",
+                  "spmm_bwd_t_relu[layer 2]", "spmm_bwd_t_relu[layer 1]"]
+        srcs = ["spmm.cu", "common.cuh"]
+        for lab, k in zip(labels, sp[5:10]):
+            rd, wr = k.get("dram__bytes_read.sum", 0.0), k.get("dram__bytes_write.sum", 0.0)
+            pending[lab] = {"dram_bytes_per_call": int(rd + wr), "dram_read": int(rd), "dram_write": int(wr),
+                            "ncu_us_serialised": round(k.get("gpu__time_duration.sum", 0.0) / 1e3, 1),
+                            "kernels": [k["name"].split("(")[0].replace("csrt::", "").replace("void ", "")],
+                            "sources": srcs, "sha256_16": source_digest(srcs)}
     for layer, call in zip((2, 1, 0), calls[3:6]):
         rd = sum(k.get("dram__bytes_read.sum", 0.0) for k in call)
         wr = sum(k.get("dram__bytes_write.sum", 0.0) for k in call)
@@ -360,6 +375,7 @@ def record_traffic(csv_path: str, out_path: str) -> dict:
             "ncu_us_serialised": round(us, 1),
             "kernels": [k["name"].split("(")[0].replace("csrt::", "").replace("void ", "") for k in call],
             "sources": FUSED_OP_SOURCES, "sha256_16": source_digest(FUSED_OP_SOURCES)}
+    rec.update(pending)
     with open(out_path, "w") as f:
         json.dump(rec, f, indent=1)
         f.write("\n")
@@ -517,6 +533,15 @@ def main():
                       "frac": round(bytes_ / t_s / 1e9 / hbm, 4),
                       "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)" if peak_kind == "measured"
                       else "fallback 6.8 TB/s"})
+    if dom["name"] in ("spmm_fwd", "spmm_bwd_t", "spmm_fwd_bias_act", "spmm_bwd_t_relu") and dom["info"].get("n"):
+        # a product on the FP32 CUDA cores (no tensor cores for the sparse
+        # operand): 2*nnz*n flops against the FMA rate measured by the
+        # library's probe on this GPU (nominal 152 SMs x 128 lanes x 2 x clock)
+        flops = 2.0 * dom["info"]["nnz"] * dom["info"]["n"]
+        peak = C.fma_peak_tflops()
+        cands.append({"bound": "alu", "achieved": round(flops / t_s / 1e12, 2), "peak": round(peak, 1),
+                      "unit": "TFLOP/s", "frac": round(flops / t_s / 1e12 / peak, 4),
+                      "peak_source": "measured FP32 FMA rate (library probe, fma_peak_kernel)"})
     if dom["name"] in ("weight_grad_dense", "weight_grad_prox_update") and dom["info"].get("n"):
         # a TF32 contraction: its peak is the measured bf16 rate x the nominal tf32/bf16 ratio (1.1 / 2.25);
         # algorithmic flops 2MKN (the fused op's second pass recomputes them: not counted)
