@@ -281,6 +281,17 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_merge_kernel(SpmmArgs a) {
 // spmm_merge_kernel (carries of TN = G*VW floats).
 // ---------------------------------------------------------------------------
 template <int VW> struct NarrowSteps { static constexpr int value = VW == 1 ? 8 : 4; };
+constexpr int kNarrowChunk = 256;   // entries per ring chunk
+constexpr int kNarrowStages = 3;    // ring chunks per warp
+constexpr int kNarrowSmem = (kSpThreads / 32) * 2 * kNarrowStages * kNarrowChunk * (int)sizeof(int32_t);
+
+__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 template <int VW, int G>
 __global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
@@ -321,19 +332,6 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
     float acc[VW];
 #pragma unroll
     for (int e = 0; e < VW; ++e) acc[e] = 0.f;
-    int cn[U];
-    float wn[U];
-    auto fetch = [&](int64_t kb) {
-        const int32_t *cp = a.col + kb + grp;
-        const float *vp = a.val + kb + grp;
-        const int lim = (int)imin<int64_t>(k1 - kb - grp, B);
-#pragma unroll
-        for (int s = 0; s < U; ++s) {
-            const bool ok = s * E < lim;
-            cn[s] = ok ? __ldg(cp + s * E) : 0;
-            wn[s] = ok ? __ldg(vp + s * E) : 0.f;
-        }
-    };
     // the groups' partial sums of one row, summed over the lane bits above G
     auto combine = [&](float (&v)[VW]) {
 #pragma unroll
@@ -348,10 +346,8 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
     int i = i0;
     int64_t e_row = row_end(i);
     int64_t kr = k0;   // first entry of the current row inside this unit
-    int64_t kb = k0;
-    if (kb < k1) fetch(kb);
-    for (;;) {
-        while (i < i1 && e_row <= kb) {   // rows that end here are complete
+    auto finish_rows = [&](int64_t kb) {   // rows that end at or before kb are complete
+        while (i < i1 && e_row <= kb) {
             float v[VW];
             combine(v);
             if (grp == 0 && in_n) {
@@ -362,30 +358,114 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
             ++i;
             e_row = row_end(i);
         }
-        if (kb >= k1) break;
-        int c[U];
-        float w[U];
+    };
+    if constexpr (G == 1) {
+        // one nonzero per lane: the indices and values of the next batch are
+        // loaded into registers while the current batch is consumed (the
+        // instructions of a shared-memory ring cost more than they hide here)
+        int cn[U];
+        float wn[U];
+        auto fetch = [&](int64_t kb) {
+            const int32_t *cp = a.col + kb + lane;
+            const float *vp = a.val + kb + lane;
+            const int lim = (int)imin<int64_t>(k1 - kb - lane, B);
 #pragma unroll
-        for (int s = 0; s < U; ++s) {
-            c[s] = cn[s];
-            w[s] = wn[s];
-        }
-        const int64_t kn = imin<int64_t>(kb + B, e_row);
-        const int rem = in_n ? (int)imin<int64_t>(e_row - kb - grp, B) : 0;
-        if (kn < k1) fetch(kn);
-        typename Vec<VW>::T xv[U];
-#pragma unroll
-        for (int s = 0; s < U; ++s)
-            if (s * E < rem) xv[s] = ldv<VW>(a.x + (int64_t)c[s] * a.n + c0);
-#pragma unroll
-        for (int s = 0; s < U; ++s)
-            if (s * E < rem) {
-                float f[VW];
-                unpack<VW>(xv[s], f);
-#pragma unroll
-                for (int e = 0; e < VW; ++e) acc[e] = fmaf(w[s], f[e], acc[e]);
+            for (int st = 0; st < U; ++st) {
+                const bool ok = st * 32 < lim;
+                cn[st] = ok ? __ldg(cp + st * 32) : 0;
+                wn[st] = ok ? __ldg(vp + st * 32) : 0.f;
             }
-        kb = kn;
+        };
+        int64_t kb = k0;
+        if (kb < k1) fetch(kb);
+        while (true) {
+            finish_rows(kb);
+            if (kb >= k1) break;
+            int c[U];
+            float w[U];
+#pragma unroll
+            for (int st = 0; st < U; ++st) {
+                c[st] = cn[st];
+                w[st] = wn[st];
+            }
+            const int64_t kn = imin<int64_t>(kb + B, e_row);
+            const int rem = in_n ? (int)imin<int64_t>(e_row - kb - lane, B) : 0;
+            if (kn < k1) fetch(kn);
+            typename Vec<VW>::T xv[U];
+#pragma unroll
+            for (int st = 0; st < U; ++st)
+                if (st * 32 < rem) xv[st] = ldv<VW>(a.x + (int64_t)c[st] * a.n + c0);
+#pragma unroll
+            for (int st = 0; st < U; ++st)
+                if (st * 32 < rem) {
+                    float f[VW];
+                    unpack<VW>(xv[st], f);
+#pragma unroll
+                    for (int e = 0; e < VW; ++e) acc[e] = fmaf(w[st], f[e], acc[e]);
+                }
+            kb = kn;
+        }
+    } else {
+    // The unit's column indices and values stream through a ring of
+    // kNarrowStages chunks of kNarrowChunk entries in shared memory (this
+    // warp's slice), copied with cp.async kNarrowStages - 1 chunks ahead of
+    // the one being consumed, so the loads in flight cost no registers.
+    extern __shared__ __align__(16) int32_t narrow_smem[];
+    int32_t *ring_c = narrow_smem + (threadIdx.x >> 5) * (2 * kNarrowStages * kNarrowChunk);
+    float *ring_v = reinterpret_cast<float *>(ring_c + kNarrowStages * kNarrowChunk);
+    auto issue = [&](int64_t cs) {   // chunk starting at entry cs into its ring slot (an empty group past k1)
+        if (cs < k1) {
+            const int slot = (int)(((cs - k0) / kNarrowChunk) % kNarrowStages) * kNarrowChunk;
+#pragma unroll
+            for (int q = 0; q < kNarrowChunk / 32; ++q) {
+                const int64_t idx = cs + q * 32 + lane;
+                if (idx < k1) {
+                    cp_async4(ring_c + slot + q * 32 + lane, a.col + idx);
+                    cp_async4(ring_v + slot + q * 32 + lane, a.val + idx);
+                }
+            }
+        }
+        cp_async_commit();
+    };
+#pragma unroll
+    for (int q = 0; q < kNarrowStages - 1; ++q) issue(k0 + (int64_t)q * kNarrowChunk);
+    for (int64_t cs = k0; cs < k1; cs += kNarrowChunk) {
+        issue(cs + (int64_t)(kNarrowStages - 1) * kNarrowChunk);
+        cp_async_wait<kNarrowStages - 1>();
+        __syncwarp();
+        const int slot = (int)(((cs - k0) / kNarrowChunk) % kNarrowStages) * kNarrowChunk;
+        const int64_t ce = imin<int64_t>(cs + kNarrowChunk, k1);
+        for (int64_t kb = cs; kb < ce;) {
+            finish_rows(kb);
+            const int64_t kn = imin<int64_t>(imin<int64_t>(kb + B, e_row), ce);
+            const int rem = in_n ? (int)(kn - kb - grp) : 0;
+            const int off = slot + (int)(kb - cs) + grp;
+            int c[U];
+            float w[U];
+#pragma unroll
+            for (int st = 0; st < U; ++st)
+                if (st * E < rem) {
+                    c[st] = ring_c[off + st * E];
+                    w[st] = ring_v[off + st * E];
+                }
+            typename Vec<VW>::T xv[U];
+#pragma unroll
+            for (int st = 0; st < U; ++st)
+                if (st * E < rem) xv[st] = ldv<VW>(a.x + (int64_t)c[st] * a.n + c0);
+#pragma unroll
+            for (int st = 0; st < U; ++st)
+                if (st * E < rem) {
+                    float f[VW];
+                    unpack<VW>(xv[st], f);
+#pragma unroll
+                    for (int e = 0; e < VW; ++e) acc[e] = fmaf(w[st], f[e], acc[e]);
+                }
+            kb = kn;
+        }
+        __syncwarp();   // the slot is read before the copy issued next refills it
+    }
+    cp_async_wait<0>();
+    finish_rows(k1);
     }
     // the unit ends inside row i1: its part is a carry
     const bool has_carry = k1 > kr;
@@ -448,12 +528,12 @@ struct SpmmShape {
 };
 
 template <typename K>
-static int kernel_warps_per_sm(K kernel, int (&cache)[64], int cap) {
+static int kernel_warps_per_sm(K kernel, int (&cache)[64], int cap, size_t smem = 0) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cap;
     if (cache[dev] == 0) {
         int blocks = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kernel, kSpThreads, 0) != cudaSuccess ||
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kernel, kSpThreads, smem) != cudaSuccess ||
             blocks <= 0)
             blocks = cap / (kSpThreads / 32);
         cache[dev] = imin(blocks * (kSpThreads / 32), cap);
@@ -465,7 +545,7 @@ template <int VW, int NV, int G>
 static int spmm_warps_per_sm() {
     static int cache[64] = {0};
     if constexpr (G == 32) return kernel_warps_per_sm(spmm_merge_kernel<VW, NV>, cache, kWarpsPerSM);
-    else return kernel_warps_per_sm(spmm_group_kernel<VW, G>, cache, kWarpsPerSM);
+    else return kernel_warps_per_sm(spmm_group_kernel<VW, G>, cache, kWarpsPerSM, G > 1 ? (size_t)kNarrowSmem : 0);
 }
 
 static int pow2_at_least(int v) {
@@ -523,7 +603,7 @@ static int spmm_dispatch(const SpmmShape &sh, const SpmmArgs &a, cudaStream_t s)
     const unsigned fg = (unsigned)ceil_div<int64_t>(threads, 256);
 #define CSRT_SPMM_CASE(VW, NV, G, KERNEL)                                                   \
     if (sh.vw == VW && sh.nv == NV && sh.g == G) {                                          \
-        launch_pdl(KERNEL, dim3(grid), dim3(kSpThreads), 0, s, a);                          \
+        launch_pdl(KERNEL, dim3(grid), dim3(kSpThreads), (G > 1 && G < 32) ? (size_t)kNarrowSmem : 0, s, a); \
         if (fix) launch_pdl(spmm_fixup_kernel<G * VW * NV>, dim3(fg), dim3(256), 0, s, a); \
         return fix ? 2 : 1;                                                                 \
     }

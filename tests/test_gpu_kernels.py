@@ -182,6 +182,15 @@ SPMM_CASES = [
     (1000, 600, 48, 0.1, True),
     (300, 2000, 64, 0.2, False),
     (90, 70, 9, 0.0, False),
+    # row-tiled wide products (n % 64 == 0, >= 2432 rows at n = 256, density
+    # >= 1/32): power-law rows (the long ones left to the long-row kernel),
+    # a partial last chunk of X rows, n = 1024 and 128, and a product just
+    # below the density threshold (taken by the merge-path kernels)
+    (2600, 300, 256, 0.2, True),
+    (5000, 600, 128, 0.3, True),
+    (2500, 2000, 256, 0.04, False),
+    (2500, 500, 256, 0.02, False),
+    (2432, 130, 1024, 0.3, False),
 ]
 
 
@@ -210,7 +219,7 @@ def test_spmm_fwd_and_bwd_against_oracle(C, m, k, n, density, zipf):
 
 
 @pytest.mark.parametrize("m,k,n,zipf", [(700, 900, 256, True), (129, 257, 70, False), (50, 40, 1, False),
-                                         (300, 784, 64, False), (4100, 4100, 256, False)])
+                                         (300, 784, 64, False), (4100, 4100, 256, False), (5000, 5000, 128, True)])
 def test_fused_epilogues_match_unfused(C, m, k, n, zipf):
     rng = np.random.default_rng(m + k + n)
     a = _sparse(rng, m, k, 0.1, zipf)
@@ -235,16 +244,17 @@ def test_fused_epilogues_match_unfused(C, m, k, n, zipf):
     np.testing.assert_array_equal(dx.cpu().numpy().view(np.uint32), dx_ref.cpu().numpy().view(np.uint32))
 
 
-@pytest.mark.parametrize("n", [1, 8, 32, 96, 256])
-def test_spmm_is_deterministic(C, n):
+@pytest.mark.parametrize("m,k,n", [(700, 900, 1), (700, 900, 8), (700, 900, 32), (700, 900, 96), (700, 900, 256),
+                                   (5000, 900, 256)])
+def test_spmm_is_deterministic(C, m, k, n):
     rng = np.random.default_rng(11)
-    a = _sparse(rng, 700, 900, 0.08, zipf=True)
-    x = _dev(rng.standard_normal((900, n)).astype(F32))
-    ws = _ws(C, 900, 900, n)
+    a = _sparse(rng, m, k, 0.08, zipf=True)
+    x = _dev(rng.standard_normal((k, n)).astype(F32))
+    ws = _ws(C, m, k, n)
     w = _gpu_csr(C, a, ws)
     ys = []
     for _ in range(3):
-        y = torch.zeros(700, n, device="cuda")
+        y = torch.zeros(m, n, device="cuda")
         C.spmm_fwd(w, x, y, ws)
         ys.append(y.cpu().numpy())
     np.testing.assert_array_equal(ys[0].view(np.uint32), ys[1].view(np.uint32))
