@@ -773,6 +773,86 @@ __global__ void __launch_bounds__(kSpThreads, 3) sddmm_kernel(SddmmArgs a) {
 
     int64_t e_row = row_end(row);
     if (n_tiles == 1) load_dy(row, 0);
+    if constexpr (G > 1 && G < 32) {
+        // 2..16 lanes per entry (one tile covers n): the unit's column indices
+        // stream through a per-warp cp.async ring of kNarrowStages chunks of
+        // kNarrowChunk entries, two chunks ahead of the one being consumed
+        extern __shared__ __align__(16) int32_t sddmm_smem[];
+        int32_t *ring = sddmm_smem + (threadIdx.x >> 5) * (kNarrowStages * kNarrowChunk);
+        auto issue = [&](int64_t cs) {
+            if (cs < k1) {
+                const int slot = (int)(((cs - k0) / kNarrowChunk) % kNarrowStages) * kNarrowChunk;
+#pragma unroll
+                for (int q = 0; q < kNarrowChunk / 32; ++q) {
+                    const int64_t idx = cs + q * 32 + lane;
+                    if (idx < k1) cp_async4(ring + slot + q * 32 + lane, a.col + idx);
+                }
+            }
+            cp_async_commit();
+        };
+#pragma unroll
+        for (int q = 0; q < kNarrowStages - 1; ++q) issue(k0 + (int64_t)q * kNarrowChunk);
+        for (int64_t cs = k0; cs < k1; cs += kNarrowChunk) {
+            issue(cs + (int64_t)(kNarrowStages - 1) * kNarrowChunk);
+            cp_async_wait<kNarrowStages - 1>();
+            __syncwarp();
+            const int slot = (int)(((cs - k0) / kNarrowChunk) % kNarrowStages) * kNarrowChunk;
+            const int64_t ce = imin<int64_t>(cs + kNarrowChunk, k1);
+            for (int64_t kb = cs; kb < ce;) {
+                while (e_row <= kb) {   // the row holding entry kb (empty rows are passed over)
+                    ++row;
+                    e_row = row_end(row);
+                    load_dy(row, 0);
+                }
+                const int64_t kn = imin<int64_t>(imin<int64_t>(kb + B, e_row), ce);
+                const int rem = (int)(kn - kb - grp);
+                const int off = slot + (int)(kb - cs) + grp;
+                bool ok[U];
+                int c[U];
+                float p[U];
+#pragma unroll
+                for (int st = 0; st < U; ++st) {
+                    ok[st] = st * E < rem;
+                    c[st] = ok[st] ? ring[off + st * E] : 0;
+                    p[st] = 0.f;
+                }
+                typename Vec<VW>::T xv[U][NV];
+#pragma unroll
+                for (int st = 0; st < U; ++st)
+#pragma unroll
+                    for (int v = 0; v < NV; ++v) {
+                        const int col = gl * VW + v * kStride;
+                        if (ok[st] && col < a.n) xv[st][v] = ldv<VW>(a.x + (int64_t)c[st] * a.n + col);
+                    }
+#pragma unroll
+                for (int st = 0; st < U; ++st)
+#pragma unroll
+                    for (int v = 0; v < NV; ++v) {
+                        const int col = gl * VW + v * kStride;
+                        if (ok[st] && col < a.n) {
+                            float f[VW];
+                            unpack<VW>(xv[st][v], f);
+#pragma unroll
+                            for (int e = 0; e < VW; ++e) p[st] = fmaf(dyv[v][e], f[e], p[st]);
+                        }
+                    }
+                group_reduce_multi<U, G>(p, gl);
+                if (gl % (G / R) == 0) {
+                    float *op = a.out + kb + grp;
+                    const int r = gl / (G / R);
+#pragma unroll
+                    for (int b = 0; b < U / R; ++b) {
+                        const int st = b * R + r;
+                        if (st * E < rem) op[st * E] = p[b * R];
+                    }
+                }
+                kb = kn;
+            }
+            __syncwarp();   // the slot is read before the copy issued next refills it
+        }
+        cp_async_wait<0>();
+        return;
+    }
     int64_t kb = k0;
     fetch(kb);
     while (kb < k1) {
@@ -940,15 +1020,18 @@ int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_
     CSRT_SDDMM_CASE(1, 1, 16) CSRT_SDDMM_CASE(1, 1, 32) CSRT_SDDMM_CASE(1, 2, 32)
 #undef CSRT_SDDMM_CASE
     CSRT_ARG(kern != nullptr, "sddmm: no kernel for vw=%d nv=%d g=%d", vw, nv, g);
+    // 2..16 lanes per entry: the per-warp ring of column indices in shared memory
+    const size_t smem = (g > 1 && g < 32) ? (size_t)(kSpThreads / 32) * kNarrowStages * kNarrowChunk * sizeof(int32_t) : 0;
     if (wps == 0) {
         int blocks = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kern, kSpThreads, 0) != cudaSuccess || blocks <= 0)
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kern, kSpThreads, smem) != cudaSuccess ||
+            blocks <= 0)
             blocks = kWarpsPerSM / (kSpThreads / 32);
         wps = imin(blocks * (kSpThreads / 32), kWarpsPerSM);
     }
     a.units = (int)imax<int64_t>(1, imin<int64_t>((int64_t)num_sms() * wps, w->capacity));
     const unsigned grid = (unsigned)ceil_div<int64_t>((int64_t)a.units * 32, kSpThreads);
-    launch_pdl(kern, dim3(grid), dim3(kSpThreads), 0, s, a);
+    launch_pdl(kern, dim3(grid), dim3(kSpThreads), smem, s, a);
     count_launch();
     return check_launch("sddmm_kernel");
 }
