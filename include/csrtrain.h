@@ -64,6 +64,7 @@ extern "C" {
                                  the count that was needed. */
 #define CSRT_DEV_TIMEOUT 2    /* a bounded inter-block wait gave up; results invalid */
 #define CSRT_DEV_NONFINITE 4  /* the prox step met a NaN in w - eta*G (dropped) */
+#define CSRT_DEV_INVALID 8    /* csrt_validate_csr found a broken invariant */
 
 /* weight_grad_dense precision. */
 #define CSRT_PREC_FP32 0      /* float32 FMA on the CUDA cores */
@@ -133,6 +134,28 @@ int csrt_get_status(const void *ws, int32_t *flags, int64_t *required_nnz, void 
 
 /* Clear the status word on `stream`. */
 int csrt_clear_status(void *ws, void *stream);
+
+/* csrt_validate_csr -- structural check of a CSR (the paper has no
+ * counterpart; the preconditions every call here assumes, Section 3.1's
+ * format): row_ptr[0] == 0, 0 <= row_ptr[r] <= row_ptr[r+1] <= capacity,
+ * and within each row 0 <= col_idx < cols, strictly ascending. If t_row_ptr
+ * is set, the transposed arrays too: the same checks on (t_row_ptr,
+ * t_col_idx) with rows and cols swapped, equal entry counts, and for every
+ * entry k of row r: t_pos[k] lies in column col_idx[k]'s range, t_col_idx
+ * there is r and t_val holds val[k]'s bits. Every index is bounded before it
+ * is used, so a corrupted CSR cannot cause an out-of-range read. A broken
+ * invariant sets CSRT_DEV_INVALID in the status word (csrt_get_status) and
+ * records the first row found (csrt_get_invalid_row). Arrays are device
+ * memory of the lengths the csrt_csr comment gives; nothing is written but
+ * the status header. */
+int csrt_validate_csr(const csrt_csr *w, void *ws, size_t ws_bytes, void *stream);
+
+/* Synchronise `stream`, then report the row where csrt_validate_csr first
+ * found a broken invariant: r < rows for the CSR, rows + 1 + c for column c
+ * of the transposed copy (rows for unequal entry counts), rows + cols + 1 + r
+ * for a transposed position of row r's entries; -1 if none (cleared by
+ * csrt_clear_status). */
+int csrt_get_invalid_row(const void *ws, int64_t *row, void *stream);
 
 /* Message for the last failing call on this host thread ("" if none). */
 const char *csrt_last_error(void);

@@ -13,7 +13,7 @@ namespace csrt {
 // ---------------------------------------------------------------------------
 struct WsHeader {
     unsigned int flags;             // CSRT_DEV_* bits, OR-ed by kernels
-    unsigned int pad0;
+    unsigned int invalid_row;       // csrt_validate_csr: 0xffffffff - first invalid row (0: none)
     unsigned long long required;    // largest nnz an overflowing output needed
     unsigned int ticket;            // tile ticket of the running compaction
     unsigned int timeout_site;      // last wait that gave up (diagnostics)

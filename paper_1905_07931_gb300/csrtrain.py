@@ -18,7 +18,7 @@ import torch
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libcsrtrain.so")
 
 CSRT_OK, CSRT_ERR_ARG, CSRT_ERR_CUDA, CSRT_ERR_WORKSPACE = 0, 1, 2, 3
-CSRT_DEV_CAPACITY, CSRT_DEV_TIMEOUT, CSRT_DEV_NONFINITE = 1, 2, 4
+CSRT_DEV_CAPACITY, CSRT_DEV_TIMEOUT, CSRT_DEV_NONFINITE, CSRT_DEV_INVALID = 1, 2, 4, 8
 CSRT_PREC_FP32, CSRT_PREC_TF32 = 0, 1
 
 
@@ -42,6 +42,8 @@ _SIGS = {
     "csrt_workspace_init": [c_void_p, c_size_t, c_void_p],
     "csrt_get_status": [c_void_p, POINTER(c_int32), POINTER(c_int64), c_void_p],
     "csrt_clear_status": [c_void_p, c_void_p],
+    "csrt_validate_csr": [POINTER(csrt_csr), c_void_p, c_size_t, c_void_p],
+    "csrt_get_invalid_row": [c_void_p, POINTER(c_int64), c_void_p],
     "csr_from_dense": [c_void_p, c_int32, c_int32, POINTER(csrt_csr), c_void_p, c_size_t, c_void_p],
     "csr_transpose": [POINTER(csrt_csr), c_void_p, c_size_t, c_void_p],
     "spmm_fwd": [POINTER(csrt_csr), c_void_p, c_int32, c_void_p, c_void_p, c_size_t, c_void_p],
@@ -225,6 +227,16 @@ def csr_from_dense(dense: torch.Tensor, out: CSR, ws: Workspace, stream=None):
     _f32(dense, "dense", out.rows * out.cols)
     _check(lib().csr_from_dense(_ptr(dense), out.rows, out.cols, out.struct, ws.ptr, ws.nbytes, _stream(stream)),
            "csr_from_dense")
+
+
+def validate_csr(w: CSR, ws: Workspace, stream=None):
+    """Structural check of w (and its transposed copy). Returns the first row
+    with a broken invariant (see csrt_get_invalid_row), or None. Synchronises;
+    leaves CSRT_DEV_INVALID set in the status word when it finds one."""
+    _check(lib().csrt_validate_csr(w.struct, ws.ptr, ws.nbytes, _stream(stream)), "csrt_validate_csr")
+    row = c_int64(0)
+    _check(lib().csrt_get_invalid_row(ws.ptr, ctypes.byref(row), _stream(stream)), "csrt_get_invalid_row")
+    return None if row.value < 0 else int(row.value)
 
 
 def csr_transpose(w: CSR, ws: Workspace, stream=None):
