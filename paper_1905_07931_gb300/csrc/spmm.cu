@@ -272,13 +272,14 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_merge_kernel(SpmmArgs a) {
 // (n = 1: one lane in 32) and keeps only a few loads in flight, so it runs
 // far below the HBM rate that its CSR stream could reach. Here a group of
 // G lanes (G*VW >= n) takes one nonzero, so a warp step covers E = 32/G
-// nonzeros; every lane loads its group's column index and value itself
-// (one coalesced request per step), the next batch of U steps is requested
-// before the current one is consumed (also across row ends: a row's entries
-// follow the previous row's), and at the end of a row the groups' partial
-// sums are combined by a butterfly over the lane bits above G. The unit
-// split, the row-end window and the shared-row protocol are those of
-// spmm_merge_kernel (carries of TN = G*VW floats).
+// nonzeros and a batch of U steps B = U*E nonzeros, cut at row ends. The
+// column indices and values arrive ahead of their use: with G = 1 the next
+// batch is loaded into registers while the current one is consumed; with
+// G >= 2 they stream through a per-warp ring of cp.async chunks in shared
+// memory (see below). At the end of a row the groups' partial sums are
+// combined by a butterfly over the lane bits above G. The unit split, the
+// row-end window and the shared-row protocol are those of spmm_merge_kernel
+// (carries of TN = G*VW floats).
 // ---------------------------------------------------------------------------
 template <int VW> struct NarrowSteps { static constexpr int value = VW == 1 ? 8 : 4; };
 constexpr int kNarrowChunk = 256;   // entries per ring chunk
