@@ -373,20 +373,24 @@ def test_prox_chain_of_steps_bit_exact(C, m, k):
         _check_csr_equal(bufs[(step + 1) % 2], ref)
 
 
-@pytest.mark.parametrize("m,k,n,density,lam,transposed", [
-    (300, 512, 64, 0.1, 0.05, True),
-    (129, 320, 36, 0.2, 0.02, False),
-    (200, 800, 128, 0.05, 0.03, True),
-    (1000, 4096, 256, 0.15, 0.01, True),
-    (64, 64, 4, 0.0, 0.0, True),
-    (260, 9216, 64, 0.05, 0.02, True),
-    (70, 16384, 32, 0.05, 0.02, False),
+@pytest.mark.parametrize("m,k,n,density,lam,transposed,zipf", [
+    (300, 512, 64, 0.1, 0.05, True, False),
+    (129, 320, 36, 0.2, 0.02, False, False),
+    (200, 800, 128, 0.05, 0.03, True, False),
+    (1000, 4096, 256, 0.15, 0.01, True, False),
+    (64, 64, 4, 0.0, 0.0, True, False),
+    (260, 9216, 64, 0.05, 0.02, True, False),
+    (70, 16384, 32, 0.05, 0.02, False, False),
+    # power-law rows (dense rows: every word past the prefetched weights) and
+    # a fully dense input
+    (400, 1024, 64, 0.3, 0.02, True, True),
+    (160, 256, 32, 1.0, 0.05, True, False),
 ])
-def test_fused_gradient_prox_matches_unfused(C, m, k, n, density, lam, transposed):
+def test_fused_gradient_prox_matches_unfused(C, m, k, n, density, lam, transposed, zipf):
     """weight_grad_prox_update (G never written) gives the same bits as
     weight_grad_dense (TF32) followed by prox_update_compact."""
     rng = np.random.default_rng(m + k + n)
-    a = _sparse(rng, m, k, density) * F32(0.05)
+    a = _sparse(rng, m, k, density, zipf) * F32(0.05)
     dy = _dev((rng.standard_normal((m, n)) * 0.1).astype(F32))
     x = _dev(rng.standard_normal((k, n)).astype(F32))
     ws = _ws(C, m, k, n)
