@@ -15,8 +15,9 @@ Workloads: single_fc (one FC layer 784->300, upstream gradient given, prox
 steps only), mlp (784-300-100-10), lenet (LeNet-5 style), fc_head
 (9216-4096-4096-1000). The inputs are synthetic, drawn with the workload's
 distribution (U[0,1] images, half-normal features, uniform labels) into a
-pool of --batches seeded batches that the steps cycle through; each step
-copies its batch from pinned host memory.
+pool of --batches seeded batches that the steps cycle through; each batch
+is copied from pinned host memory on a copy stream while the previous step
+runs (train.BatchPrefetcher).
 
 --save writes every layer's CSR arrays (row_ptr, col_idx, val, trimmed to the
 stored count) and bias to an .npz; --load puts such arrays back into the
@@ -37,7 +38,7 @@ import torch
 
 from . import csrtrain as C
 from . import synth
-from .train import SingleLayer, SparseNet, lenet_layers, mlp_layers
+from .train import BatchPrefetcher, SingleLayer, SparseNet, lenet_layers, mlp_layers
 
 WORKLOADS = ("single_fc", "mlp", "lenet", "fc_head")
 
@@ -148,6 +149,8 @@ def run(config: str, prox_steps: int, debias_steps: int, seed: int = 0, batches:
     stream = torch.cuda.current_stream()
     records = []
     phases = [("prox", prox_steps)] + ([("debias", debias_steps)] if config != "single_fc" else [])
+    total = sum(c for _, c in phases)
+    pf = None if pool is None else BatchPrefetcher(net)
     step = 0
     for phase, count in phases:
         for _ in range(count):
@@ -158,9 +161,13 @@ def run(config: str, prox_steps: int, debias_steps: int, seed: int = 0, batches:
                 net.step(eta, lam)
                 batch = net.x.shape[1]
             else:
-                x, y = pool[step % len(pool)]
-                net.x_in.copy_(x.view(net.x_in.shape), non_blocking=True)
-                net.labels.copy_(y, non_blocking=True)
+                # batch `step` was copied while the previous step ran; the copy
+                # of the next one overlaps this step
+                if step == 0:
+                    pf.issue(*pool[0], after=st)
+                pf.load()
+                if step + 1 < total:
+                    pf.issue(*pool[(step + 1) % len(pool)], after=st)
                 lt = net.step(phase, eta, lam)
                 batch = net.batch
             en.record(stream)

@@ -258,6 +258,61 @@ class SparseNet:
                     L[key].zero_()
 
 
+class BatchPrefetcher:
+    """Input pipeline of a SparseNet: batch i+1 is copied from pinned host
+    memory into one of two device slots on a copy stream while step i runs;
+    ``load`` then hands a slot to the network (``x_in`` / ``labels``) with a
+    device-to-device copy on the network's stream. The network keeps reading
+    ``x_in`` until its last weight gradient, so the next batch cannot be
+    copied into ``x_in`` itself while a step is in flight.
+
+      pf.issue(x0, y0, after=start_event)          # batch 0
+      for i in range(steps):
+          pf.load(i)                                # waits for batch i's copy
+          if i + 1 < steps: pf.issue(x[i+1], y[i+1])  # overlaps step i
+          net.step(...)
+    """
+
+    def __init__(self, net):
+        self.net = net
+        self.copy_stream = torch.cuda.Stream(device=net.x_in.device)
+        self.x = [torch.empty_like(net.x_in) for _ in range(2)]
+        self.y = [torch.empty_like(net.labels) for _ in range(2)]
+        self.ready = [torch.cuda.Event() for _ in range(2)]
+        self.free = [torch.cuda.Event() for _ in range(2)]
+        self.issued = 0
+        self.loaded = 0
+
+    def issue(self, x_host: torch.Tensor, y_host: torch.Tensor, after: torch.cuda.Event | None = None):
+        """Enqueue the host-to-device copy of the next batch (pinned host
+        tensors of the shapes of ``x_in`` and ``labels``); the copy starts
+        after ``after`` (an event on the network's stream) if given, and after
+        the slot's previous batch has been loaded."""
+        slot = self.issued % 2
+        cs = self.copy_stream
+        if after is not None:
+            cs.wait_event(after)
+        cs.wait_event(self.free[slot])
+        with torch.cuda.stream(cs):
+            self.x[slot].copy_(x_host.view(self.x[slot].shape), non_blocking=True)
+            self.y[slot].copy_(y_host, non_blocking=True)
+            self.ready[slot].record(cs)
+        self.issued += 1
+
+    def load(self):
+        """Make the oldest issued batch the network's input, on its stream."""
+        if self.loaded >= self.issued:
+            raise RuntimeError("no batch issued")
+        slot = self.loaded % 2
+        s = self.net.stream or torch.cuda.current_stream()
+        s.wait_event(self.ready[slot])
+        with torch.cuda.stream(s):
+            self.net.x_in.copy_(self.x[slot])
+            self.net.labels.copy_(self.y[slot])
+            self.free[slot].record(s)
+        self.loaded += 1
+
+
 def mlp_layers(n_layers: int):
     return [{"kind": "fc", "relu": i < n_layers - 1} for i in range(n_layers)]
 
