@@ -575,19 +575,13 @@ __global__ void __launch_bounds__(kCThreads, 4) compact_rows_kernel(CompactArgs 
 // compact_rows_kernel, one read of G: pass 1 evaluates every entry once,
 // counts the kept ones per lane and parks each result in the shared old-weight
 // tile (the kept value, or NaN for a dropped entry: a kept value is never
-// NaN); pass 2 reads only shared memory. With kBits (K % 32 == 0 and a
-// transposed copy wanted) pass 2 also emits, per 32-entry word of a row, the
-// keep bitmask and the CSR position of the word's first entry, from which the
-// transposed copy is built without re-reading the CSR.
+// NaN); pass 2 reads only shared memory, one entry per lane, and ranks the
+// kept entries with one ballot per 32 (their stores form one run). With kBits
+// (K % 32 == 0 and a transposed copy wanted) pass 2 also emits, per 32-entry
+// word of a row, the keep bitmask and the CSR position of the word's first
+// entry, from which the transposed copy is built without re-reading the CSR.
 // ---------------------------------------------------------------------------
-// bit t of x (t < 8) -> bit 4t
-__device__ __forceinline__ uint32_t spread8(uint32_t x) {
-    x &= 0xFFu;
-    x = (x | (x << 12)) & 0x000F000Fu;
-    x = (x | (x << 6)) & 0x03030303u;
-    x = (x | (x << 3)) & 0x11111111u;
-    return x;
-}
+constexpr int kPsSteps = 4;   // 32-entry steps per warp iteration of pass 2 (independent loads)
 
 template <bool kBits>
 __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, int32_t rows_per_tile,
@@ -735,57 +729,126 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
     pos += s_excl;
     const uint32_t cap = (uint32_t)imin<int64_t>(a.capacity, 0x7fffffff);
 
-    // pass 2: positions from ballots, writes
-    int row = e_beg / K;
-    int col = e_beg - row * K + 4 * lane;
-    while (col >= K) { col -= K; ++row; }
-    for (int base = e_beg; base < e_end; base += 128) {
-        const int b = base + 4 * lane;
-        const bool in = b < e_end;
-        const float4 v = in ? *reinterpret_cast<const float4 *>(tile_v + b) : make_float4(__int_as_float(0x7fc00000),
-                                                                                   __int_as_float(0x7fc00000),
-                                                                                   __int_as_float(0x7fc00000),
-                                                                                   __int_as_float(0x7fc00000));
-        const float vv[4] = {v.x, v.y, v.z, v.w};
-        // keep bits of this lane's four entries; warp scan of their counts gives the ranks
-        const unsigned nib = (unsigned)(vv[0] == vv[0]) | ((unsigned)(vv[1] == vv[1]) << 1) |
-                             ((unsigned)(vv[2] == vv[2]) << 2) | ((unsigned)(vv[3] == vv[3]) << 3);
-        const uint32_t c = __popc(nib);
-        uint32_t incl = c;
+    // pass 2. A tile that keeps most of its entries: lane = entry of a 32-entry
+    // step; one ballot gives the step's keep word and every lane's rank in it,
+    // so the kept entries go out as one coalesced run (measured 14-34% faster
+    // on dense outputs). Other tiles: four entries per lane and a warp scan,
+    // whose shorter dependency chain per 128 entries wins on sparse outputs.
+    // With K % 32 == 0 a step (the segments are whole 128-entry groups) is
+    // exactly one 32-column word of one row: its ballot is the keep bitmask of
+    // the transposed copy.
+    if (2 * (int64_t)tile_count > n_el) {   // dense tile
+        const unsigned lt = (1u << lane) - 1u;
+        const float qnan = __int_as_float(0x7fc00000);
+        const bool wide = K >= 32;                               // a step crosses at most one row end
+        const bool fits = (uint64_t)s_excl + tile_count <= cap;   // no position of the tile reaches the capacity
+        int row = e_beg / K;           // row and column of the step's first entry
+        int c0 = e_beg - row * K;
+        for (int base = e_beg; base < e_end; base += 32 * kPsSteps) {
+            float v4[kPsSteps];
 #pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-            const uint32_t t = __shfl_up_sync(0xffffffffu, incl, off);
-            if (lane >= off) incl += t;
-        }
-        uint32_t p = pos + incl - c;
-        if (in && col == 0) a.out_row_ptr[r0 + row] = (int32_t)min(p, cap);
-        if (kBits) {
-            // 32-entry word of lanes 8q .. 8q+7 (four bits per lane, in order)
-            uint32_t word = nib << (4 * (lane & 7));
-            word |= __shfl_xor_sync(0xffffffffu, word, 1);
-            word |= __shfl_xor_sync(0xffffffffu, word, 2);
-            word |= __shfl_xor_sync(0xffffffffu, word, 4);
-            if (in && (lane & 7) == 0) {
-                const int64_t wi = (int64_t)(r0 + row) * wpr + (col >> 5);
-                keepbits[wi] = word;
-                wordpos[wi] = (int32_t)p;
+            for (int u = 0; u < kPsSteps; ++u) {
+                const int e = base + 32 * u + lane;
+                v4[u] = e < e_end ? tile_v[e] : qnan;
             }
-        }
-        if (nib) {
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                if ((nib >> j) & 1u) {
-                    if (p < cap) {
-                        a.out_col[p] = col + j;
-                        a.out_val[p] = vv[j];
+            for (int u = 0; u < kPsSteps; ++u) {
+                if (base + 32 * u >= e_end) break;   // warp-uniform
+                const bool k = v4[u] == v4[u];
+                const unsigned m = __ballot_sync(0xffffffffu, k);
+                const uint32_t p = pos + __popc(m & lt);
+                int col = c0 + lane, rowl = row;
+                if (wide) {
+                    if (col >= K) {
+                        col -= K;
+                        ++rowl;
                     }
-                    ++p;
+                } else {
+                    while (col >= K) {
+                        col -= K;
+                        ++rowl;
+                    }
+                }
+                if (c0 == 0 || c0 + 32 > K) {   // a row starts in this step
+                    if (base + 32 * u + lane < e_end && col == 0) a.out_row_ptr[r0 + rowl] = (int32_t)min(p, cap);
+                }
+                if (kBits && lane == 0) {
+                    const int64_t wi = (int64_t)(r0 + row) * wpr + (c0 >> 5);
+                    keepbits[wi] = m;
+                    wordpos[wi] = (int32_t)pos;
+                }
+                if (k && (fits || p < cap)) {
+                    a.out_col[p] = col;
+                    a.out_val[p] = v4[u];
+                }
+                pos += __popc(m);
+                c0 += 32;
+                if (wide) {
+                    if (c0 >= K) {
+                        c0 -= K;
+                        ++row;
+                    }
+                } else {
+                    while (c0 >= K) {
+                        c0 -= K;
+                        ++row;
+                    }
                 }
             }
         }
-        pos += __shfl_sync(0xffffffffu, incl, 31);
-        col += 128;
+    } else {
+        // pass 2, sparse tile: four consecutive entries per lane, ranks from a warp scan
+        int row = e_beg / K;
+        int col = e_beg - row * K + 4 * lane;
         while (col >= K) { col -= K; ++row; }
+        for (int base = e_beg; base < e_end; base += 128) {
+            const int b = base + 4 * lane;
+            const bool in = b < e_end;
+            const float4 v = in ? *reinterpret_cast<const float4 *>(tile_v + b) : make_float4(__int_as_float(0x7fc00000),
+                                                                                       __int_as_float(0x7fc00000),
+                                                                                       __int_as_float(0x7fc00000),
+                                                                                       __int_as_float(0x7fc00000));
+            const float vv[4] = {v.x, v.y, v.z, v.w};
+            // keep bits of this lane's four entries; warp scan of their counts gives the ranks
+            const unsigned nib = (unsigned)(vv[0] == vv[0]) | ((unsigned)(vv[1] == vv[1]) << 1) |
+                                 ((unsigned)(vv[2] == vv[2]) << 2) | ((unsigned)(vv[3] == vv[3]) << 3);
+            const uint32_t c = __popc(nib);
+            uint32_t incl = c;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const uint32_t t = __shfl_up_sync(0xffffffffu, incl, off);
+                if (lane >= off) incl += t;
+            }
+            uint32_t p = pos + incl - c;
+            if (in && col == 0) a.out_row_ptr[r0 + row] = (int32_t)min(p, cap);
+            if (kBits) {
+                // 32-entry word of lanes 8q .. 8q+7 (four bits per lane, in order)
+                uint32_t word = nib << (4 * (lane & 7));
+                word |= __shfl_xor_sync(0xffffffffu, word, 1);
+                word |= __shfl_xor_sync(0xffffffffu, word, 2);
+                word |= __shfl_xor_sync(0xffffffffu, word, 4);
+                if (in && (lane & 7) == 0) {
+                    const int64_t wi = (int64_t)(r0 + row) * wpr + (col >> 5);
+                    keepbits[wi] = word;
+                    wordpos[wi] = (int32_t)p;
+                }
+            }
+            if (nib) {
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    if ((nib >> j) & 1u) {
+                        if (p < cap) {
+                            a.out_col[p] = col + j;
+                            a.out_val[p] = vv[j];
+                        }
+                        ++p;
+                    }
+                }
+            }
+            pos += __shfl_sync(0xffffffffu, incl, 31);
+            col += 128;
+            while (col >= K) { col -= K; ++row; }
+        }
     }
     if (tile == a.num_tiles - 1 && tid == 0) {
         const int64_t total = (int64_t)s_excl + tile_count;

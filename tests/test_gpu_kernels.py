@@ -344,6 +344,8 @@ def test_prox_hand_cases_on_gpu(C):
     (2, 20000, 0.3, 1.0, 0.01, 0.5),
     (4100, 512, 0.05, 1.0, 0.01, 1e-4),
     (700, 900, 0.5, 0.1, 0.1, 1.0),
+    (20000, 784, 0.05, 1.0, 0.01, 1e-2),   # 2000 row tiles: several per resident block
+    (1500, 9216, 0.05, 1.0, 0.01, 1e-4),   # one-row tiles, dense output
 ])
 def test_prox_bit_exact(C, m, k, density, gscale, eta, lam):
     rng = np.random.default_rng(m + k)
