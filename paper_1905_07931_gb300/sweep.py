@@ -125,7 +125,8 @@ def run_layer(m: int, k: int, density: float, zipf: bool, batches, ops, reps: in
             ms = _time(fn, reps, flush)
             nnz_out = W_out.nnz()
             byts = 4 * m * k + 8 * nnz + 4 * (m + 1) + 8 * nnz_out + 4 * (m + 1)
-            byts += 12 * nnz_out + 8 * nnz_out + 4 * (k + 1) + 4 * (m + 1)   # transposed pattern
+            if transposed:   # the transposed pattern: t_col, t_val, t_pos written, col and val read back
+                byts += 12 * nnz_out + 8 * nnz_out + 4 * (k + 1) + 4 * (m + 1)
             rows.append({"op": f"prox ({tag})", "m": m, "k": k, "density": density,
                          "rows": "zipf" if zipf else "uniform", "n": 0, "nnz": nnz, "nnz_out": nnz_out,
                          "us": round(ms * 1e3, 2), "bytes": byts, "gbs": round(byts / (ms / 1e3) / 1e9, 1)})
