@@ -165,6 +165,53 @@ __device__ __forceinline__ int64_t warp_first_false(int64_t lo, int64_t hi, Pred
     return lo + __popc(__ballot_sync(0xffffffffu, p));
 }
 
+// Two independent searches of warp_first_false, run round by round together
+// so that the latencies of their probes overlap (each round issues both
+// probes before either ballot). Results in ra and rb.
+template <typename PredA, typename PredB>
+__device__ __forceinline__ void warp_first_false2(int64_t lo_a, int64_t hi_a, PredA pred_a, int64_t lo_b,
+                                                  int64_t hi_b, PredB pred_b, int64_t &ra, int64_t &rb) {
+    const int lane = threadIdx.x & 31;
+    bool done_a = false, done_b = false;
+    ra = hi_a;
+    rb = hi_b;
+    while (true) {
+        const int64_t len_a = hi_a - lo_a, len_b = hi_b - lo_b;
+        const bool wa = !done_a && len_a > 32, wb = !done_b && len_b > 32;   // warp-uniform
+        if (!wa && !wb) break;
+        const int64_t ia = lo_a + ((int64_t)(lane + 1) * len_a) / 32 - 1;
+        const int64_t ib = lo_b + ((int64_t)(lane + 1) * len_b) / 32 - 1;
+        const bool pa = wa && pred_a(ia);
+        const bool pb = wb && pred_b(ib);
+        const int la = __popc(__ballot_sync(0xffffffffu, pa));
+        const int lb = __popc(__ballot_sync(0xffffffffu, pb));
+        if (wa) {
+            if (la == 32) {
+                done_a = true;
+            } else {
+                const int64_t nlo = lo_a + ((int64_t)la * len_a) / 32;
+                hi_a = lo_a + ((int64_t)(la + 1) * len_a) / 32;
+                lo_a = nlo;
+            }
+        }
+        if (wb) {
+            if (lb == 32) {
+                done_b = true;
+            } else {
+                const int64_t nlo = lo_b + ((int64_t)lb * len_b) / 32;
+                hi_b = lo_b + ((int64_t)(lb + 1) * len_b) / 32;
+                lo_b = nlo;
+            }
+        }
+    }
+    const bool pa = !done_a && lo_a + lane < hi_a && pred_a(lo_a + lane);
+    const bool pb = !done_b && lo_b + lane < hi_b && pred_b(lo_b + lane);
+    const int la = __popc(__ballot_sync(0xffffffffu, pa));
+    const int lb = __popc(__ballot_sync(0xffffffffu, pb));
+    if (!done_a) ra = lo_a + la;
+    if (!done_b) rb = lo_b + lb;
+}
+
 // First position p in [s, e) with col[p] >= target (col ascending in [s, e)).
 __device__ __forceinline__ int64_t warp_lower_bound(const int32_t *__restrict__ col, int64_t s, int64_t e,
                                                     int32_t target) {

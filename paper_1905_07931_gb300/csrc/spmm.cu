@@ -57,6 +57,18 @@ __device__ __forceinline__ int merge_rows_before(const int32_t *__restrict__ row
                                                  int64_t hi) {
     return (int)warp_first_false(lo, hi, [&](int64_t i) { return (int64_t)__ldg(row_ptr + i + 1) + i < d; });
 }
+// The rows before diagonals d0 and d1 (a unit's start and end), both
+// searches run together.
+__device__ __forceinline__ void merge_rows_before2(const int32_t *__restrict__ row_ptr, int32_t rows, int64_t nnz,
+                                                   int64_t d0, int64_t d1, int &i0, int &i1) {
+    int64_t r0, r1;
+    warp_first_false2(
+        imax<int64_t>(0, d0 - nnz), imin<int64_t>(d0, rows),
+        [&](int64_t i) { return (int64_t)__ldg(row_ptr + i + 1) + i < d0; }, imax<int64_t>(0, d1 - nnz),
+        imin<int64_t>(d1, rows), [&](int64_t i) { return (int64_t)__ldg(row_ptr + i + 1) + i < d1; }, r0, r1);
+    i0 = (int)r0;
+    i1 = (int)r1;
+}
 
 struct SpmmArgs {
     const int32_t *row_ptr;
@@ -76,6 +88,7 @@ struct SpmmArgs {
     const float *bias;
     int32_t relu;
     const float *mask;
+    WsHeader *hdr;    // status word for a bounded wait that gives up (null: not reported)
 };
 
 // The epilogue of one row segment held by a lane (VW floats at column c).
@@ -283,16 +296,37 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_merge_kernel(SpmmArgs a) {
 // ---------------------------------------------------------------------------
 template <int VW> struct NarrowSteps { static constexpr int value = VW == 1 ? 8 : 4; };
 constexpr int kNarrowChunk = 256;   // entries per ring chunk
-constexpr int kNarrowStages = 3;    // ring chunks per warp
-constexpr int kNarrowSmem = (kSpThreads / 32) * 2 * kNarrowStages * kNarrowChunk * (int)sizeof(int32_t);
+constexpr int kNarrowStages = 4;    // ring chunks per warp
+constexpr int kNarrowRingInts = 2 * kNarrowStages * kNarrowChunk;   // per warp: indices, then values
+constexpr int kNarrowSmem = (kSpThreads / 32) * (kNarrowRingInts * (int)sizeof(int32_t) + kNarrowStages * 8);
 
-__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+__device__ __forceinline__ uint32_t sp_smem_addr(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+// One bulk asynchronous copy global -> shared (16-byte aligned, a multiple of
+// 16 bytes) that completes on the mbarrier bar.
+__device__ __forceinline__ void sp_bulk_copy(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     sp_smem_addr(dst)),
+                 "l"(src), "r"(bytes), "r"(sp_smem_addr(bar))
                  : "memory");
 }
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+// Bounded wait for the phase of the given parity; false if it gave up.
+__device__ __forceinline__ bool sp_bar_wait(uint64_t *bar, uint32_t parity) {
+    const uint32_t addr = sp_smem_addr(bar);
+    for (unsigned i = 0; i < kSpinLimit; ++i) {
+        uint32_t done;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            " selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(done)
+            : "r"(addr), "r"(parity)
+            : "memory");
+        if (done) return true;
+        if (i > 16) __nanosleep(32);
+    }
+    return false;
+}
 
 template <int VW, int G>
 __global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
@@ -310,8 +344,8 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
     const int64_t items = (int64_t)a.rows + nnz;
     const int64_t per = ceil_div<int64_t>(items, a.units);
     const int64_t d0 = min((int64_t)u * per, items), d1 = min(d0 + per, items);
-    const int i0 = merge_rows_before(a.row_ptr, d0, imax<int64_t>(0, d0 - nnz), imin<int64_t>(d0, a.rows));
-    const int i1 = merge_rows_before(a.row_ptr, d1, imax<int64_t>(0, d1 - nnz), imin<int64_t>(d1, a.rows));
+    int i0, i1;
+    merge_rows_before2(a.row_ptr, a.rows, nnz, d0, d1, i0, i1);
     const int64_t k0 = d0 - i0, k1 = d1 - i1;
     const int c0 = t * TN + gl * VW;
     const bool in_n = c0 < a.n;
@@ -360,87 +394,69 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
             e_row = row_end(i);
         }
     };
-    if constexpr (G == 1) {
-        // one nonzero per lane: the indices and values of the next batch are
-        // loaded into registers while the current batch is consumed (the
-        // instructions of a shared-memory ring cost more than they hide here)
-        int cn[U];
-        float wn[U];
-        auto fetch = [&](int64_t kb) {
-            const int32_t *cp = a.col + kb + lane;
-            const float *vp = a.val + kb + lane;
-            const int lim = (int)imin<int64_t>(k1 - kb - lane, B);
-#pragma unroll
-            for (int st = 0; st < U; ++st) {
-                const bool ok = st * 32 < lim;
-                cn[st] = ok ? __ldg(cp + st * 32) : 0;
-                wn[st] = ok ? __ldg(vp + st * 32) : 0.f;
-            }
-        };
-        int64_t kb = k0;
-        if (kb < k1) fetch(kb);
-        while (true) {
-            finish_rows(kb);
-            if (kb >= k1) break;
-            int c[U];
-            float w[U];
-#pragma unroll
-            for (int st = 0; st < U; ++st) {
-                c[st] = cn[st];
-                w[st] = wn[st];
-            }
-            const int64_t kn = imin<int64_t>(kb + B, e_row);
-            const int rem = in_n ? (int)imin<int64_t>(e_row - kb - lane, B) : 0;
-            if (kn < k1) fetch(kn);
-            typename Vec<VW>::T xv[U];
-#pragma unroll
-            for (int st = 0; st < U; ++st)
-                if (st * 32 < rem) xv[st] = ldv<VW>(a.x + (int64_t)c[st] * a.n + c0);
-#pragma unroll
-            for (int st = 0; st < U; ++st)
-                if (st * 32 < rem) {
-                    float f[VW];
-                    unpack<VW>(xv[st], f);
-#pragma unroll
-                    for (int e = 0; e < VW; ++e) acc[e] = fmaf(w[st], f[e], acc[e]);
-                }
-            kb = kn;
-        }
-    } else {
     // The unit's column indices and values stream through a ring of
     // kNarrowStages chunks of kNarrowChunk entries in shared memory (this
-    // warp's slice), copied with cp.async kNarrowStages - 1 chunks ahead of
-    // the one being consumed, so the loads in flight cost no registers.
+    // warp's slice): lane 0 starts one bulk copy per array and chunk,
+    // kNarrowStages - 1 chunks ahead of the one being consumed, so the bytes
+    // in flight cost neither registers nor per-entry copy instructions.
+    // Chunks start at 16-byte boundaries (abase = k0 rounded down to 4
+    // entries); the last 0-3 entries of the unit past a boundary, which a
+    // bulk copy of whole 16-byte units could only cover by reading beyond
+    // k1, are loaded by plain loads.
     extern __shared__ __align__(16) int32_t narrow_smem[];
-    int32_t *ring_c = narrow_smem + (threadIdx.x >> 5) * (2 * kNarrowStages * kNarrowChunk);
+    const int wib = threadIdx.x >> 5;
+    int32_t *ring_c = narrow_smem + wib * kNarrowRingInts;
     float *ring_v = reinterpret_cast<float *>(ring_c + kNarrowStages * kNarrowChunk);
-    auto issue = [&](int64_t cs) {   // chunk starting at entry cs into its ring slot (an empty group past k1)
-        if (cs < k1) {
-            const int slot = (int)(((cs - k0) / kNarrowChunk) % kNarrowStages) * kNarrowChunk;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(narrow_smem + (kSpThreads / 32) * kNarrowRingInts) +
+                     wib * kNarrowStages;
+    if (lane == 0) {
 #pragma unroll
-            for (int q = 0; q < kNarrowChunk / 32; ++q) {
-                const int64_t idx = cs + q * 32 + lane;
-                if (idx < k1) {
-                    cp_async4(ring_c + slot + q * 32 + lane, a.col + idx);
-                    cp_async4(ring_v + slot + q * 32 + lane, a.val + idx);
-                }
+        for (int q = 0; q < kNarrowStages; ++q)
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(sp_smem_addr(bars + q)) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncwarp();
+    const int64_t abase = k0 & ~int64_t(3);
+    const int64_t k1a = k1 & ~int64_t(3);
+    bool failed = false;
+    auto issue = [&](int64_t j) {   // chunk j: entries abase + j*C .. + C, clipped to k1
+        const int64_t A = abase + j * kNarrowChunk;
+        if (A >= k1) return;
+        const int slot = (int)(j % kNarrowStages) * kNarrowChunk;
+        const int64_t fe = imin<int64_t>(A + kNarrowChunk, k1a);
+        const uint32_t nb = fe > A ? (uint32_t)(fe - A) * 4u : 0u;
+        const int64_t t0 = imax<int64_t>(A, k1a), t1 = imin<int64_t>(A + kNarrowChunk, k1);
+        if (lane < t1 - t0) {
+            ring_c[slot + (int)(t0 - A) + lane] = __ldg(a.col + t0 + lane);
+            ring_v[slot + (int)(t0 - A) + lane] = __ldg(a.val + t0 + lane);
+        }
+        if (lane == 0) {
+            uint64_t *bar = bars + j % kNarrowStages;
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(sp_smem_addr(bar)),
+                         "r"(2u * nb)
+                         : "memory");
+            if (nb) {
+                sp_bulk_copy(ring_c + slot, a.col + A, nb, bar);
+                sp_bulk_copy(ring_v + slot, a.val + A, nb, bar);
             }
         }
-        cp_async_commit();
     };
 #pragma unroll
-    for (int q = 0; q < kNarrowStages - 1; ++q) issue(k0 + (int64_t)q * kNarrowChunk);
-    for (int64_t cs = k0; cs < k1; cs += kNarrowChunk) {
-        issue(cs + (int64_t)(kNarrowStages - 1) * kNarrowChunk);
-        cp_async_wait<kNarrowStages - 1>();
+    for (int q = 0; q < kNarrowStages - 1; ++q) issue(q);
+    for (int64_t j = 0;; ++j) {
+        const int64_t A = abase + j * kNarrowChunk;
+        if (A >= k1) break;
+        issue(j + kNarrowStages - 1);
+        if (!sp_bar_wait(bars + j % kNarrowStages, (uint32_t)((j / kNarrowStages) & 1))) failed = true;
         __syncwarp();
-        const int slot = (int)(((cs - k0) / kNarrowChunk) % kNarrowStages) * kNarrowChunk;
-        const int64_t ce = imin<int64_t>(cs + kNarrowChunk, k1);
-        for (int64_t kb = cs; kb < ce;) {
+        const int slot = (int)(j % kNarrowStages) * kNarrowChunk;
+        const int64_t ce = imin<int64_t>(A + kNarrowChunk, k1);
+        for (int64_t kb = imax<int64_t>(A, k0); kb < ce;) {
             finish_rows(kb);
             const int64_t kn = imin<int64_t>(imin<int64_t>(kb + B, e_row), ce);
             const int rem = in_n ? (int)(kn - kb - grp) : 0;
-            const int off = slot + (int)(kb - cs) + grp;
+            const int off = slot + (int)(kb - A) + grp;
             int c[U];
             float w[U];
 #pragma unroll
@@ -465,8 +481,10 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
         }
         __syncwarp();   // the slot is read before the copy issued next refills it
     }
-    cp_async_wait<0>();
     finish_rows(k1);
+    if (failed && lane == 0 && a.hdr) {
+        dev_flag(a.hdr, CSRT_DEV_TIMEOUT);
+        a.hdr->timeout_site = 10;
     }
     // the unit ends inside row i1: its part is a carry
     const bool has_carry = k1 > kr;
@@ -528,11 +546,15 @@ struct SpmmShape {
     int vw, nv, g, tn, n_tiles, units;
 };
 
+// Resident warps per SM of a kernel with `smem` bytes of dynamic shared
+// memory (cached per device); above 48 KB the kernel is first allowed that
+// much, once per device, which its launches rely on.
 template <typename K>
 static int kernel_warps_per_sm(K kernel, int (&cache)[64], int cap, size_t smem = 0) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return cap;
     if (cache[dev] == 0) {
+        if (smem > 48 * 1024) cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         int blocks = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kernel, kSpThreads, smem) != cudaSuccess ||
             blocks <= 0)
@@ -546,7 +568,7 @@ template <int VW, int NV, int G>
 static int spmm_warps_per_sm() {
     static int cache[64] = {0};
     if constexpr (G == 32) return kernel_warps_per_sm(spmm_merge_kernel<VW, NV>, cache, kWarpsPerSM);
-    else return kernel_warps_per_sm(spmm_group_kernel<VW, G>, cache, kWarpsPerSM, G > 1 ? (size_t)kNarrowSmem : 0);
+    else return kernel_warps_per_sm(spmm_group_kernel<VW, G>, cache, kWarpsPerSM, (size_t)kNarrowSmem);
 }
 
 static int pow2_at_least(int v) {
@@ -558,8 +580,10 @@ static int pow2_at_least(int v) {
 // Tile shape of a product with n columns: 32 lanes on one nonzero with NV
 // vectors of VW floats each (n >= 128 for float4, 64 for float2, 32 for
 // scalars), else the narrow kernel with G = the smallest power of two with
-// G*VW >= n lanes per nonzero.
-static SpmmShape spmm_shape(int32_t n, int64_t max_items, bool vec4_ok, bool vec2_ok) {
+// G*VW >= n lanes per nonzero. The narrow kernel streams the index and value
+// arrays with bulk copies, which need them 16-byte aligned (csr16); without
+// that the 32-lane kernel takes narrow products too.
+static SpmmShape spmm_shape(int32_t n, int64_t max_items, bool vec4_ok, bool vec2_ok, bool csr16) {
     SpmmShape s;
     s.nv = 1;
     s.g = 32;
@@ -569,6 +593,7 @@ static SpmmShape spmm_shape(int32_t n, int64_t max_items, bool vec4_ok, bool vec
     else if (vec2_ok && n <= 32) { s.vw = 2; s.g = pow2_at_least((n + 1) / 2); }
     else if (n <= 16) { s.vw = 1; s.g = pow2_at_least(n); }
     else { s.vw = 1; }
+    if (!csr16) s.g = 32;
     s.tn = s.g * s.vw * s.nv;
     s.n_tiles = (int)ceil_div<int64_t>(n, s.tn);
     // one full wave of resident warps (a partial second wave would run at low occupancy)
@@ -604,7 +629,7 @@ static int spmm_dispatch(const SpmmShape &sh, const SpmmArgs &a, cudaStream_t s)
     const unsigned fg = (unsigned)ceil_div<int64_t>(threads, 256);
 #define CSRT_SPMM_CASE(VW, NV, G, KERNEL)                                                   \
     if (sh.vw == VW && sh.nv == NV && sh.g == G) {                                          \
-        launch_pdl(KERNEL, dim3(grid), dim3(kSpThreads), (G > 1 && G < 32) ? (size_t)kNarrowSmem : 0, s, a); \
+        launch_pdl(KERNEL, dim3(grid), dim3(kSpThreads), G < 32 ? (size_t)kNarrowSmem : 0, s, a);           \
         if (fix) launch_pdl(spmm_fixup_kernel<G * VW * NV>, dim3(fg), dim3(256), 0, s, a); \
         return fix ? 2 : 1;                                                                 \
     }
@@ -637,7 +662,8 @@ static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *
     if (rows == 0 || n == 0) return CSRT_OK;
     const bool v4 = (n % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15) == 0;
     const bool v2 = (n % 2 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 7) == 0;
-    const SpmmShape sh = spmm_shape(n, (int64_t)rows + capacity, v4, v2);
+    const bool csr16 = ((reinterpret_cast<uintptr_t>(col) | reinterpret_cast<uintptr_t>(val)) & 15) == 0;
+    const SpmmShape sh = spmm_shape(n, (int64_t)rows + capacity, v4, v2, csr16);
     SpmmArgs a;
     a.row_ptr = row_ptr;
     a.col = col;
@@ -651,6 +677,7 @@ static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *
     a.bias = bias;
     a.relu = relu;
     a.mask = mask;
+    a.hdr = static_cast<WsHeader *>(ws);
     const size_t carry_floats = (size_t)sh.units * sh.n_tiles * sh.tn;
     a.carry = reinterpret_cast<float *>(ws_scratch(ws));
     a.carry_row = reinterpret_cast<int32_t *>(a.carry + ((carry_floats + 63) / 64) * 64);
@@ -672,6 +699,19 @@ static int spmm_launch(const int32_t *row_ptr, const int32_t *col, const float *
     count_launch(launched);
     return check_launch("spmm_merge_kernel");
 }
+
+// Column-index ring of the narrow SDDMM: chunks of kSdChunk entries copied
+// with 4-byte cp.async, kSdStages - 1 chunks ahead.
+constexpr int kSdChunk = 256;
+constexpr int kSdStages = 3;
+
+__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 // ---------------------------------------------------------------------------
 // SDDMM: g[k] = <dY[i_k, :], X[j_k, :]>
@@ -780,15 +820,15 @@ __global__ void __launch_bounds__(kSpThreads, 3) sddmm_kernel(SddmmArgs a) {
     if (n_tiles == 1) load_dy(row, 0);
     if constexpr (G > 1 && G < 32) {
         // 2..16 lanes per entry (one tile covers n): the unit's column indices
-        // stream through a per-warp cp.async ring of kNarrowStages chunks of
-        // kNarrowChunk entries, two chunks ahead of the one being consumed
+        // stream through a per-warp cp.async ring of kSdStages chunks of
+        // kSdChunk entries, two chunks ahead of the one being consumed
         extern __shared__ __align__(16) int32_t sddmm_smem[];
-        int32_t *ring = sddmm_smem + (threadIdx.x >> 5) * (kNarrowStages * kNarrowChunk);
+        int32_t *ring = sddmm_smem + (threadIdx.x >> 5) * (kSdStages * kSdChunk);
         auto issue = [&](int64_t cs) {
             if (cs < k1) {
-                const int slot = (int)(((cs - k0) / kNarrowChunk) % kNarrowStages) * kNarrowChunk;
+                const int slot = (int)(((cs - k0) / kSdChunk) % kSdStages) * kSdChunk;
 #pragma unroll
-                for (int q = 0; q < kNarrowChunk / 32; ++q) {
+                for (int q = 0; q < kSdChunk / 32; ++q) {
                     const int64_t idx = cs + q * 32 + lane;
                     if (idx < k1) cp_async4(ring + slot + q * 32 + lane, a.col + idx);
                 }
@@ -796,13 +836,13 @@ __global__ void __launch_bounds__(kSpThreads, 3) sddmm_kernel(SddmmArgs a) {
             cp_async_commit();
         };
 #pragma unroll
-        for (int q = 0; q < kNarrowStages - 1; ++q) issue(k0 + (int64_t)q * kNarrowChunk);
-        for (int64_t cs = k0; cs < k1; cs += kNarrowChunk) {
-            issue(cs + (int64_t)(kNarrowStages - 1) * kNarrowChunk);
-            cp_async_wait<kNarrowStages - 1>();
+        for (int q = 0; q < kSdStages - 1; ++q) issue(k0 + (int64_t)q * kSdChunk);
+        for (int64_t cs = k0; cs < k1; cs += kSdChunk) {
+            issue(cs + (int64_t)(kSdStages - 1) * kSdChunk);
+            cp_async_wait<kSdStages - 1>();
             __syncwarp();
-            const int slot = (int)(((cs - k0) / kNarrowChunk) % kNarrowStages) * kNarrowChunk;
-            const int64_t ce = imin<int64_t>(cs + kNarrowChunk, k1);
+            const int slot = (int)(((cs - k0) / kSdChunk) % kSdStages) * kSdChunk;
+            const int64_t ce = imin<int64_t>(cs + kSdChunk, k1);
             for (int64_t kb = cs; kb < ce;) {
                 while (e_row <= kb) {   // the row holding entry kb (empty rows are passed over)
                     ++row;
@@ -1026,7 +1066,7 @@ int weight_grad_sddmm(const csrt_csr *w, const float *dy, const float *x, int32_
 #undef CSRT_SDDMM_CASE
     CSRT_ARG(kern != nullptr, "sddmm: no kernel for vw=%d nv=%d g=%d", vw, nv, g);
     // 2..16 lanes per entry: the per-warp ring of column indices in shared memory
-    const size_t smem = (g > 1 && g < 32) ? (size_t)(kSpThreads / 32) * kNarrowStages * kNarrowChunk * sizeof(int32_t) : 0;
+    const size_t smem = (g > 1 && g < 32) ? (size_t)(kSpThreads / 32) * kSdStages * kSdChunk * sizeof(int32_t) : 0;
     if (wps == 0) {
         int blocks = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, kern, kSpThreads, smem) != cudaSuccess ||
@@ -1127,7 +1167,9 @@ extern "C" int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, fl
     }
     const bool v4 = (n % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15) == 0;
     const bool v2 = (n % 2 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 7) == 0;
-    const SpmmShape sh = spmm_shape(n, (int64_t)w->rows + w->capacity, v4, v2);
+    const bool csr16 =
+        ((reinterpret_cast<uintptr_t>(w->col_idx) | reinterpret_cast<uintptr_t>(w->val)) & 15) == 0;
+    const SpmmShape sh = spmm_shape(n, (int64_t)w->rows + w->capacity, v4, v2, csr16);
     const int64_t carry_floats = (int64_t)sh.units * sh.n_tiles * sh.tn;
     CSRT_ARG(sh.units == 1 || (carry_floats <= kNoAllocFloats && sh.units <= kNoAllocRows),
              "spmm_fwd_noalloc: n = %d needs %lld floats of static scratch, the maximum is %lld", n,
@@ -1148,6 +1190,7 @@ extern "C" int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, fl
     a.bias = nullptr;
     a.relu = 0;
     a.mask = nullptr;
+    a.hdr = nullptr;   // no status word: a wait that gives up is not reported
     const int launched = spmm_dispatch(sh, a, as_stream(stream));
     CSRT_ARG(launched > 0, "spmm_fwd_noalloc: no kernel for shape vw=%d nv=%d g=%d", sh.vw, sh.nv, sh.g);
     count_launch(launched);
