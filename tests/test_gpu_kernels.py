@@ -218,6 +218,49 @@ def test_spmm_fwd_and_bwd_against_oracle(C, m, k, n, density, zipf):
     assert ws.status()[0] == 0
 
 
+class _Shifted:
+    """A CSR whose index and value arrays start 4 bytes past a 16-byte
+    boundary (a caller's sub-array): the narrow kernel's bulk copies need
+    16-byte alignment, so the library takes the 32-lane kernel for it."""
+
+    def __init__(self, C, w):
+        nnz = w.nnz()
+        self.rows, self.cols = w.rows, w.cols
+        self._c = torch.zeros(nnz + 1, dtype=torch.int32, device="cuda")
+        self._v = torch.zeros(nnz + 1, dtype=torch.float32, device="cuda")
+        self._c[1:].copy_(w.col_idx[:nnz])
+        self._v[1:].copy_(w.val[:nnz])
+        assert (self._c[1:].data_ptr() % 16) == 4 and (self._v[1:].data_ptr() % 16) == 4
+        self._s = C.csrt_csr(w.rows, w.cols, max(nnz, 1), C._ptr(w.row_ptr), C._ptr(self._c[1:]),
+                             C._ptr(self._v[1:]), None, None, None, None)
+        self._keep = w
+
+    @property
+    def struct(self):
+        import ctypes
+        return ctypes.byref(self._s)
+
+
+@pytest.mark.parametrize("n", [1, 3, 8, 16])
+def test_spmm_narrow_unaligned_csr_arrays(C, n):
+    m, k = 600, 700
+    rng = np.random.default_rng(90 + n)
+    a = _sparse(rng, m, k, 0.2)
+    x = rng.standard_normal((k, n)).astype(F32)
+    ws = _ws(C, m, k, n)
+    w = _gpu_csr(C, a, ws)
+    ref = O.csr_from_dense(a)
+    want = torch.zeros(m, n, device="cuda")
+    C.spmm_fwd(w, _dev(x), want, ws)            # aligned arrays: the narrow kernel
+    got = torch.zeros(m, n, device="cuda")
+    C.spmm_fwd(_Shifted(C, w), _dev(x), got, ws)   # shifted arrays: the 32-lane kernel
+    lens = np.diff(ref.row_ptr)[:, None]
+    for y in (want, got):
+        assert_close(y.cpu().numpy(), O.spmm_fwd(ref, x), O.spmm_fwd(O.csr_abs(ref), np.abs(x)), lens,
+                     what="spmm_fwd")
+    assert ws.status()[0] == 0
+
+
 @pytest.mark.parametrize("m,k,n,zipf", [(700, 900, 256, True), (129, 257, 70, False), (50, 40, 1, False),
                                          (300, 784, 64, False), (4100, 4100, 256, False), (5000, 5000, 128, True)])
 def test_fused_epilogues_match_unfused(C, m, k, n, zipf):
@@ -357,6 +400,28 @@ def test_prox_bit_exact(C, m, k, density, gscale, eta, lam):
     C.prox_update_compact(w, _dev(g), eta, lam, out, ws)
     ref = O.prox_update_compact(O.csr_from_dense(a), g, eta, lam)
     _check_csr_equal(out, ref)
+    assert ws.status()[0] == 0
+
+
+@pytest.mark.parametrize("m,k,transposed", [(3000, 512, True), (800, 9216, False), (5000, 300, True)])
+def test_prox_mixed_dense_and_sparse_tiles(C, m, k, transposed):
+    """Rows whose G is large keep nearly every entry (their tiles take the
+    one-entry-per-lane pass 2), rows whose G is tiny keep only some stored
+    weights (four-entries-per-lane pass 2): both forms in one call, bit-exact."""
+    rng = np.random.default_rng(m + k)
+    a = _sparse(rng, m, k, 0.1)
+    scale = np.where((np.arange(m) // 37) % 2 == 0, 1.0, 1e-4).astype(F32)[:, None]
+    g = (rng.standard_normal((m, k)).astype(F32) * scale).astype(F32)
+    eta, lam = 0.01, 1e-2
+    ws = _ws(C, m, k, 1)
+    w = _gpu_csr(C, a, ws)
+    out = C.CSR(m, k, transposed=transposed)
+    C.prox_update_compact(w, _dev(g), eta, lam, out, ws)
+    ref = O.prox_update_compact(O.csr_from_dense(a), g, eta, lam)
+    kept = np.diff(ref.row_ptr)
+    assert kept[::2].mean() > 0.5 * k or kept.max() > 0.5 * k   # some tiles dense
+    assert kept.min() < 0.2 * k                                  # some tiles sparse
+    _check_csr_equal(out, ref, transposed=transposed)
     assert ws.status()[0] == 0
 
 
