@@ -591,10 +591,10 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
     // shared: the tile's G (bulk-copied), then z in place, then the kept values
     // (NaN = dropped); a bitmask of the positions that hold a stored weight;
     // the tile's row pointers.
-    extern __shared__ __align__(128) float row_smem[];
-    float *tile_v = row_smem;
+    extern __shared__ __align__(128) float prox_smem[];
+    float *tile_v = prox_smem;
     const int tile_cap = rows_per_tile * a.cols;
-    uint32_t *onbits = reinterpret_cast<uint32_t *>(row_smem + tile_cap);
+    uint32_t *onbits = reinterpret_cast<uint32_t *>(prox_smem + tile_cap);
     int32_t *s_rp = reinterpret_cast<int32_t *>(onbits + (tile_cap + 31) / 32);
     __shared__ __align__(8) uint64_t s_bar;
     __shared__ uint32_t s_wtot[kCThreads / 32];
