@@ -19,7 +19,8 @@ step times.
 
 Also reported: `e2e` (the same step with the batch copied from pinned host
 memory and the loss read back inside the timed region; the library's input
-pipeline copies batch i+1 on a copy stream while step i runs), `roofline` of the
+pipeline copies batch i+1 on a copy stream into one of two device slots while
+step i runs, and a graph per slot reads it in place), `roofline` of the
 dominant kernel (timed with CUDA events in an instrumented eager step),
 `cpu_baseline` (the CPU oracle on a row sample of the same step) and the SM
 clocks sampled during the timed region.
@@ -532,23 +533,38 @@ def main():
         raise SystemExit(f"device status {flags} after the timed steps")
 
     # end to end: pinned host batch -> device, step, loss -> pinned host. The
-    # input pipeline copies batch i+1 on a copy stream while step i runs (its
-    # copy starts after step i's start event, so every copy lies inside a
-    # timed step); batch 0 is copied inside step 0.
+    # input pipeline copies batch i+1 on a copy stream into one of two device
+    # slots while step i runs (its copy starts after step i's start event, so
+    # every copy lies inside a timed step); batch 0 is copied inside step 0.
+    # One graph per slot reads the slot's buffers directly (net.set_input).
+    pf = BatchPrefetcher(net)
+    x_orig, y_orig = net.x_in, net.labels
+    slot_graphs = []
+    for slot in range(2):
+        net.set_input(pf.x[slot], pf.y[slot])
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(s):
+            restore()
+            with torch.cuda.graph(g, stream=s):
+                net.step("prox", eta, lam)
+        slot_graphs.append(g)
+    net.set_input(x_orig, y_orig)
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
     loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
     e_starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     e_ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    pf = BatchPrefetcher(net)
     for i in range(args.steps):
         restore()
         flush.fill_(float(i))
         e_starts[i].record(stream)
         if i == 0:
             pf.issue(x_host, lab_host, after=e_starts[0])
-        pf.load()
+        slot = pf.acquire()
         if i + 1 < args.steps:
             pf.issue(x_host, lab_host, after=e_starts[i])
-        graph.replay()
+        slot_graphs[slot].replay()
+        pf.release(slot)
         loss_host.copy_(net.loss[:1], non_blocking=True)
         e_ends[i].record(stream)
     torch.cuda.synchronize()

@@ -62,7 +62,8 @@ extern "C" {
                                  the CSR written is truncated but structurally valid
                                  (row_ptr clamped to capacity). required_nnz reports
                                  the count that was needed. */
-#define CSRT_DEV_TIMEOUT 2    /* a bounded inter-block wait gave up; results invalid */
+#define CSRT_DEV_TIMEOUT 2    /* a bounded wait (on another block, or on a bulk copy
+                                 into shared memory) gave up; results invalid */
 #define CSRT_DEV_NONFINITE 4  /* the prox step met a NaN in w - eta*G (dropped) */
 #define CSRT_DEV_INVALID 8    /* csrt_validate_csr found a broken invariant */
 
@@ -185,7 +186,11 @@ int csr_transpose(csrt_csr *w, void *ws, size_t ws_bytes, void *stream);
 
 /* spmm_fwd -- Section 3.2.1 (dense x compressed', the forward pass).
  * Y[M x n] = W X[K x n]: Y[i, c] = sum over stored k of row i of
- * val[k] * X[col_idx[k], c], float32 accumulation. Y is overwritten. */
+ * val[k] * X[col_idx[k], c], float32 accumulation. Y is overwritten.
+ * Products with n <= 16 (64 for float4-aligned X and Y) stream col_idx and
+ * val through shared memory with bulk copies when both arrays are 16-byte
+ * aligned (else a 32-lane kernel runs); a copy that does not complete within
+ * the wait's limit sets CSRT_DEV_TIMEOUT. */
 int spmm_fwd(const csrt_csr *w, const float *x, int32_t n, float *y,
              void *ws, size_t ws_bytes, void *stream);
 

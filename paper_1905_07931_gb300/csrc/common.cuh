@@ -165,6 +165,25 @@ __device__ __forceinline__ int64_t warp_first_false(int64_t lo, int64_t hi, Pred
     return lo + __popc(__ballot_sync(0xffffffffu, p));
 }
 
+// Bounded wait for the phase with the given parity of an mbarrier in shared
+// memory (a bulk copy's completion): false if it gave up after kSpinLimit
+// polls, backing off after the first few. Callers flag CSRT_DEV_TIMEOUT.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
+    const uint32_t addr = (uint32_t)__cvta_generic_to_shared(bar);
+    for (unsigned i = 0; i < kSpinLimit; ++i) {
+        uint32_t done;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+            " selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(done)
+            : "r"(addr), "r"(parity)
+            : "memory");
+        if (done) return true;
+        if (i > 16) __nanosleep(32);
+    }
+    return false;
+}
+
 // Two independent searches of warp_first_false, run round by round together
 // so that the latencies of their probes overlap (each round issues both
 // probes before either ballot). Results in ra and rb.

@@ -376,27 +376,13 @@ __global__ void __launch_bounds__(kCThreads) compact_kernel(CompactArgs a) {
 constexpr int kRowBudget = 8192;     // entries per tile when rows are short
 constexpr int kRowMaxK = 16384;      // longest row the row-tile path takes
 
-constexpr unsigned kRowWaitLimit = 1u << 22;
-
 __device__ __forceinline__ uint32_t cvta_smem(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
 // Bounded wait for the phase with the given parity of an mbarrier.
 __device__ __forceinline__ bool row_mbar_wait(uint64_t *bar, uint32_t parity) {
-    const uint32_t addr = cvta_smem(bar);
-    for (unsigned i = 0; i < kRowWaitLimit; ++i) {
-        uint32_t done;
-        asm volatile(
-            "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-            " selp.u32 %0, 1, 0, p;\n}\n"
-            : "=r"(done)
-            : "r"(addr), "r"(parity)
-            : "memory");
-        if (done) return true;
-        if (i > 32) __nanosleep(32);
-    }
-    return false;
+    return mbar_wait_bounded(bar, parity);
 }
 
 // Thread 0 only: stream `bytes` (16-byte aligned source, multiple of 16) into
@@ -868,8 +854,10 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_rows_kernel(CompactArgs a, 
 // The library's bounded waits run against events that never happen (failure
 // detection without a fault): (0) the decoupled look-back of tile 1 while
 // tile 0 never publishes, (1) an mbarrier wait on a barrier nothing arrives
-// on. Each gives up after its iteration limit, sets CSRT_DEV_TIMEOUT (with
-// the site of the wait) and the kernel returns normally.
+// on (mbar_wait_bounded: the waits for the prox kernel's tile copy and for
+// the narrow SpMM's ring chunks). Each gives up after its iteration limit,
+// sets CSRT_DEV_TIMEOUT (with the site of the wait) and the kernel returns
+// normally.
 __global__ void bounded_wait_check_kernel(unsigned long long *__restrict__ status, WsHeader *hdr, int which) {
     pdl_enter();
     __shared__ __align__(8) uint64_t bar;

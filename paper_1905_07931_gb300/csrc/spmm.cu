@@ -311,22 +311,6 @@ __device__ __forceinline__ void sp_bulk_copy(void *dst, const void *src, uint32_
                  "l"(src), "r"(bytes), "r"(sp_smem_addr(bar))
                  : "memory");
 }
-// Bounded wait for the phase of the given parity; false if it gave up.
-__device__ __forceinline__ bool sp_bar_wait(uint64_t *bar, uint32_t parity) {
-    const uint32_t addr = sp_smem_addr(bar);
-    for (unsigned i = 0; i < kSpinLimit; ++i) {
-        uint32_t done;
-        asm volatile(
-            "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-            " selp.u32 %0, 1, 0, p;\n}\n"
-            : "=r"(done)
-            : "r"(addr), "r"(parity)
-            : "memory");
-        if (done) return true;
-        if (i > 16) __nanosleep(32);
-    }
-    return false;
-}
 
 template <int VW, int G>
 __global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
@@ -448,7 +432,7 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_group_kernel(SpmmArgs a) {
         const int64_t A = abase + j * kNarrowChunk;
         if (A >= k1) break;
         issue(j + kNarrowStages - 1);
-        if (!sp_bar_wait(bars + j % kNarrowStages, (uint32_t)((j / kNarrowStages) & 1))) failed = true;
+        if (!mbar_wait_bounded(bars + j % kNarrowStages, (uint32_t)((j / kNarrowStages) & 1))) failed = true;
         __syncwarp();
         const int slot = (int)(j % kNarrowStages) * kNarrowChunk;
         const int64_t ce = imin<int64_t>(A + kNarrowChunk, k1);

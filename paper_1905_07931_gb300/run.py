@@ -165,10 +165,12 @@ def run(config: str, prox_steps: int, debias_steps: int, seed: int = 0, batches:
                 # of the next one overlaps this step
                 if step == 0:
                     pf.issue(*pool[0], after=st)
-                pf.load()
+                slot = pf.acquire()
+                net.set_input(pf.x[slot], pf.y[slot])   # the step reads the slot in place
                 if step + 1 < total:
                     pf.issue(*pool[(step + 1) % len(pool)], after=st)
                 lt = net.step(phase, eta, lam)
+                pf.release(slot)
                 batch = net.batch
             en.record(stream)
             torch.cuda.synchronize()

@@ -156,6 +156,23 @@ class SparseNet:
         L = self.params[li]
         return L["W"][L["cur"]]
 
+    def set_input(self, x_in: torch.Tensor, labels: torch.Tensor):
+        """Point the network at other device buffers for its input batch and
+        labels (same shapes and dtypes as ``x_in`` / ``labels``); a step
+        captured in a graph afterwards reads them directly."""
+        if x_in.shape != self.x_in.shape or x_in.dtype != self.x_in.dtype or x_in.device != self.x_in.device:
+            raise ValueError(f"input {tuple(x_in.shape)} {x_in.dtype} does not match {tuple(self.x_in.shape)}")
+        if labels.shape != self.labels.shape or labels.dtype != self.labels.dtype:
+            raise ValueError("labels do not match")
+        if not (x_in.is_contiguous() and labels.is_contiguous()):
+            raise ValueError("input buffers must be contiguous")
+        old = self.x_in
+        for L in self.layers:
+            for key in ("x", "xmat"):
+                if L.get(key) is old:
+                    L[key] = x_in
+        self.x_in, self.labels = x_in, labels
+
     def forward(self):
         s = self.stream
         for L in self.layers:
@@ -260,15 +277,20 @@ class SparseNet:
 
 class BatchPrefetcher:
     """Input pipeline of a SparseNet: batch i+1 is copied from pinned host
-    memory into one of two device slots on a copy stream while step i runs;
-    ``load`` then hands a slot to the network (``x_in`` / ``labels``) with a
-    device-to-device copy on the network's stream. The network keeps reading
-    ``x_in`` until its last weight gradient, so the next batch cannot be
-    copied into ``x_in`` itself while a step is in flight.
+    memory into one of two device slots on a copy stream while step i runs.
+    Two ways to hand a slot to the network:
 
-      pf.issue(x0, y0, after=start_event)          # batch 0
+    * ``load()``: a device-to-device copy into the network's ``x_in`` /
+      ``labels`` on its stream (the network keeps reading ``x_in`` until its
+      last weight gradient, so the next batch cannot be copied into ``x_in``
+      itself while a step is in flight);
+    * ``acquire()`` / ``release(slot)``: the step reads the slot's buffers
+      directly (``net.set_input(pf.x[slot], pf.y[slot])``, e.g. one captured
+      graph per slot), no copy.
+
+      pf.issue(x0, y0, after=start_event)            # batch 0
       for i in range(steps):
-          pf.load(i)                                # waits for batch i's copy
+          pf.load()                                   # waits for batch i's copy
           if i + 1 < steps: pf.issue(x[i+1], y[i+1])  # overlaps step i
           net.step(...)
     """
@@ -283,11 +305,14 @@ class BatchPrefetcher:
         self.issued = 0
         self.loaded = 0
 
+    def _stream(self):
+        return self.net.stream or torch.cuda.current_stream()
+
     def issue(self, x_host: torch.Tensor, y_host: torch.Tensor, after: torch.cuda.Event | None = None):
         """Enqueue the host-to-device copy of the next batch (pinned host
         tensors of the shapes of ``x_in`` and ``labels``); the copy starts
         after ``after`` (an event on the network's stream) if given, and after
-        the slot's previous batch has been loaded."""
+        the slot's previous batch has been released."""
         slot = self.issued % 2
         cs = self.copy_stream
         if after is not None:
@@ -299,18 +324,29 @@ class BatchPrefetcher:
             self.ready[slot].record(cs)
         self.issued += 1
 
-    def load(self):
-        """Make the oldest issued batch the network's input, on its stream."""
+    def acquire(self) -> int:
+        """Make the network's stream wait for the oldest issued batch; returns
+        its slot (the step then reads ``x[slot]`` / ``y[slot]``)."""
         if self.loaded >= self.issued:
             raise RuntimeError("no batch issued")
         slot = self.loaded % 2
-        s = self.net.stream or torch.cuda.current_stream()
-        s.wait_event(self.ready[slot])
+        self._stream().wait_event(self.ready[slot])
+        self.loaded += 1
+        return slot
+
+    def release(self, slot: int):
+        """The work that reads the slot is enqueued: its next copy may follow it."""
+        self.free[slot].record(self._stream())
+
+    def load(self):
+        """Make the oldest issued batch the network's input (copied into
+        ``x_in`` / ``labels`` on its stream)."""
+        slot = self.acquire()
+        s = self._stream()
         with torch.cuda.stream(s):
             self.net.x_in.copy_(self.x[slot])
             self.net.labels.copy_(self.y[slot])
-            self.free[slot].record(s)
-        self.loaded += 1
+        self.release(slot)
 
 
 def mlp_layers(n_layers: int):

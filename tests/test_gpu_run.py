@@ -75,35 +75,47 @@ def test_load_rejects_a_broken_checkpoint(R, tmp_path):
 
 def test_prefetched_batches_match_direct_copies(R):
     """The input pipeline (copy of batch i+1 on a copy stream while step i
-    runs) feeds every step the same batch as a plain copy before the step."""
+    runs) feeds every step the same batch as a plain copy before the step,
+    whether the slot is copied into the network's input (load) or the
+    network reads the slot itself (set_input + acquire / release)."""
     from paper_1905_07931_gb300.train import BatchPrefetcher
     cfg_pool = None
     losses, finals = [], []
-    for mode in ("direct", "prefetch"):
+    for mode in ("direct", "load", "bound"):
         net, cfg = R.build("mlp", seed=3, precision=1)
         if cfg_pool is None:
             cfg_pool = R._pool("mlp", cfg, 3, seed=3)
-        pf = BatchPrefetcher(net) if mode == "prefetch" else None
+        pf = BatchPrefetcher(net) if mode != "direct" else None
         out = []
         for i in range(5):
             x, y = cfg_pool[i % 3]
+            slot = None
             if pf is None:
                 net.x_in.copy_(x.view(net.x_in.shape), non_blocking=True)
                 net.labels.copy_(y, non_blocking=True)
             else:
                 if i == 0:
                     pf.issue(x, y)
-                pf.load()
+                if mode == "load":
+                    pf.load()
+                else:
+                    slot = pf.acquire()
+                    net.set_input(pf.x[slot], pf.y[slot])
                 if i + 1 < 5:
                     pf.issue(*cfg_pool[(i + 1) % 3])
             lt = net.step("prox", 0.01, 1e-4)
+            if slot is not None:
+                pf.release(slot)
             out.append(float(lt[0].item()))
         torch.cuda.synchronize()
         losses.append(out)
         finals.append([W.to_host()[0] for W in R.weights(net)])
-    assert losses[0] == losses[1]
-    for a, b in zip(*finals):
-        for u, v in zip(a, b):
-            np.testing.assert_array_equal(u, v)
+    assert losses[0] == losses[1] == losses[2]
+    for other in finals[1:]:
+        for a, b in zip(finals[0], other):
+            for u, v in zip(a, b):
+                np.testing.assert_array_equal(u, v)
     with pytest.raises(RuntimeError, match="no batch"):
         BatchPrefetcher(net).load()
+    with pytest.raises(ValueError):
+        net.set_input(torch.zeros(3, device="cuda"), net.labels)
