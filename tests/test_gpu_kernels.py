@@ -388,6 +388,9 @@ def test_prox_hand_cases_on_gpu(C):
     (4100, 512, 0.05, 1.0, 0.01, 1e-4),
     (700, 900, 0.5, 0.1, 0.1, 1.0),
     (20000, 784, 0.05, 1.0, 0.01, 1e-2),   # 2000 row tiles: several per resident block
+    (2000, 20, 0.3, 1.0, 0.01, 1e-4),      # dense tiles of short rows: a 32-entry step spans 2-3 rows
+    (3000, 8, 0.5, 1.0, 0.01, 1e-4),       # ... 4-5 rows
+    (1500, 36, 0.2, 1.0, 0.01, 1e-4),      # K >= 32, not a multiple of 32
     (1500, 9216, 0.05, 1.0, 0.01, 1e-4),   # one-row tiles, dense output
 ])
 def test_prox_bit_exact(C, m, k, density, gscale, eta, lam):
