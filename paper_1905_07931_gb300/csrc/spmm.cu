@@ -15,9 +15,10 @@
 // warp moves 512*NV contiguous bytes per nonzero. Column indices and values
 // are loaded 32 at a time, coalesced, and broadcast with shuffles; four
 // nonzeros are in flight per lane. A row cut by a unit boundary leaves a
-// partial sum ("carry") in the workspace; a fix-up kernel adds the carries of
-// each cut row in unit order, so the result is deterministic and no float
-// atomics are used. Narrow products (n <= 16 floats per vector width) put a
+// partial sum ("carry") in the workspace; the carries of each cut row are
+// added in unit order (by the last of the row's units to finish, counted in
+// the workspace, or by a fix-up kernel), so the result is deterministic and
+// no float atomics are used. Narrow products (n <= 16 floats per vector width) put a
 // group of G < 32 lanes on each nonzero instead (spmm_group_kernel), and the
 // SDDMM uses the same grouped layout.
 #include "common.cuh"
@@ -286,10 +287,9 @@ __global__ void __launch_bounds__(kSpThreads, 3) spmm_merge_kernel(SpmmArgs a) {
 // far below the HBM rate that its CSR stream could reach. Here a group of
 // G lanes (G*VW >= n) takes one nonzero, so a warp step covers E = 32/G
 // nonzeros and a batch of U steps B = U*E nonzeros, cut at row ends. The
-// column indices and values arrive ahead of their use: with G = 1 the next
-// batch is loaded into registers while the current one is consumed; with
-// G >= 2 they stream through a per-warp ring of cp.async chunks in shared
-// memory (see below). At the end of a row the groups' partial sums are
+// column indices and values arrive ahead of their use through a per-warp
+// ring of chunks in shared memory filled by bulk asynchronous copies (see
+// below). At the end of a row the groups' partial sums are
 // combined by a butterfly over the lane bits above G. The unit split, the
 // row-end window and the shared-row protocol are those of spmm_merge_kernel
 // (carries of TN = G*VW floats).

@@ -182,10 +182,8 @@ SPMM_CASES = [
     (1000, 600, 48, 0.1, True),
     (300, 2000, 64, 0.2, False),
     (90, 70, 9, 0.0, False),
-    # row-tiled wide products (n % 64 == 0, >= 2432 rows at n = 256, density
-    # >= 1/32): power-law rows (the long ones left to the long-row kernel),
-    # a partial last chunk of X rows, n = 1024 and 128, and a product just
-    # below the density threshold (taken by the merge-path kernels)
+    # wide products with thousands of rows at n = 128 to 1024: power-law
+    # rows, a ragged last block of X rows, densities from 2% to 30%
     (2600, 300, 256, 0.2, True),
     (5000, 600, 128, 0.3, True),
     (2500, 2000, 256, 0.04, False),
