@@ -593,7 +593,15 @@ def main():
         cands.append({"bound": "alu", "achieved": round(flops / t_s / 1e12, 2), "peak": round(peak, 1),
                       "unit": "TFLOP/s", "frac": round(flops / t_s / 1e12 / peak, 4),
                       "peak_source": "measured FP32 FMA rate (library probe, fma_peak_kernel)"})
-    if dom["name"] in ("weight_grad_dense", "weight_grad_prox_update") and dom["info"].get("n"):
+    if dom["name"] in ("weight_grad_dense", "weight_grad_prox_update") and dom["info"].get("n") \
+            and args.precision == "fp32":
+        # --precision fp32: the contraction runs on the FP32 CUDA cores
+        flops = 2.0 * dom["info"]["M"] * dom["info"]["K"] * dom["info"]["n"]
+        peak = C.fma_peak_tflops()
+        cands.append({"bound": "alu", "achieved": round(flops / t_s / 1e12, 2), "peak": round(peak, 1),
+                      "unit": "TFLOP/s", "frac": round(flops / t_s / 1e12 / peak, 4),
+                      "peak_source": "measured FP32 FMA rate (library probe, fma_peak_kernel)"})
+    elif dom["name"] in ("weight_grad_dense", "weight_grad_prox_update") and dom["info"].get("n"):
         # a TF32 contraction: its peak is the cuBLAS TF32 rate measured here (the
         # measured bf16 rate x the nominal tf32/bf16 ratio 1.1/2.25 beside it);
         # algorithmic flops 2MKN (the fused op's second pass recomputes them: not counted)
