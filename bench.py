@@ -615,7 +615,15 @@ def main():
     cands.sort(key=lambda c: -c["frac"])
     roof = dict(cands[0]) if cands else None
     if roof is not None:
-        roof.update({"traffic": recorded_traffic(dom["label"]), "kernel": kernel, "op": dom["label"],
+        # the committed traffic record is of the default configuration (TF32,
+        # fused path, SGD): the sparse products run the same kernels under
+        # every option, the gradient + prox ops do not
+        same_kernels = dom["name"] in ("spmm_fwd", "spmm_bwd_t", "spmm_fwd_bias_act", "spmm_bwd_t_relu") or (
+            args.precision == "tf32" and args.prox_path == "fused" and args.optimizer == "sgd")
+        if args.precision == "fp32" and dom["name"] == "weight_grad_prox_update":
+            kernel = "gemm_nt_f32_kernel + prox_rows_kernel (the op's unfused route at FP32)"
+        roof.update({"traffic": recorded_traffic(dom["label"]) if same_kernels else None, "kernel": kernel,
+                     "op": dom["label"],
                      "algorithmic_bytes": int(bytes_) if bytes_ else None, "launch_ms": round(dom["ms"], 4)})
         if len(cands) > 1:
             roof["other"] = {k: cands[1][k] for k in ("bound", "achieved", "peak", "unit", "frac")}
