@@ -64,6 +64,10 @@ def parse_args():
     p.add_argument("--record-traffic", metavar="CSV",
                    help="write profiles/traffic.json from an ncu CSV of this bench (dram__bytes_read.sum, "
                         "dram__bytes_write.sum, gpu__time_duration.sum; --steps 1 --warmup 1) and exit")
+    p.add_argument("--clocks-csv", default=None,
+                   help="where nvidia-smi writes its clock samples (default: a file in the system temp dir)")
+    p.add_argument("--no-kernels", action="store_true",
+                   help="skip the per-kernel HBM measurements on the 4096 x 4096 and 4096 x 9216 layers")
     p.add_argument("--optimizer", choices=["sgd", "rmsprop", "adam"], default="sgd",
                    help="proximal method of the prox phase: SGD, Prox-RMSProp (Algorithm 1) or Prox-ADAM "
                         "(Algorithm 2); the adaptive ones take the unfused gradient + prox calls")
@@ -119,8 +123,9 @@ class OracleSample:
         new_rp[1:] = np.cumsum(lens)
         return O.CSR(len(rows), w.cols, new_rp.astype(np.int32), w.col_idx[idx], w.val[idx])
 
-    def step(self) -> float:
-        """Run one sample; return the estimated seconds of one full step."""
+    def step(self):
+        """Run one sample; return (measured seconds of the sample, estimated
+        seconds of one full step = the row-separable part x F + the loss)."""
         O, np = self.O, self.np
         t0 = time.perf_counter()
         for L in self.layers:
@@ -141,12 +146,22 @@ class OracleSample:
                 O.csr_transpose(new)
             L["delta"].sum(axis=1)
         t_rows += time.perf_counter() - t2
-        return t_rows * self.F + t_once
+        return t_rows + t_once, t_rows * self.F + t_once
 
     def describe(self) -> str:
         return (f"CPU oracle (numpy, float64 sums) on every operation of one step restricted to 1/{self.F} "
                 f"of each layer's output rows (forward, loss, weight gradient, W^T dY, prox + compaction, "
-                f"transposed pattern); time x {self.F}")
+                f"transposed pattern); the row-separable time x {self.F} + the loss once")
+
+
+def workload_config(world: int, precision: str = "tf32", prox_path: str = "fused", optimizer: str = "sgd") -> dict:
+    """The `config` of both arms' lines: the workload and its settings."""
+    return {"workload": WORKLOAD, "global_batch": BATCH * world, "per_gpu_batch": BATCH,
+            "layers": list(SIZES), "densities": list(DENSITIES),
+            "weight_grad": "tf32 tcgen05" if precision == "tf32" else "fp32 simt",
+            "prox_path": prox_path if optimizer == "sgd" else "unfused", "optimizer": optimizer,
+            "l2": "flushed between steps (256 MB write, outside the timed region)",
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU"}
 
 
 def cpu_cores() -> int:
@@ -165,16 +180,21 @@ def run_reference(args):
     samp = OracleSample(cfg, fraction_denominator=8)
     for _ in range(args.warmup):
         samp.step()
-    times = [samp.step() for _ in range(args.steps)]
-    total = sum(times)
-    value = args.steps * BATCH / total
+    runs = [samp.step() for _ in range(args.steps)]
+    measured = sum(r[0] for r in runs)          # seconds the timed steps took (1/8-row samples)
+    estimated = sum(r[1] for r in runs)         # the same steps scaled to whole steps
+    # each timed step is one 1/8-row sample of the workload's step: it counts
+    # as the samples of the batch it covers in full-step time
+    value = args.steps * BATCH / estimated
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * measured / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": WORKLOAD, "global_batch": BATCH, "parallelism": "none"},
+        "data": "synthetic", "config": workload_config(world),
         "cpu_baseline": {"kind": "oracle", "value": value, "unit": UNIT, "cores": cpu_cores(),
-                         "sample": samp.describe()},
+                         "sample": samp.describe() + f"; each step is one sample, {args.steps} timed",
+                         "measured_s": round(measured, 3), "scale_factor": samp.F,
+                         "estimated_full_step_ms": round(1e3 * estimated / args.steps, 1)},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -190,10 +210,11 @@ class ClockSampler:
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, path=None):
+        import tempfile
         self.gpu = gpu_index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
+        self.path = path or os.path.join(tempfile.gettempdir(), f"csrtrain_clocks_gpu{gpu_index}_{os.getpid()}.csv")
 
     def start(self):
         try:
@@ -421,6 +442,37 @@ def record_traffic(csv_path: str, out_path: str) -> dict:
 
 
 # ---------------------------------------------------------------------------
+# The sparse kernels on the largest sparse layers (the metric's second half)
+# ---------------------------------------------------------------------------
+
+KERNEL_OF_OP = {"spmm_fwd": "spmm_group_kernel", "spmm_bwd_t": "spmm_group_kernel", "sddmm": "sddmm_kernel",
+                "prox (lambda=1e-4)": "prox_rows_kernel", "prox (lambda*)": "prox_rows_kernel"}
+
+
+def measure_kernels(hbm_peak: float, reps: int = 20):
+    """SpMM, SpMM^T and SDDMM at n = 1 on the 4096 x 4096 sweep layer at 5%
+    and 50% (uniform rows), and the prox step at lambda = 1e-4 (dense output)
+    and at the density-preserving lambda* on the same layers (with the
+    transposed copy) and on the 4096 x 9216 first layer of the classifier head
+    (without it, as the step runs it). Each call timed alone with CUDA events,
+    the 256 MB L2 flush written before every launch, median of `reps`;
+    algorithmic bytes count each operand once (the sweep's formulas)."""
+    from paper_1905_07931_gb300 import sweep
+    out = []
+    cases = [(4096, 4096, 0.05, {"spmm_fwd", "spmm_bwd_t", "sddmm", "prox"}, [1], True),
+             (4096, 4096, 0.50, {"spmm_fwd", "spmm_bwd_t", "sddmm", "prox"}, [1], True),
+             (4096, 9216, 0.05, {"prox"}, [1], False)]
+    for m, k, d, ops, batches, transposed in cases:
+        for r in sweep.run_layer(m, k, d, False, batches, ops, reps, transposed=transposed):
+            gbs = r["bytes"] / (r["us"] / 1e6) / 1e9
+            out.append({"kernel": KERNEL_OF_OP.get(r["op"], r["op"]), "op": r["op"], "m": m, "k": k,
+                        "density": d, "n": r["n"], "transposed_copy": transposed if r["op"].startswith("prox") else None,
+                        "nnz": r["nnz"], "nnz_out": r.get("nnz_out"), "algorithmic_bytes": int(r["bytes"]),
+                        "us": r["us"], "gbs": round(gbs, 1), "hbm_frac": round(gbs / hbm_peak, 4)})
+    return out
+
+
+# ---------------------------------------------------------------------------
 # Multi-rank bookkeeping (replicas: no collective on the data path)
 # ---------------------------------------------------------------------------
 
@@ -516,7 +568,7 @@ def main():
     stream = torch.cuda.current_stream()
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    clocks = ClockSampler(local_rank)
+    clocks = ClockSampler(local_rank, args.clocks_csv)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -661,14 +713,8 @@ def main():
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(total_max_ms / args.steps, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "global_batch": BATCH * world, "per_gpu_batch": BATCH,
-                   "layers": list(SIZES), "densities": list(DENSITIES),
-                   "weight_grad": "tf32 tcgen05" if prec == C.CSRT_PREC_TF32 else "fp32 simt",
-                   "prox_path": args.prox_path if args.optimizer == "sgd" else "unfused",
-                   "optimizer": args.optimizer,
-                   "l2": "flushed between steps (256 MB write, outside the timed region)",
-                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                   "step_ops": [r["label"] for r in prof]},
+        "config": dict(workload_config(world, args.precision, args.prox_path, args.optimizer),
+                       step_ops=[r["label"] for r in prof]),
         "e2e": {"value": round(e2e_value, 1), "unit": UNIT,
                 "h2d_bytes_per_step": int(x_host.numel() * 4 + lab_host.numel() * 4), "d2h_bytes_per_step": 4},
         "gpu_launches": int(launches_per_step * args.steps),
@@ -677,12 +723,19 @@ def main():
         "clocks": clk,
         "wall_s_timed_region": round(wall, 3),
     }
+    if rank == 0 and not args.no_kernels:
+        line["kernels"] = measure_kernels(peaks["hbm_gbs"])
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         samp = OracleSample(cfg, fraction_denominator=4)
-        est = [samp.step() for _ in range(2)]
+        samp.step()
+        runs = [samp.step() for _ in range(5)]
+        est = [r[1] for r in runs]
         v = BATCH / (sum(est) / len(est))
         line["cpu_baseline"] = {"value": round(v, 3), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
-                                "sample": samp.describe() + ", 2 samples"}
+                                "sample": samp.describe() + ", mean of 5 samples after one untimed",
+                                "measured_s": round(sum(r[0] for r in runs), 3), "samples": len(runs),
+                                "scale_factor": samp.F,
+                                "estimated_full_step_ms": round(1e3 * sum(est) / len(est), 1)}
     if args.profile_ops and rank == 0:
         for r in prof:
             b = op_bytes(r["name"], r["info"])

@@ -221,11 +221,22 @@ int spmm_bwd_t_relu(const csrt_csr *w, const float *dy, int32_t n, const float *
  * rejected with CSRT_ERR_ARG). The scratch for rows split between work units
  * lives in a fixed device array inside the library (8 MiB of floats + 256 KiB
  * of row slots, held by every GPU that loads the library until the process
- * exits). The
- * first call on a device looks the array up with cudaGetSymbolAddress (make
- * it before any stream capture). All calls share the array: calls whose
- * kernels overlap on the GPU race and must be serialised by the caller. */
+ * exits). A call needs (units x n-tiles) x (columns per tile) floats of it,
+ * at most (SMs x 32 + n-tiles) x 256, so every n <= 4096 fits on GPUs of up
+ * to 255 SMs; a shape that does not fit is rejected with CSRT_ERR_ARG. A
+ * bounded wait that gives up sets CSRT_DEV_TIMEOUT in the library's own
+ * status word (read it with spmm_fwd_noalloc_status). The first call of
+ * either entry point on a device looks the arrays up with
+ * cudaGetSymbolAddress (make it before any stream capture). All calls share
+ * the array: calls whose kernels overlap on the GPU race and must be
+ * serialised by the caller. */
 int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, float *y, void *stream);
+
+/* spmm_fwd_noalloc_status -- synchronise `stream`, then copy the status word
+ * of spmm_fwd_noalloc (its own, not a workspace's: CSRT_DEV_TIMEOUT if a
+ * bounded wait of any call since the last clear gave up) to *flags (host).
+ * clear != 0 then zeroes it. Allocates nothing. */
+int spmm_fwd_noalloc_status(int32_t *flags, int32_t clear, void *stream);
 
 /* weight_grad_dense -- gradient of every weight for the prox phase (the
  * matrix w - eta*G of Section 3.3 needs G at all M x K entries).

@@ -21,6 +21,8 @@
 // no float atomics are used. Narrow products (n <= 16 floats per vector width) put a
 // group of G < 32 lanes on each nonzero instead (spmm_group_kernel), and the
 // SDDMM uses the same grouped layout.
+#include <mutex>
+
 #include "common.cuh"
 
 namespace csrt {
@@ -1108,16 +1110,22 @@ extern "C" int debias_update(csrt_csr *w, const float *g_nnz, float eta, void *s
 //
 // Limits and rules:
 //  * The product may have at most kNoAllocMaxN = 4096 columns (n); larger n
-//    is rejected with CSRT_ERR_ARG. The array holds kNoAllocFloats floats of
-//    partial sums (8 MiB) and kNoAllocRows row slots (256 KiB), enough for
-//    n <= 4096 on GPUs of up to 256 SMs (a shape that still does not fit is
-//    rejected the same way). Every GPU that loads the library holds the
-//    array until the process exits.
-//  * The first call on each device looks up the array's device address with
-//    cudaGetSymbolAddress (once per device, with that device current); make
-//    that first call before any stream capture begins.
+//    is rejected with CSRT_ERR_ARG. The array holds kNoAllocFloats = 2^21
+//    floats of partial sums (8 MiB) and kNoAllocRows = 2^16 row slots
+//    (256 KiB). A call needs (units x n_tiles) x tn floats, where units x
+//    n_tiles is at most SMs x 32 + n_tiles and tn at most 256, so every
+//    n <= 4096 fits on GPUs of up to 255 SMs (GB300 has 152); a shape that
+//    does not fit is rejected the same way. Every GPU that loads the library
+//    holds the array until the process exits.
+//  * A 256-byte status word beside the array collects CSRT_DEV_TIMEOUT when a
+//    bounded wait of the product gives up (the result is then invalid);
+//    spmm_fwd_noalloc_status reads and optionally clears it.
+//  * The first call of either entry point on a device looks up the device
+//    addresses with cudaGetSymbolAddress (once per device, guarded by a
+//    std::call_once, with that device current); make that first call before
+//    any stream capture begins.
 //  * All calls share the one array and it keeps the last call's contents.
-//    Nothing in it needs to start at zero: each launch writes every slot it
+//    The partial sums need no clearing: each launch writes every slot it
 //    later reads. Calls whose kernels overlap on the GPU (two streams, or two
 //    threads) race on the array and give wrong results; serialise them.
 // ---------------------------------------------------------------------------
@@ -1125,10 +1133,52 @@ namespace csrt {
 constexpr int32_t kNoAllocMaxN = 4096;
 constexpr int64_t kNoAllocFloats = (int64_t)1 << 21;
 constexpr int64_t kNoAllocRows = (int64_t)1 << 16;
+constexpr int kNoAllocMaxDevices = 64;
 static __device__ __align__(256) float g_noalloc_carry[kNoAllocFloats];
 static __device__ __align__(256) int32_t g_noalloc_carry_row[kNoAllocRows];
-static float *g_noalloc_carry_addr[64] = {nullptr};
-static int32_t *g_noalloc_row_addr[64] = {nullptr};
+static __device__ __align__(256) WsHeader g_noalloc_status;
+
+struct NoAllocAddrs {
+    float *carry = nullptr;
+    int32_t *carry_row = nullptr;
+    WsHeader *status = nullptr;
+    cudaError_t err = cudaSuccess;
+};
+static NoAllocAddrs g_noalloc_addrs[kNoAllocMaxDevices];
+static std::once_flag g_noalloc_once[kNoAllocMaxDevices];
+
+// The device addresses of the static arrays on the current device, looked
+// up once per device; returns nullptr (with the message set) on failure.
+static const NoAllocAddrs *noalloc_addrs() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        fail(CSRT_ERR_CUDA, "cudaGetDevice failed");
+        return nullptr;
+    }
+    if (dev < 0 || dev >= kNoAllocMaxDevices) {
+        fail(CSRT_ERR_ARG, "device ordinal %d out of range", dev);
+        return nullptr;
+    }
+    std::call_once(g_noalloc_once[dev], [dev] {
+        NoAllocAddrs &a = g_noalloc_addrs[dev];
+        void *p = nullptr, *q = nullptr, *r = nullptr;
+        a.err = cudaGetSymbolAddress(&p, g_noalloc_carry);
+        if (a.err == cudaSuccess) a.err = cudaGetSymbolAddress(&q, g_noalloc_carry_row);
+        if (a.err == cudaSuccess) a.err = cudaGetSymbolAddress(&r, g_noalloc_status);
+        if (a.err == cudaSuccess) {
+            a.carry = static_cast<float *>(p);
+            a.carry_row = static_cast<int32_t *>(q);
+            a.status = static_cast<WsHeader *>(r);
+        }
+    });
+    const NoAllocAddrs &a = g_noalloc_addrs[dev];
+    if (a.err != cudaSuccess) {
+        fail(CSRT_ERR_CUDA, "cudaGetSymbolAddress of the static scratch failed on device %d: %s", dev,
+             cudaGetErrorString(a.err));
+        return nullptr;
+    }
+    return &a;
+}
 }  // namespace csrt
 
 extern "C" int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, float *y, void *stream) {
@@ -1139,16 +1189,8 @@ extern "C" int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, fl
              n, kNoAllocMaxN);
     CSRT_ARG((x && y) || n == 0 || w->rows == 0, "X or Y is NULL");
     if (w->rows == 0 || n == 0) return CSRT_OK;
-    int dev = 0;
-    CSRT_CHECK_CUDA(cudaGetDevice(&dev));
-    CSRT_ARG(dev >= 0 && dev < 64, "device ordinal %d out of range", dev);
-    if (g_noalloc_carry_addr[dev] == nullptr) {
-        void *p = nullptr, *q = nullptr;
-        CSRT_CHECK_CUDA(cudaGetSymbolAddress(&p, g_noalloc_carry));
-        CSRT_CHECK_CUDA(cudaGetSymbolAddress(&q, g_noalloc_carry_row));
-        g_noalloc_carry_addr[dev] = static_cast<float *>(p);
-        g_noalloc_row_addr[dev] = static_cast<int32_t *>(q);
-    }
+    const NoAllocAddrs *na = noalloc_addrs();
+    if (na == nullptr) return CSRT_ERR_CUDA;
     const bool v4 = (n % 4 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15) == 0;
     const bool v2 = (n % 2 == 0) && ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 7) == 0;
     const bool csr16 =
@@ -1168,15 +1210,31 @@ extern "C" int spmm_fwd_noalloc(const csrt_csr *w, const float *x, int32_t n, fl
     a.y = y;
     a.units = sh.units;
     a.n_tiles = sh.n_tiles;
-    a.carry = g_noalloc_carry_addr[dev];
-    a.carry_row = g_noalloc_row_addr[dev];
+    a.carry = na->carry;
+    a.carry_row = na->carry_row;
     a.cnt = nullptr;   // shared rows are completed by the fix-up kernel
     a.bias = nullptr;
     a.relu = 0;
     a.mask = nullptr;
-    a.hdr = nullptr;   // no status word: a wait that gives up is not reported
+    a.hdr = na->status;   // a bounded wait that gives up sets CSRT_DEV_TIMEOUT here
     const int launched = spmm_dispatch(sh, a, as_stream(stream));
     CSRT_ARG(launched > 0, "spmm_fwd_noalloc: no kernel for shape vw=%d nv=%d g=%d", sh.vw, sh.nv, sh.g);
     count_launch(launched);
     return check_launch("spmm_fwd_noalloc");
+}
+
+extern "C" int spmm_fwd_noalloc_status(int32_t *flags, int32_t clear, void *stream) {
+    CSRT_ARG(flags != nullptr, "flags is NULL");
+    const NoAllocAddrs *na = noalloc_addrs();
+    if (na == nullptr) return CSRT_ERR_CUDA;
+    cudaStream_t s = as_stream(stream);
+    CSRT_CHECK_CUDA(cudaStreamSynchronize(s));
+    unsigned int word = 0;
+    CSRT_CHECK_CUDA(cudaMemcpy(&word, &na->status->flags, sizeof(word), cudaMemcpyDeviceToHost));
+    *flags = (int32_t)word;
+    if (clear) {
+        CSRT_CHECK_CUDA(cudaMemsetAsync(na->status, 0, sizeof(WsHeader), s));
+        CSRT_CHECK_CUDA(cudaStreamSynchronize(s));
+    }
+    return CSRT_OK;
 }

@@ -52,6 +52,7 @@ _SIGS = {
                           c_void_p],
     "spmm_bwd_t_relu": [POINTER(csrt_csr), c_void_p, c_int32, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p],
     "spmm_fwd_noalloc": [POINTER(csrt_csr), c_void_p, c_int32, c_void_p, c_void_p],
+    "spmm_fwd_noalloc_status": [POINTER(c_int32), c_int32, c_void_p],
     "weight_grad_dense": [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32, c_void_p,
                           c_size_t, c_void_p],
     "weight_grad_sddmm": [POINTER(csrt_csr), c_void_p, c_void_p, c_int32, c_void_p, c_void_p, c_size_t,

@@ -4,8 +4,9 @@ Float32 results pass if |gpu - ref| <= atol + rtol*|ref| (rtol 1e-4, atol
 1e-6; rtol 1e-3 for TF32 tensor-core products). An entry that misses this
 (cancellation: |ref| much smaller than the terms it sums) must still meet the
 worst-case summation bound |gpu - ref| <= gamma_n * S + unit*|ref|, where
-S = sum |terms| (computed by the oracle on |W| and |X|), n the number of
-terms, gamma_n = n*u / (1 - n*u) with u = 2^-24, and for TF32 operands an
+S = sum |terms| (computed by the oracle on |W| and |X|; ``bound`` may be a
+callable returning S, evaluated only when some entry misses the first test),
+n the number of terms, gamma_n = n*u / (1 - n*u) with u = 2^-24, and for TF32 operands an
 extra 2 * 2^-10 * S for the truncation of both factors. Integer arrays and
 sparsity patterns are compared bit for bit.
 """
@@ -37,6 +38,8 @@ def assert_close(gpu, ref, bound=None, n_terms=None, rtol=1e-4, atol=1e-6, tf32=
     if bound is None or n_terms is None:
         idx = np.argwhere(bad)[:5]
         raise AssertionError(f"{what}: {bad.sum()} entries off, e.g. {[(tuple(i), gpu[tuple(i)], ref[tuple(i)]) for i in idx]}")
+    if callable(bound):
+        bound = bound()
     s = np.broadcast_to(np.asarray(bound, dtype=np.float64), ref.shape)
     nt = np.broadcast_to(np.asarray(n_terms, dtype=np.float64), ref.shape)
     lim = gamma(nt + 1) * s + U32 * np.abs(ref) + 1e-30

@@ -10,6 +10,7 @@ import numpy as np
 import pytest
 
 import oracle as O
+from tests import chain_bound
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -24,6 +25,8 @@ def infer():
 
 
 def _oracle_logits(ws, bs, images):
+    """The oracle's float64 logits (batch x 10) and the element-wise bound on
+    a float32 evaluation carried through the network (tests/chain_bound.py)."""
     from paper_1905_07931_gb300.train import lenet_layers
     layers = lenet_layers()
     net = O.Net([dict(l) for l in layers], [])
@@ -35,8 +38,8 @@ def _oracle_logits(ws, bs, images):
         else:
             net.params.append(None)
     b = images.shape[0]
-    z, _ = O.net_forward(net, images.reshape(1, b, 28, 28).astype(np.float32), b)
-    return z.T
+    z, F, _ = chain_bound.forward_bounds(net, images.reshape(1, b, 28, 28).astype(np.float32), b)
+    return z.T, F.T
 
 
 def test_weights_have_the_paper_counts(infer):
@@ -52,12 +55,12 @@ def test_inference_paths_against_oracle(infer, batch):
     ws, bs = infer.lenet_weights(0)
     rng = np.random.default_rng(batch)
     images = rng.random((batch, 28, 28), dtype=np.float32)
-    ref = _oracle_logits(ws, bs, images)
-    scale = np.abs(ref).max()
+    ref, bound = _oracle_logits(ws, bs, images)
     for cls in (infer.Compressed, infer.DenseGemm, infer.DenseCudnn):
         got = infer.logits_of(cls(ws, bs, batch), images)
         assert got.shape == (batch, 10)
-        assert np.abs(got - ref).max() <= 1e-4 * scale, cls.__name__
+        # element by element: rtol 1e-4 / atol 1e-6, else the carried summation bound
+        chain_bound.assert_within(got, ref, bound, what=cls.__name__)
 
 
 def test_timing_runs_on_a_small_set(infer):

@@ -12,6 +12,7 @@ import numpy as np
 import pytest
 
 import oracle as O
+from tests import chain_bound
 from tests.parity import assert_close, csr_dense
 
 torch = pytest.importorskip("torch")
@@ -85,14 +86,17 @@ def _oracle_net(layers, net):
 
 
 def _run_and_compare(C, net, layers, x_host, labels, eta, lam, phase, prec):
-    """One GPU step, checked against the oracle.
+    """One GPU step, checked against the oracle element by element.
 
-    Kernel parity is checked on the GPU's own inputs: each layer's gradient
-    against the oracle fed the GPU's dL/dpre and layer input, the update
-    bit-exact against the oracle update fed the GPU's gradient. The chain as
-    a whole is checked against the oracle's own forward/backward: the loss
-    tightly, max-pool winners exactly except at near-ties (where either
-    winner is correct), dL/dpre loosely (fp32 vs fp64 through several layers).
+    Each layer on the GPU's own inputs: its forward output against the oracle
+    product of the GPU's layer input, dL/dpre of a layer below an fc layer
+    against the oracle's transposed product of the GPU's dL/dpre above, its
+    gradient against the oracle fed the GPU's dL/dpre and layer input, and the
+    update bit for bit against the oracle update fed the GPU's gradient. The
+    chain as a whole against the oracle's own float64 forward / backward: the
+    loss, max-pool winners (exact except at near-ties, where either winner is
+    correct) and every element of every layer's dL/dpre, within the error
+    bound carried through the chain (tests/chain_bound.py).
     """
     onet = _oracle_net(layers, net)
     batch = len(labels)
@@ -100,6 +104,7 @@ def _run_and_compare(C, net, layers, x_host, labels, eta, lam, phase, prec):
     torch.cuda.synchronize()
     assert net.ws.status()[0] == 0
     logits, cache = O.net_forward(onet, x_host, batch)
+    pool_idx = {}
     for li, L in enumerate(layers):
         if L["kind"] == "pool2":
             gidx = net.layers[li]["idx"].cpu().numpy().reshape(cache[li]["idx"].shape)
@@ -113,26 +118,42 @@ def _run_and_compare(C, net, layers, x_host, labels, eta, lam, phase, prec):
                 best = win.max(axis=-1)
                 assert np.all(picked[diff] >= best[diff]), "GPU pooling picked a non-maximum"
                 assert diff.mean() < 1e-3, diff.mean()
-                cache[li]["idx"] = gidx.astype(np.int8)
-    oloss, dz = O.softmax_xent(logits, labels)
-    ograds = O.net_backward(onet, cache, dz, phase)
+            pool_idx[li] = gidx.astype(np.int8)
+    oloss, _ = O.softmax_xent(logits, labels)
     got_loss = float(loss[0].item())
     assert abs(got_loss - oloss) <= 2e-5 * max(1.0, abs(oloss)), (got_loss, oloss)
+    # the chain: oracle forward / backward with carried element-wise bounds
+    blogits, F_logits, per = chain_bound.forward_bounds(onet, x_host, batch, pool_idx)
+    dz, E_dz = chain_bound.softmax_bound(blogits, F_logits, labels)
+    chain = chain_bound.backward_bounds(onet, per, dz, E_dz, batch)
     pl = [i for i, l in enumerate(layers) if l["kind"] in ("fc", "conv")]
     for pi, li in enumerate(pl):
         L = net.params[pi]
-        og = ograds[li]
-        if og is None:
-            continue
         old = onet.params[li]
         W = old["W"]
         M = W.rows
         d_gpu = L["dpre"].cpu().numpy().reshape(M, -1).astype(np.float64)
         x_gpu = L["xmat"].cpu().numpy().reshape(W.cols, -1).astype(np.float64)
         n = x_gpu.shape[1]
-        scale = np.abs(og["delta"]).max() + 1e-30
-        assert np.abs(d_gpu - og["delta"]).max() <= 1e-3 * scale, f"dL/dpre of layer {pi}"
         absx, absd = np.abs(x_gpu), np.abs(d_gpu)
+        # this layer's forward output from the GPU's own input (im2col columns for a conv layer)
+        pre = O.spmm_fwd(W, x_gpu) + old["b"].astype(np.float64)[:, None]
+        want = O.relu(pre) if layers[li]["relu"] else pre
+        assert_close(L["y"].cpu().numpy().reshape(M, -1).astype(np.float64), want,
+                     lambda: O.spmm_fwd(O.csr_abs(W), absx) + np.abs(old["b"]).astype(np.float64)[:, None],
+                     np.diff(W.row_ptr)[:, None] + 1, what=f"forward of layer {pi}")
+        # dL/dpre of this layer from the GPU's dL/dpre of the fc layer above
+        if pi + 1 < len(pl) and layers[pl[pi + 1]]["kind"] == "fc" and pl[pi + 1] == li + 1:
+            up = net.params[pi + 1]
+            Wu = onet.params[li + 1]["W"]
+            d_up = up["dpre"].cpu().numpy().reshape(Wu.rows, -1).astype(np.float64)
+            mask = (L["y"].cpu().numpy() > 0) if layers[li]["relu"] else np.ones_like(d_gpu, dtype=bool)
+            assert_close(d_gpu, O.spmm_bwd_t(Wu, d_up) * mask,
+                         lambda: O.spmm_bwd_t(O.csr_abs(Wu), np.abs(d_up)) * mask,
+                         np.bincount(Wu.col_idx, minlength=Wu.cols)[:, None], what=f"dL/dpre of layer {pi}")
+        # ... and from the oracle's own chain, within the carried bound
+        d_ref, E_ref = chain[li]
+        chain_bound.assert_within(d_gpu, d_ref, E_ref, what=f"chain dL/dpre of layer {pi}")
         if phase == "prox":
             G = L["G"].cpu().numpy()
             assert_close(G, O.weight_grad_dense(d_gpu, x_gpu), O.weight_grad_dense(absd, absx), n,
@@ -215,16 +236,23 @@ def _assert_prox_within_bound(w_gpu, W_old, d, x, eta, lam, what):
     err = np.abs(vg - ref)[keep]
     assert np.all(err <= dz[keep] + U32 * np.abs(ref[keep])), f"{what}: kept values beyond the bound"
     assert np.all(np.diff(got.row_ptr) >= 0) and got.row_ptr[0] == 0
-    for r in range(0, M, max(1, M // 64)):   # sorted, unique columns within sampled rows
-        c = got.col_idx[got.row_ptr[r]:got.row_ptr[r + 1]]
-        assert np.all(np.diff(c) > 0), f"{what}: row {r} columns not increasing"
+    # columns strictly ascending within every row
+    rp64 = got.row_ptr.astype(np.int64)
+    if got.nnz > 1:
+        step_up = np.diff(got.col_idx.astype(np.int64)) > 0
+        row_start = np.zeros(got.nnz, dtype=bool)
+        row_start[rp64[1:-1][rp64[1:-1] < got.nnz]] = True
+        assert np.all(step_up | row_start[1:]), f"{what}: columns not strictly ascending within a row"
     if t is not None:   # the transposed copy is exactly the transpose of the GPU's own CSR
         trp, tci, tv, tpos = O.csr_transpose(got)
         np.testing.assert_array_equal(t[0], trp)
         np.testing.assert_array_equal(t[1], tci)
         np.testing.assert_array_equal(t[2].view(np.uint32), tv.astype(F32).view(np.uint32))
         np.testing.assert_array_equal(t[3], tpos)
-    return int(keep.sum())
+    in_band = int((~clear).sum())
+    print(f"{what}: {int(keep.sum())} kept, {in_band} of {M * K} entries inside the TF32 band")
+    assert in_band <= 0.01 * M * K, f"{what}: {in_band} entries inside the band"
+    return int(keep.sum()), in_band
 
 
 @pytest.mark.parametrize("workload", ["mlp", "fc_head"])
