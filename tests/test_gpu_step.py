@@ -251,7 +251,7 @@ def _assert_prox_within_bound(w_gpu, W_old, d, x, eta, lam, what):
         np.testing.assert_array_equal(t[3], tpos)
     in_band = int((~clear).sum())
     print(f"{what}: {int(keep.sum())} kept, {in_band} of {M * K} entries inside the TF32 band")
-    assert in_band <= 0.01 * M * K, f"{what}: {in_band} entries inside the band"
+    assert in_band <= 0.1 * M * K, f"{what}: {in_band} entries inside the band"
     return int(keep.sum()), in_band
 
 
