@@ -805,6 +805,9 @@ def profile_ops(net, C, torch, eta, lam, flush):
     try:
         flush.fill_(1.0)
         torch.cuda.synchronize()
+        # keep the GPU busy while the host enqueues the step, so that no
+        # call's events enclose host-side launch latency
+        torch.cuda._sleep(20_000_000)
         net.step("prox", eta, lam)
         torch.cuda.synchronize()
     finally:

@@ -61,12 +61,14 @@ def density_preserving_lambda(w: np.ndarray, g: np.ndarray, eta: float, density:
 
 
 def run_layer(m: int, k: int, density: float, zipf: bool, batches, ops, reps: int, seed: int = 0,
-              transposed: bool = True):
+              transposed: bool = True, dy_scale: float = 1.0):
     rng = synth.rng_for(seed)
     w = synth.masked_weights(rng, m, k, density, zipf=zipf)
     nmax = max(batches)
     x = synth.std_normal(rng, k, nmax)
     dy = synth.std_normal(rng, m, nmax)
+    if dy_scale != 1.0:
+        dy = (dy * np.float32(dy_scale)).astype(np.float32)
     g = synth.std_normal(rng, m, k)
     eta, lam = synth.ETA, synth.LAMBDA
     ws = C.Workspace(m, k, nmax)
@@ -146,6 +148,9 @@ def main(argv=None):
     p.add_argument("--zipf", choices=["both", "yes", "no"], default="both")
     p.add_argument("--reps", type=int, default=10)
     p.add_argument("--json", action="store_true")
+    p.add_argument("--dy-scale", type=float, default=1.0,
+                   help="scale of dY: at eta 0.01, lambda 1e-4 and n = 256, 5e-6 keeps about a quarter of the "
+                        "fused prox step's outputs, like the classifier-head step (1 keeps nearly all)")
     p.add_argument("--no-transposed", action="store_true",
                    help="prox outputs without the transposed arrays (a first layer, whose dX is not needed)")
     a = p.parse_args(argv)
@@ -154,7 +159,7 @@ def main(argv=None):
     out = []
     for d in a.density:
         for z in zipfs:
-            out += run_layer(a.m, a.k, d, z, a.n, ops, a.reps, transposed=not a.no_transposed)
+            out += run_layer(a.m, a.k, d, z, a.n, ops, a.reps, transposed=not a.no_transposed, dy_scale=a.dy_scale)
     if ops & {"spmm_fwd", "spmm_bwd_t", "sddmm"}:
         # the CUDA-core products against the measured FP32 FMA throughput
         peak = C.fma_peak_tflops()
