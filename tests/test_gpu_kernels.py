@@ -441,6 +441,37 @@ def test_prox_chain_of_steps_bit_exact(C, m, k):
         _check_csr_equal(bufs[(step + 1) % 2], ref)
 
 
+@pytest.mark.parametrize("eta,lam", [(0.0, 1e-4), (0.01, 0.0), (1e-3, 1e-38), (0.5, 1e30), (3.0, 1e-7),
+                                     (1e-20, 1e-20)])
+def test_fused_gradient_prox_threshold_edges(C, eta, lam):
+    """The fused count pass decides an unstored entry by |G| > g*, the largest
+    float with fl(eta*g*) <= fl(eta*lambda) (found on the host): the same keep
+    decisions and values as weight_grad_dense (TF32) + prox_update_compact at
+    eta = 0, lambda = 0, a subnormal threshold, a threshold above every
+    product, and gradients scaled so that many products land on it."""
+    m, k, n = 256, 512, 64
+    rng = np.random.default_rng(int(1e3 * eta) + 7)
+    a = _sparse(rng, m, k, 0.1) * F32(0.05)
+    dy = _dev((rng.standard_normal((m, n)) * 1e-3).astype(F32))
+    x = _dev(rng.standard_normal((k, n)).astype(F32))
+    ws = _ws(C, m, k, n)
+    w_in = _gpu_csr(C, a, ws, transposed=False)
+    g = torch.zeros(m, k, device="cuda")
+    C.weight_grad_dense(dy, x, g, ws, precision=C.CSRT_PREC_TF32)
+    ref = C.CSR(m, k, transposed=True)
+    C.prox_update_compact(w_in, g, eta, lam, ref, ws)
+    out = C.CSR(m, k, transposed=True)
+    C.weight_grad_prox_update(w_in, dy, x, eta, lam, out, ws)
+    assert ws.status()[0] == 0
+    (rp, ci, v), t = out.to_host()
+    (rp2, ci2, v2), t2 = ref.to_host()
+    np.testing.assert_array_equal(rp, rp2)
+    np.testing.assert_array_equal(ci, ci2)
+    np.testing.assert_array_equal(v.view(np.uint32), v2.view(np.uint32))
+    for p_, q_ in zip(t, t2):
+        np.testing.assert_array_equal(p_.view(np.uint32), q_.view(np.uint32))
+
+
 @pytest.mark.parametrize("m,k,n,density,lam,transposed,zipf", [
     (300, 512, 64, 0.1, 0.05, True, False),
     (129, 320, 36, 0.2, 0.02, False, False),
