@@ -9,6 +9,10 @@ loss, dense weight gradients (tcgen05 TF32), transposed SpMM x2, bias SGD,
 prox update + CSR re-compaction x3 (and the transposed pattern of the two
 layers whose input gradient is needed).
 
+The prox phase runs each layer's bias and weight update (but the first
+layer's) on a second stream, concurrently with the transposed products that
+carry dL/dX down the network (--overlap off: one stream).
+
 Timing: W eager warm-up steps, then the step is captured in a CUDA graph and
 K replays are timed one by one with CUDA events on the replay stream. Before
 every step (outside the timed region) the biases are restored and a 256 MB
@@ -61,6 +65,9 @@ def parse_args():
     p.add_argument("--prox-path", choices=["fused", "unfused"], default="fused",
                    help="fused: weight gradient and prox update in one tensor-core pass (G not written)")
     p.add_argument("--profile-ops", action="store_true", help="print the per-operation breakdown to stderr")
+    p.add_argument("--overlap", choices=["on", "off"], default="on",
+                   help="run each layer's bias and weight update (but the first layer's) on a second stream, "
+                        "concurrently with the transposed products")
     p.add_argument("--record-traffic", metavar="CSV",
                    help="write profiles/traffic.json from an ncu CSV of this bench (dram__bytes_read.sum, "
                         "dram__bytes_write.sum, gpu__time_duration.sum; --steps 1 --warmup 1) and exit")
@@ -154,12 +161,14 @@ class OracleSample:
                 f"transposed pattern); the row-separable time x {self.F} + the loss once")
 
 
-def workload_config(world: int, precision: str = "tf32", prox_path: str = "fused", optimizer: str = "sgd") -> dict:
+def workload_config(world: int, precision: str = "tf32", prox_path: str = "fused", optimizer: str = "sgd",
+                    overlap: str = "on") -> dict:
     """The `config` of both arms' lines: the workload and its settings."""
     return {"workload": WORKLOAD, "global_batch": BATCH * world, "per_gpu_batch": BATCH,
             "layers": list(SIZES), "densities": list(DENSITIES),
             "weight_grad": "tf32 tcgen05" if precision == "tf32" else "fp32 simt",
             "prox_path": prox_path if optimizer == "sgd" else "unfused", "optimizer": optimizer,
+            "backward_streams": 2 if overlap == "on" else 1,
             "l2": "flushed between steps (256 MB write, outside the timed region)",
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU"}
 
@@ -521,7 +530,7 @@ def main():
     cfg = synth.fc_head(seed=0)
     layers = mlp_layers(3)
     net = SparseNet(layers, cfg["W"], cfg["b"], BATCH, (SIZES[0],), precision=prec,
-                    fused=args.prox_path == "fused", optimizer=args.optimizer)
+                    fused=args.prox_path == "fused", optimizer=args.optimizer, overlap=args.overlap == "on")
     x_host = torch.from_numpy(cfg["X"]).pin_memory()
     lab_host = torch.from_numpy(cfg["labels"]).pin_memory()
     net.x_in.copy_(x_host)
@@ -543,7 +552,7 @@ def main():
         restore()
         net.step("prox", eta, lam)
     torch.cuda.synchronize()
-    flags, _ = net.ws.status()
+    flags, _ = net.status()
     if flags:
         raise SystemExit(f"device status {flags} after warm-up")
 
@@ -590,7 +599,7 @@ def main():
     times_ms = [a.elapsed_time(b) for a, b in zip(starts, ends)]
     total_max_ms = max_over_ranks(sum(times_ms), world, "cuda")
     value = whole_job_rate(BATCH, args.steps, world, total_max_ms)
-    flags, _ = net.ws.status()
+    flags, _ = net.status()
     if flags:
         raise SystemExit(f"device status {flags} after the timed steps")
 
@@ -713,7 +722,7 @@ def main():
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(total_max_ms / args.steps, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": dict(workload_config(world, args.precision, args.prox_path, args.optimizer),
+        "config": dict(workload_config(world, args.precision, args.prox_path, args.optimizer, args.overlap),
                        step_ops=[r["label"] for r in prof]),
         "e2e": {"value": round(e2e_value, 1), "unit": UNIT,
                 "h2d_bytes_per_step": int(x_host.numel() * 4 + lab_host.numel() * 4), "d2h_bytes_per_step": 4},
@@ -802,6 +811,8 @@ def profile_ops(net, C, torch, eta, lam, flush):
                 records.append({"name": nm, "st": st, "en": en, "info": info, "layer": li})
             return fn
         setattr(C, nm, make(nm, orig))
+    overlap = net.overlap
+    net.overlap = False   # one stream: every call's events bracket that call alone
     try:
         flush.fill_(1.0)
         torch.cuda.synchronize()
@@ -811,6 +822,7 @@ def profile_ops(net, C, torch, eta, lam, flush):
         net.step("prox", eta, lam)
         torch.cuda.synchronize()
     finally:
+        net.overlap = overlap
         for nm, orig in wrapped.items():
             setattr(C, nm, orig)
     out = []

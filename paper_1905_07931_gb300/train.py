@@ -33,7 +33,7 @@ class SparseNet:
     def __init__(self, layers, dense_weights, biases, batch: int, in_shape, *, device="cuda",
                  precision: int = C.CSRT_PREC_TF32, stream=None, grad_per_layer: bool = False,
                  fused: bool = True, optimizer: str = "sgd", beta1: float = 0.9, beta2: float = 0.999,
-                 rms_beta: float = 0.9, eps: float = 1e-8):
+                 rms_beta: float = 0.9, eps: float = 1e-8, overlap: bool = False):
         """layers: layer dicts; dense_weights/biases: numpy arrays, one per fc/conv
         layer (weights M x K, zero off the initial pattern); in_shape: (K,) for an
         fc-first net or (C, H, W) for a conv-first net. The dense gradients of
@@ -46,7 +46,16 @@ class SparseNet:
         eps is the safeguard of both. The adaptive methods keep dense M x K
         moment arrays per layer and count their steps on the host (the step
         number is passed by value, so a captured graph replays the step it was
-        captured at). The debias phase is plain SGD in every case."""
+        captured at). The debias phase is plain SGD in every case.
+
+        overlap: in the prox phase, the bias update and the weight update of
+        every layer but the first run on a second stream (with its own
+        workspace and gradient buffer), concurrently with the transposed
+        products that carry dL/dX down the network: the weight update of a
+        layer reads its current CSR and writes the other buffer, the
+        transposed product only reads the current one. The second stream
+        joins the caller's at the end of the step. (The debias phase updates
+        the stored values in place and stays on one stream.)"""
         if optimizer not in ("sgd", "rmsprop", "adam"):
             raise ValueError(f"unknown optimizer {optimizer!r}")
         self.optimizer = optimizer
@@ -148,10 +157,26 @@ class SparseNet:
         self.loss = torch.zeros(B + 1, **dev)
         self.G = torch.zeros(max_mk, **dev)
         self.ws = C.Workspace(max_rows, max_cols, max_n, device=device, stream=stream)
+        self.overlap = overlap
+        if overlap:
+            self.side = torch.cuda.Stream(device=device)
+            self.ws_side = C.Workspace(max_rows, max_cols, max_n, device=device, stream=stream)
+            self.G_side = torch.zeros(max_mk, **dev)
+            n_fc = sum(1 for L in self.layers if L["kind"] in ("fc", "conv"))
+            self._events = [torch.cuda.Event() for _ in range(n_fc + 1)]
         for L in self.params:
             C.csr_from_dense(L["W0"], L["W"][0], self.ws, stream)
 
     # ------------------------------------------------------------------
+    def status(self):
+        """Device status of the step (synchronises): the flags of every
+        workspace the network uses, OR-ed, and the largest required nnz."""
+        flags, req = self.ws.status(self.stream)
+        if self.overlap:
+            f2, r2 = self.ws_side.status(self.stream)
+            flags, req = flags | f2, max(req, r2)
+        return flags, req
+
     def weights(self, li: int) -> C.CSR:
         L = self.params[li]
         return L["W"][L["cur"]]
@@ -199,6 +224,9 @@ class SparseNet:
         s = self.stream
         if phase == "prox":
             self.t += 1   # step number of the adaptive methods (Algorithms 1 and 2)
+        ov = self.overlap and phase == "prox"
+        main = (s if s is not None else torch.cuda.current_stream()) if ov else s
+        ev_i = 0
         self.forward()
         C.softmax_xent(self.logits, self.labels, self.dlogits, self.loss, s)
         d = self.dlogits
@@ -214,13 +242,23 @@ class SparseNet:
                 d_masked = False
                 L["dpre"] = dpre   # dL/d(pre-activation) of this layer (a view kept for inspection)
                 M, K = W.rows, W.cols
+                # this layer's bias and weight update: on the second stream
+                # when overlapping (not for the first layer, the last of the step)
+                side = ov and L["needs_dx"]
+                us, uws = (self.side, self.ws_side) if side else (s, self.ws)
+                if side:
+                    ev = self._events[ev_i]
+                    ev_i += 1
+                    ev.record(main)
+                    self.side.wait_event(ev)
                 if phase == "prox":
-                    G = L["G"] if self.grad_per_layer else self.G[: M * K].view(M, K)
+                    Gbuf = self.G_side if side else self.G
+                    G = L["G"] if self.grad_per_layer else Gbuf[: M * K].view(M, K)
                     if not self.fused:
-                        C.weight_grad_dense(dpre, L["xmat"], G, self.ws, self.precision, s)
+                        C.weight_grad_dense(dpre, L["xmat"], G, uws, self.precision, us)
                 else:
                     C.weight_grad_sddmm(W, dpre, L["xmat"], L["g"], self.ws, s)
-                C.bias_grad_sgd(dpre, L["b"], eta, None, s)
+                C.bias_grad_sgd(dpre, L["b"], eta, None, us)
                 if L["needs_dx"]:
                     below = self.layers[li - 1] if li > 0 else None
                     if kind == "fc" and below is not None and below["kind"] == "fc" and below["relu"]:
@@ -236,14 +274,14 @@ class SparseNet:
                 if phase == "prox":
                     Wn = L["W"][1 - L["cur"]]
                     if self.fused:
-                        C.weight_grad_prox_update(W, dpre, L["xmat"], eta, lam, Wn, self.ws, self.precision, G, s)
+                        C.weight_grad_prox_update(W, dpre, L["xmat"], eta, lam, Wn, uws, self.precision, G, us)
                     elif self.optimizer == "rmsprop":
-                        C.prox_rmsprop_update_compact(W, G, L["v"], eta, lam, self.rms_beta, self.eps, Wn, self.ws, s)
+                        C.prox_rmsprop_update_compact(W, G, L["v"], eta, lam, self.rms_beta, self.eps, Wn, uws, us)
                     elif self.optimizer == "adam":
                         C.prox_adam_update_compact(W, G, L["m"], L["v"], self.t, eta, lam, self.beta1, self.beta2,
-                                                   self.eps, Wn, self.ws, s)
+                                                   self.eps, Wn, uws, us)
                     else:
-                        C.prox_update_compact(W, G, eta, lam, Wn, self.ws, s)
+                        C.prox_update_compact(W, G, eta, lam, Wn, uws, us)
                     L["cur"] = 1 - L["cur"]
                 else:
                     C.debias_update(W, L["g"], eta, s)
@@ -258,6 +296,10 @@ class SparseNet:
                 c, h, w = L["shape"]
                 C.unflatten(d, c, self.batch, h * w, L["dx"], s)
                 d = L["dx"]
+        if ov and ev_i:   # the second stream's work is part of the step
+            ev = self._events[ev_i]
+            ev.record(self.side)
+            main.wait_event(ev)
         return self.loss
 
     def reset_weights(self):

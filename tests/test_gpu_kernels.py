@@ -827,16 +827,56 @@ def test_bounded_waits_give_up_and_report(C):
     assert ws.status()[0] == 0
 
 
+@pytest.mark.parametrize("m,k,n,density,mix", [(256, 512, 64, 0.05, False), (1000, 4096, 256, 0.05, False),
+                                               (512, 2048, 128, 0.05, True), (300, 1024, 32, 0.02, True),
+                                               (128, 9216, 256, 0.08, True)])
+def test_fused_gradient_prox_sparse_and_dense_words(C, m, k, n, density, mix):
+    """The write pass stores a 32-column word whose 32 rows keep few entries
+    (at most 96) by per-row compaction and one entry per lane, and other words
+    by the row walk. Small gradients keep little more than the stored weights
+    (sparse words); with `mix`, alternate 32-row bands get large gradients
+    (dense words), so both forms run in one call. Bit-identical to
+    weight_grad_dense (TF32) + prox_update_compact, transposed copy included."""
+    rng = np.random.default_rng(m + k + n)
+    a = _sparse(rng, m, k, density) * F32(0.05)
+    scale = np.full((m, 1), 1e-5, dtype=F32)
+    if mix:
+        scale[(np.arange(m) // 32) % 2 == 1] = F32(0.1)
+    dy = _dev((rng.standard_normal((m, n)) * scale).astype(F32))
+    x = _dev(rng.standard_normal((k, n)).astype(F32))
+    ws = _ws(C, m, k, n)
+    w_in = _gpu_csr(C, a, ws, transposed=False)
+    g = torch.zeros(m, k, device="cuda")
+    C.weight_grad_dense(dy, x, g, ws, precision=C.CSRT_PREC_TF32)
+    ref = C.CSR(m, k, transposed=True)
+    C.prox_update_compact(w_in, g, 0.5, 2e-3, ref, ws)
+    out = C.CSR(m, k, transposed=True)
+    C.weight_grad_prox_update(w_in, dy, x, 0.5, 2e-3, out, ws)
+    assert ws.status()[0] == 0
+    (rp, ci, v), t = out.to_host()
+    (rp2, ci2, v2), t2 = ref.to_host()
+    kept = np.diff(rp.astype(np.int64))
+    assert kept.min() < 0.1 * k   # sparse rows present
+    if mix:
+        assert kept.max() > 0.5 * k   # and dense ones
+    np.testing.assert_array_equal(rp, rp2)
+    np.testing.assert_array_equal(ci, ci2)
+    np.testing.assert_array_equal(v.view(np.uint32), v2.view(np.uint32))
+    for p_, q_ in zip(t, t2):
+        np.testing.assert_array_equal(p_.view(np.uint32), q_.view(np.uint32))
+
+
+@pytest.mark.parametrize("dy_scale", [0.1, 1e-5])
 @pytest.mark.parametrize("transposed", [False, True])
-def test_fused_gradient_prox_capacity_overflow(C, transposed):
+def test_fused_gradient_prox_capacity_overflow(C, transposed, dy_scale):
     """An output CSR too small for the fused op's result: the overflow and the
     needed nnz are reported, the row pointers are clamped, and the stored
     prefix equals the unfused result's (the transposed copy, when asked for,
     writes only inside the capacity)."""
     m, k, n = 256, 512, 64
     rng = np.random.default_rng(9)
-    a = _sparse(rng, m, k, 0.1) * F32(0.05)
-    dy = _dev((rng.standard_normal((m, n)) * 0.1).astype(F32))
+    a = _sparse(rng, m, k, 0.1 if dy_scale > 1e-3 else 0.05) * F32(0.05)   # dense words, or sparse ones
+    dy = _dev((rng.standard_normal((m, n)) * dy_scale).astype(F32))
     x = _dev(rng.standard_normal((k, n)).astype(F32))
     ws = _ws(C, m, k, n)
     w_in = _gpu_csr(C, a, ws, transposed=False)

@@ -317,3 +317,38 @@ def test_mlp_adaptive_prox_steps(C, optimizer):
                 ref, st["v"] = O.prox_rmsprop_update_compact(old[pi], G, st["v"], eta, lam, 0.9, 1e-8)
             np.testing.assert_array_equal(L["v"].cpu().numpy().view(np.uint32), st["v"].view(np.uint32))
             _assert_csr_bits(net.weights(pi), ref)
+
+
+@pytest.mark.parametrize("workload,fused,optimizer", [("mlp", True, "sgd"), ("mlp", False, "sgd"),
+                                                      ("mlp", False, "adam"), ("fc_head", True, "sgd")])
+def test_overlapped_backward_matches_one_stream(C, workload, fused, optimizer):
+    """The prox phase with each layer's bias and weight update on a second
+    stream (overlap) gives the same bits as the one-stream step: weights,
+    transposed copies, biases and losses over two prox steps and a debias step."""
+    from paper_1905_07931_gb300 import synth
+    from paper_1905_07931_gb300.train import SparseNet, mlp_layers
+    cfg = synth.mlp(seed=3) if workload == "mlp" else synth.fc_head(seed=0)
+    in_dim, batch = cfg["X"].shape
+    nets = []
+    for ov in (False, True):
+        net = SparseNet(mlp_layers(3), cfg["W"], cfg["b"], batch, (in_dim,), precision=1, fused=fused,
+                        optimizer=optimizer, overlap=ov)
+        net.x_in.copy_(torch.from_numpy(cfg["X"]))
+        net.labels.copy_(torch.from_numpy(cfg["labels"]))
+        nets.append(net)
+    eta, lam = (1e-3, 0.05) if optimizer == "adam" else (cfg["eta"], cfg["lambda"])
+    for phase in ("prox", "prox", "debias"):
+        losses = [float(net.step(phase, eta, lam)[0].item()) for net in nets]
+        torch.cuda.synchronize()
+        assert losses[0] == losses[1]
+        for net in nets:
+            assert net.status()[0] == 0
+        for pi in range(3):
+            (a, ta), (b, tb) = nets[0].weights(pi).to_host(), nets[1].weights(pi).to_host()
+            for x, y in zip(a, b):
+                np.testing.assert_array_equal(x.view(np.uint32), y.view(np.uint32))
+            if ta is not None:
+                for x, y in zip(ta, tb):
+                    np.testing.assert_array_equal(x.view(np.uint32), y.view(np.uint32))
+            np.testing.assert_array_equal(nets[0].params[pi]["b"].cpu().numpy().view(np.uint32),
+                                          nets[1].params[pi]["b"].cpu().numpy().view(np.uint32))
