@@ -377,6 +377,10 @@ FUSED_OP_KERNELS = ("fp_oldbits_kernel", "gemm_prox_tc_kernel", "fp_rowscan_kern
                     "scan_single_block_kernel", "fp_finish_kernel", "trb_count_kernel", "tr_colscan_kernel",
                     "trb_write_kernel")
 FUSED_OP_SOURCES = ["fused_prox.cu", "compact.cu", "tc_common.cuh", "common.cuh"]
+# the ncu command whose CSV record_traffic reads: the ops' kernels only
+TRAFFIC_NCU = ("ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum --clock-control none "
+               "-k regex:'fp_oldbits|gemm_prox|fp_rowscan|scan_clamped|scan_single|trb_|tr_colscan|spmm_merge' "
+               "-c 60 --csv --log-file bench_dram.csv")
 
 
 def record_traffic(csv_path: str, out_path: str) -> dict:
@@ -415,12 +419,11 @@ def record_traffic(csv_path: str, out_path: str) -> dict:
     pending = {}
     rec = {"_about": "DRAM bytes (read + write) of one call of each fused weight-gradient + prox op and each "
                      "sparse product of the classifier-head step, summed over the op's kernels (second eager step "
-                     "of the run), from: ncu "
-                     "--metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum --clock-control "
-                     "none --csv --log-file bench_dram.csv python bench.py --steps 1 --warmup 1 --no-cpu-baseline, "
-                     "then python bench.py --record-traffic bench_dram.csv. ncu flushes the caches between kernels, "
-                     "so output lines still dirty in L2 when a kernel ends are not counted: an op whose output fits "
-                     "in L2 shows fewer bytes than it writes."}
+                     "of the run), from: " + TRAFFIC_NCU + " python bench.py --steps 1 --warmup 1 --no-cpu-baseline "
+                     "--no-kernels --overlap off, then python bench.py --record-traffic bench_dram.csv (the counters "
+                     "take one pass; only the ops' kernels are captured, the first 60 launches: 4 at start-up, 28 "
+                     "per step). ncu flushes the caches between kernels, so output lines still dirty in L2 when a "
+                     "kernel ends are not counted: an op whose output fits in L2 shows fewer bytes than it writes."}
     # the step's sparse products, in call order: forward layers 0, 1, 2, then
     # the backward products of layers 2 and 1 (second eager step)
     sp = [k for k in seq if "spmm_merge_kernel" in k["name"] or "spmm_group_kernel" in k["name"]]
