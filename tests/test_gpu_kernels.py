@@ -404,6 +404,39 @@ def test_prox_bit_exact(C, m, k, density, gscale, eta, lam):
     assert ws.status()[0] == 0
 
 
+@pytest.mark.parametrize("eta,lam", [(0.0, 1e-4), (0.01, 0.0), (1e-3, 1e-38), (0.5, 1e30), (1e20, 1e20),
+                                     (3.0, 1e-7)])
+def test_prox_threshold_edges(C, eta, lam):
+    """prox_update_compact bit-exact with the oracle at eta = 0, lambda = 0, a
+    subnormal threshold, a threshold above every product and an infinite one,
+    with infinite and NaN gradients among the entries; NaN in w - eta*G is
+    flagged (with eta = 0 an infinite gradient gives NaN too)."""
+    m, k = 300, 512
+    rng = np.random.default_rng(int(eta * 7) % 1000 + 3)
+    a = _sparse(rng, m, k, 0.1)
+    g = rng.standard_normal((m, k)).astype(F32)
+    g[5, 7] = np.inf
+    g[9, 100] = -np.inf
+    g[11, 3] = np.nan
+    ws = _ws(C, m, k, 1)
+    w = _gpu_csr(C, a, ws)
+    out = C.CSR(m, k)
+    C.prox_update_compact(w, _dev(g), eta, lam, out, ws)
+    with np.errstate(invalid="ignore", over="ignore"):   # inf - inf and 0 * inf in the oracle's float32 rules
+        ref = O.prox_update_compact(O.csr_from_dense(a), g, eta, lam)
+    _check_csr_equal(out, ref)
+    assert ws.status()[0] & C.CSRT_DEV_NONFINITE
+    ws.clear_status()
+    g2 = np.where(np.isfinite(g), g, 0).astype(F32)
+    g2[5, 7] = np.inf                     # an infinity alone: flagged only where eta * Inf is NaN
+    out2 = C.CSR(m, k)
+    C.prox_update_compact(w, _dev(g2), eta, lam, out2, ws)
+    with np.errstate(invalid="ignore", over="ignore"):
+        ref2 = O.prox_update_compact(O.csr_from_dense(a), g2, eta, lam)
+    _check_csr_equal(out2, ref2)
+    assert bool(ws.status()[0] & C.CSRT_DEV_NONFINITE) == (eta == 0.0)   # w - fl(0 * Inf) is NaN
+
+
 @pytest.mark.parametrize("m,k,transposed", [(3000, 512, True), (800, 9216, False), (5000, 300, True)])
 def test_prox_mixed_dense_and_sparse_tiles(C, m, k, transposed):
     """Rows whose G is large keep nearly every entry (their tiles take the
