@@ -459,6 +459,45 @@ def test_prox_mixed_dense_and_sparse_tiles(C, m, k, transposed):
     assert ws.status()[0] == 0
 
 
+@pytest.mark.parametrize("m,k,transposed", [(96, 256, True), (9, 9216, False)])
+def test_prox_stash_boundary(C, m, k, transposed):
+    """Tiles that keep exactly an eighth of their entries (written through
+    the stash and copied into place) next to tiles that keep one entry more
+    (written by the tile itself after the look-back), stored weights kept and
+    dropped among them: bit-exact with the oracle. A row tile here is
+    max(1, 8192 // k) rows; its stash holds tile_entries / 8 entries."""
+    rows_per_tile = max(1, 8192 // k)
+    cap = rows_per_tile * k // 8
+    rng = np.random.default_rng(k)
+    a = _sparse(rng, m, k, 0.02)
+    g = np.zeros((m, k), F32)   # unstored entries with G = 0 are dropped
+    eta, lam = 0.5, 0.1          # kept off the pattern iff |fl(0.5 G)| > 0.05
+    tiles = (m + rows_per_tile - 1) // rows_per_tile
+    for t in range(tiles):
+        r0 = t * rows_per_tile
+        blk = slice(r0, min(m, r0 + rows_per_tile))
+        stored = a[blk] != 0
+        n_stored = int(stored.sum())
+        # every stored weight is kept (|w - 0| = |w| > 0.05 for these draws), so the tile keeps
+        # n_stored + the unstored entries given a large G: cap, cap + 1, or fewer
+        want = [cap, cap + 1, cap // 2][t % 3]
+        free = np.flatnonzero(~stored.ravel())
+        pick = rng.choice(free, size=max(0, want - n_stored), replace=False)
+        gb = g[blk].ravel()
+        gb[pick] = rng.choice([-1.0, 1.0], size=pick.size) * (1.0 + rng.random(pick.size))
+        g[blk] = gb.reshape(g[blk].shape)
+    a[(a != 0) & (np.abs(a) <= 0.05)] = 0.2   # stored weights all above the threshold
+    ws = _ws(C, m, k, 1)
+    w = _gpu_csr(C, a, ws)
+    out = C.CSR(m, k, transposed=transposed)
+    C.prox_update_compact(w, _dev(g), eta, lam, out, ws)
+    ref = O.prox_update_compact(O.csr_from_dense(a), g, eta, lam)
+    per_tile = np.add.reduceat(np.diff(ref.row_ptr), np.arange(0, m, rows_per_tile))
+    assert (per_tile == cap).any() and (per_tile == cap + 1).any()
+    _check_csr_equal(out, ref, transposed=transposed)
+    assert ws.status()[0] == 0
+
+
 @pytest.mark.parametrize("m,k", [(200, 333), (200, 320), (70, 4096)])
 def test_prox_chain_of_steps_bit_exact(C, m, k):
     # several prox steps in a row (double-buffered), each fed the same G as the oracle
