@@ -1046,6 +1046,7 @@ __device__ __forceinline__ void prox_cp_fold(const CompactArgs &a, int nrows, fl
 }
 
 __device__ __forceinline__ int nth_set_bit(uint32_t m, int k);
+__device__ __forceinline__ int warp_last_le(int pre, int e);
 
 // The kept value of the lane's entry of a 32-entry step: z - sign(z)*thr with
 // z the folded value at a stored position and fl(0 - fl(eta*G)) elsewhere.
@@ -1062,14 +1063,14 @@ __device__ __forceinline__ float prox_cp_value(float tv, bool stored, float eta,
 // assembled by three shuffles. The keep words collect in shared memory and
 // leave afterwards as coalesced stores, with the kept count of every row
 // summed from them, and the tile's count is published at once. A tile keeping
-// at most `stash` entries then writes them in CSR order to its stash, a
-// thread per kept entry (its word found by a binary search over the words'
-// exclusive counts), and is done without waiting on any other block; the
-// place kernel copies the stash to its final position. A denser tile learns
-// the number of entries kept before it by decoupled look-back over the
-// published counts (the ones of stashed tiles never become inclusive
-// prefixes, so it may sum further back) and writes its kept entries itself, a
-// 32-entry word at a time, G read only once.
+// at most `stash` entries then writes them in CSR order to its stash (each
+// warp its segment's, lane = entry, the entry's word found by a search over
+// the words' exclusive counts), and is done without waiting on any other
+// block; the place kernel copies the stash to its final position. A denser
+// tile learns the number of entries kept before it by decoupled look-back
+// over the published counts (the ones of stashed tiles never become
+// inclusive prefixes, so it may sum further back) and writes its kept entries
+// itself, a 32-entry word at a time, G read only once.
 template <bool kBits>
 __global__ void __launch_bounds__(kCThreads, 6) prox_count_kernel(CompactArgs a, int32_t rows_per_tile,
                                                                    uint32_t *__restrict__ keepbits,
@@ -1166,36 +1167,36 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_count_kernel(CompactArgs a,
             st_release_u64(a.status + tile, (tile == 0 ? kFlagInc : kFlagAgg) | tile_count);
     }
     if (stashed) {
-        // exclusive counts of the words (skeep is free now): each warp scans its own segment's words
-        uint32_t run = wbase;
-        for (int i0 = w0; i0 < w1; i0 += 32) {
-            const int i = i0 + lane;
-            const uint32_t c = i < w1 ? __popc(kwords[i]) : 0u;
-            uint32_t incl = c;
-#pragma unroll
-            for (int off = 1; off < 32; off <<= 1) {
-                const uint32_t t = __shfl_up_sync(0xffffffffu, incl, off);
-                if (lane >= off) incl += t;
-            }
-            if (i < w1) skeep[i] = run + incl - c;
-            run += __shfl_sync(0xffffffffu, incl, 31);
-        }
-        __syncthreads();
+        // the warp's kept entries, 32 words at a time (lane = word: exclusive counts by a warp scan), then
+        // lane = entry (its word found by a search over those counts): coalesced runs in the stash
         int32_t *sc = st_col + tile * (int64_t)stash;
         float *sv = st_val + tile * (int64_t)stash;
-        for (int i = tid; i < (int)tile_count; i += kCThreads) {
-            // the last word whose exclusive count is <= i (skeep[0] = 0 <= i)
-            int lo = 0, hi = nwt - 1;
-            while (lo < hi) {
-                const int mid = (lo + hi + 1) >> 1;
-                if ((int)skeep[mid] <= i) lo = mid; else hi = mid - 1;
+        uint32_t pos = wbase;
+        for (int i0 = w0; i0 < w1; i0 += 32) {
+            const int wl = i0 + lane;
+            const uint32_t myword = wl < w1 ? kwords[wl] : 0u;
+            const int c = __popc(myword);
+            int incl = c;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const int t = __shfl_up_sync(0xffffffffu, incl, off);
+                if (lane >= off) incl += t;
             }
-            const uint32_t word = kwords[lo];
-            const int bit = nth_set_bit(word, i - (int)skeep[lo]);
-            const int e = 32 * lo + bit;
-            const int row = lo / wpr;
-            sc[i] = e - row * K;
-            sv[i] = prox_cp_value(tile_v[e], (onbits[lo] >> bit) & 1u, eta, thr);
+            const int excl = incl - c, total = __shfl_sync(0xffffffffu, incl, 31);
+            for (int e0 = 0; e0 < total; e0 += 32) {
+                const int e = e0 + lane;
+                const int src = warp_last_le(excl, e);   // the lane (word) holding entry e
+                const uint32_t word = __shfl_sync(0xffffffffu, myword, src);
+                const int k = e - __shfl_sync(0xffffffffu, excl, src);
+                if (e < total) {
+                    const int wi = i0 + src;
+                    const int bit = nth_set_bit(word, k);
+                    const int row = wi / wpr;
+                    sc[pos + e] = 32 * wi + bit - row * K;
+                    sv[pos + e] = prox_cp_value(tile_v[32 * wi + bit], (onbits[wi] >> bit) & 1u, eta, thr);
+                }
+            }
+            pos += total;
         }
     } else {
         if (warp == 0) {
