@@ -396,7 +396,7 @@ static PlaceLayout place_layout(int32_t rows, int32_t cols) {
     if (rows <= 0 || cols <= 0 || cols % 32 != 0 || cols > kRowMaxK) return L;
     L.rows_per_tile = imax<int32_t>(1, kRowBudget / cols);
     L.tiles = ceil_div<int64_t>(rows, L.rows_per_tile);
-    L.stash = (L.rows_per_tile * cols + 7) / 8;
+    L.stash = imax((L.rows_per_tile * cols + 7) / 8, 2 * kCThreads);   // the place kernel reads 512 ahead
     size_t o = 0;
     L.off_rowcnt = o;  o += al((size_t)rows * 4);
     L.off_raw = o;     o += al(((size_t)rows + 1) * 4);
@@ -1246,19 +1246,25 @@ __global__ void __launch_bounds__(kCThreads) prox_place_kernel(CompactArgs a, in
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int64_t tile = blockIdx.x;
     if (tile >= a.num_tiles) return;
-    const int32_t count = __ldg(tilecnt + tile);
-    if (count < 0) return;
     const int r0 = (int)(tile * rows_per_tile);
     const int nrows = imin(rows_per_tile, a.rows - r0);
-    const uint32_t cap = (uint32_t)imin<int64_t>(a.capacity, 0x7fffffff);
-    const uint32_t base = (uint32_t)__ldg(raw + r0);
     const int32_t *sc = st_col + tile * (int64_t)stash;
     const float *sv = st_val + tile * (int64_t)stash;
+    // the count, the position and the stash's first two entries per thread load together (a stash holds
+    // at least 512 entries, so these reads stay inside it whatever the count)
+    const int32_t count = __ldg(tilecnt + tile);
+    const uint32_t base = (uint32_t)__ldg(raw + r0);
+    const int32_t c0 = __ldg(sc + tid), c1 = __ldg(sc + tid + kCThreads);
+    const float v0 = __ldg(sv + tid), v1 = __ldg(sv + tid + kCThreads);
+    if (count < 0) return;
+    const uint32_t cap = (uint32_t)imin<int64_t>(a.capacity, 0x7fffffff);
     for (int i = tid; i < count; i += kCThreads) {
         const uint32_t p = base + (uint32_t)i;
+        const int32_t c = i < kCThreads ? c0 : i < 2 * kCThreads ? c1 : __ldg(sc + i);
+        const float v = i < kCThreads ? v0 : i < 2 * kCThreads ? v1 : __ldg(sv + i);
         if (p < cap) {
-            a.out_col[p] = __ldg(sc + i);
-            a.out_val[p] = __ldg(sv + i);
+            a.out_col[p] = c;
+            a.out_val[p] = v;
         }
     }
     if (kBits) {   // word positions: a warp per row, a scan of the words' kept counts
