@@ -180,6 +180,17 @@ def cpu_cores() -> int:
         return os.cpu_count() or 1
 
 
+def timed_samples(samp, count: int):
+    """`count` oracle samples; returns their (measured s, estimated full-step s)
+    pairs and the threads they kept busy on average (process CPU time over
+    wall time: the row loops are single-threaded Python, numpy's BLAS may add
+    threads to the weight gradients)."""
+    w0, c0 = time.perf_counter(), time.process_time()
+    runs = [samp.step() for _ in range(count)]
+    wall, cpu = time.perf_counter() - w0, time.process_time() - c0
+    return runs, max(1, round(cpu / wall)) if wall > 0 else 1, round(cpu, 3)
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -189,7 +200,7 @@ def run_reference(args):
     samp = OracleSample(cfg, fraction_denominator=8)
     for _ in range(args.warmup):
         samp.step()
-    runs = [samp.step() for _ in range(args.steps)]
+    runs, cores_used, cpu_s = timed_samples(samp, args.steps)
     measured = sum(r[0] for r in runs)          # seconds the timed steps took (1/8-row samples)
     estimated = sum(r[1] for r in runs)         # the same steps scaled to whole steps
     # each timed step is one 1/8-row sample of the workload's step: it counts
@@ -200,7 +211,8 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * measured / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": workload_config(world),
-        "cpu_baseline": {"kind": "oracle", "value": value, "unit": UNIT, "cores": cpu_cores(),
+        "cpu_baseline": {"kind": "oracle", "value": value, "unit": UNIT, "cores": cores_used,
+                         "cores_available": cpu_cores(), "cpu_s": cpu_s,
                          "sample": samp.describe() + f"; each step is one sample, {args.steps} timed",
                          "measured_s": round(measured, 3), "scale_factor": samp.F,
                          "estimated_full_step_ms": round(1e3 * estimated / args.steps, 1)},
@@ -740,10 +752,11 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         samp = OracleSample(cfg, fraction_denominator=4)
         samp.step()
-        runs = [samp.step() for _ in range(5)]
+        runs, cores_used, cpu_s = timed_samples(samp, 5)
         est = [r[1] for r in runs]
         v = BATCH / (sum(est) / len(est))
-        line["cpu_baseline"] = {"value": round(v, 3), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+        line["cpu_baseline"] = {"value": round(v, 3), "unit": UNIT, "cores": cores_used,
+                                "cores_available": cpu_cores(), "cpu_s": cpu_s, "kind": "oracle",
                                 "sample": samp.describe() + ", mean of 5 samples after one untimed",
                                 "measured_s": round(sum(r[0] for r in runs), 3), "samples": len(runs),
                                 "scale_factor": samp.F,
