@@ -144,6 +144,22 @@ __host__ __device__ __forceinline__ T ceil_div(T a, T b) {
     return (a + b - 1) / b;
 }
 
+// Transpose of a 32 x 32 bit matrix held one word per lane (bit j of lane i
+// is element (i, j)): on return bit i of lane j is element (i, j). Five rounds,
+// each exchanging half-blocks with the lane whose index differs in one bit.
+__device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int sft = 16; sft >= 1; sft >>= 1) {
+        const uint32_t lo = sft == 16 ? 0x0000FFFFu : sft == 8 ? 0x00FF00FFu : sft == 4 ? 0x0F0F0F0Fu
+                          : sft == 2 ? 0x33333333u : 0x55555555u;
+        const uint32_t other = __shfl_xor_sync(0xffffffffu, x, sft);
+        if ((lane & sft) == 0) x = (x & lo) | ((other & lo) << sft);
+        else x = (x & ~lo) | ((other & ~lo) >> sft);
+    }
+    return x;
+}
+
 // First index in [lo, hi) where the monotone predicate (true ... true,
 // false ... false) is false, or hi. All 32 lanes of a warp call it and get the
 // same answer after about log32(hi - lo) rounds of one probe per lane.

@@ -1709,19 +1709,6 @@ __global__ void __launch_bounds__(256) tr_write_kernel(const int32_t *__restrict
 //         row by row (lane = column) and column by column (lane = row),
 //         which is cheaper once most lanes hold an entry.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
-    const int lane = threadIdx.x & 31;
-#pragma unroll
-    for (int sft = 16; sft >= 1; sft >>= 1) {
-        const uint32_t lo = sft == 16 ? 0x0000FFFFu : sft == 8 ? 0x00FF00FFu : sft == 4 ? 0x0F0F0F0Fu
-                          : sft == 2 ? 0x33333333u : 0x55555555u;
-        const uint32_t other = __shfl_xor_sync(0xffffffffu, x, sft);
-        if ((lane & sft) == 0) x = (x & lo) | ((other & lo) << sft);
-        else x = (x & ~lo) | ((other & ~lo) >> sft);
-    }
-    return x;
-}
-
 __global__ void __launch_bounds__(256) trb_count_kernel(const uint32_t *__restrict__ keepbits, int32_t rows,
                                                         int32_t wpr, int32_t cols, int32_t *__restrict__ cnt) {
     pdl_enter();
@@ -1868,10 +1855,11 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
     }
 }
 
-// Transposed copy from a keep bitmask and word positions (cols % 32 == 0);
-// `scratch` holds the per-block column counts and the column totals.
-int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t *wordpos, void *scratch,
-                            size_t scratch_bytes, cudaStream_t s) {
+// Column pointers of the transposed copy (t_row_ptr) and, per 32-row block
+// and column, the block's offset in the column's run (in `scratch`, nb x cols
+// int32, followed by the column totals), from a keep bitmask (cols % 32 == 0).
+int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch, size_t scratch_bytes,
+                           cudaStream_t s) {
     const int32_t rows = w->rows, cols = w->cols;
     const int32_t wpr = cols / 32;
     CSRT_ARG(scratch_bytes >= transpose_scratch_bytes(rows, cols), "scratch too small for the transposed copy");
@@ -1883,9 +1871,25 @@ int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t
     launch_pdl(trb_count_kernel, dim3(grid), dim3(256), 0, s, keepbits, rows, wpr, cols, cnt);
     launch_pdl(tr_colscan_kernel, dim3(ceil_div(cols, 32)), dim3(256), 0, s, cnt, nb, cols, coltot);
     launch_pdl(scan_single_block_kernel, dim3(1), dim3(1024), 0, s, coltot, cols, w->t_row_ptr);
+    count_launch(3);
+    return check_launch("transposed-copy count kernels");
+}
+
+// Transposed copy from a keep bitmask and word positions (cols % 32 == 0);
+// `scratch` holds the per-block column counts and the column totals.
+int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t *wordpos, void *scratch,
+                            size_t scratch_bytes, cudaStream_t s) {
+    int rc = transpose_bits_prepare(w, keepbits, scratch, scratch_bytes, s);
+    if (rc) return rc;
+    const int32_t rows = w->rows, cols = w->cols;
+    const int32_t wpr = cols / 32;
+    const int32_t *cnt = static_cast<const int32_t *>(scratch);
+    const int nb = (int)ceil_div<int64_t>(rows, 32);
+    const int64_t warps = (int64_t)nb * wpr;
+    const unsigned grid = (unsigned)ceil_div<int64_t>(warps * 32, 256);
     launch_pdl(trb_write_kernel, dim3(grid), dim3(256), 0, s, keepbits, wordpos, rows, wpr, cols, cnt, w->t_row_ptr,
                w->val, w->t_col_idx, w->t_val, w->t_pos, w->capacity);
-    count_launch(4);
+    count_launch(1);
     return check_launch("transpose-from-bits kernels");
 }
 

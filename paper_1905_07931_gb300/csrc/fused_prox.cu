@@ -20,11 +20,16 @@
 //     the segment.
 //  3. fp_rowscan_kernel + scan_clamped_kernel: per-row offsets of the
 //     segments and the new row pointers (clamped to the capacity in w_out).
-//  4. gemm_prox_tc_kernel<write>: the same GEMM again; the epilogue recomputes
+//  4. With a transposed copy wanted: its column counts per 32-row block (from
+//     the keep bitmask), their scan down each column and the column pointers
+//     (compact.cu, transpose_bits_prepare).
+//  5. gemm_prox_tc_kernel<write>: the same GEMM again; the epilogue recomputes
 //     z, passes each 32 x 32 block through shared memory and writes the kept
 //     entries of one row at a time at their final positions (a coalesced run
-//     per row and 32 columns), plus the word positions from which the
-//     transposed copy is built out of the bitmask.
+//     per row and 32 columns). With the transposed copy (kT) the same staged
+//     block is then walked column by column (lane = row): each column's kept
+//     rows form one run of the transposed arrays, and each kept entry's
+//     transposed position goes to t_pos during the row walk.
 // The result is bit-identical to weight_grad_dense (TF32) followed by
 // prox_update_compact.
 #include "tc_common.cuh"
@@ -33,6 +38,8 @@ namespace csrt {
 
 int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t *wordpos, void *scratch,
                             size_t scratch_bytes, cudaStream_t s);
+int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch, size_t scratch_bytes,
+                           cudaStream_t s);
 size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
 
 // Segments (the unit of the per-row offsets) are 64 columns, two 32-column
@@ -194,20 +201,33 @@ struct FpArgs {
     WsHeader *hdr;
 };
 
+// Write pass with the transposed copy: the start of each column's run (t_rp)
+// and, per 32-row block and column, the block's offset in it (t_off), from the
+// count pass's keep bits; the transposed arrays.
+struct FpTArgs {
+    const int32_t *t_rp, *t_off;
+    int32_t *t_col;
+    float *t_val;
+    int32_t *t_pos;
+};
+
 
 // Per-tile inputs of an epilogue thread (its row of the tile's column span):
 // the stored-weight bitmask of each word, the index of the span's first stored
-// weight and, in the write pass, the position of its first kept entry.
-template <int W>
+// weight and, in the write pass, the position of its first kept entry and
+// (transposed copy) the start of the run of column 32 * word + lane in the
+// warp's 32-row block.
+template <int W, bool kT>
 struct FpMeta {
     uint32_t ob[W];
     uint32_t kb[W];   // write pass: the keep bitmask the count pass wrote
+    int32_t cb[kT ? W : 1];
     int32_t o0, pos;
 };
 
-template <bool kWrite, int W>
-__device__ __forceinline__ void fp_load_meta(const FpArgs &a, int t, int num_tiles, int tiles_n, int h, int64_t rowq,
-                                             FpMeta<W> &m) {
+template <bool kWrite, bool kT, int W>
+__device__ __forceinline__ void fp_load_meta(const FpArgs &a, const FpTArgs &ta, int t, int num_tiles, int tiles_n,
+                                             int h, int64_t rowq, FpMeta<W, kT> &m) {
     const int mt = t / tiles_n, nt = t % tiles_n;
     const int64_t row = (int64_t)mt * kTcBM + rowq;
     const bool rv = t < num_tiles && row < a.m;
@@ -221,6 +241,15 @@ __device__ __forceinline__ void fp_load_meta(const FpArgs &a, int t, int num_til
         m.kb[c] = (kWrite && rv && word0 + c < a.wpr) ? __ldg(a.kbits + row * a.wpr + word0 + c) : 0u;
     m.o0 = sv ? __ldg(a.ostart + row * (a.nt + 1) + seg0) : 0;
     m.pos = (kWrite && sv) ? __ldg(a.row_ptr_out + row) + __ldg(a.counts + row * a.nt + seg0) : 0;
+    if constexpr (kT) {
+        const int64_t brow = (int64_t)mt * kTcBM + (rowq & ~(int64_t)31);   // the warp's 32-row block
+        const bool bv = t < num_tiles && brow < a.m;
+#pragma unroll
+        for (int c = 0; c < W; ++c) {
+            const int64_t col = (int64_t)(word0 + c) * 32 + (rowq & 31);
+            m.cb[c] = (bv && word0 + c < a.wpr) ? __ldg(ta.t_rp + col) + __ldg(ta.t_off + (brow >> 5) * a.k + col) : 0;
+        }
+    }
 }
 
 // The first N stored weights of a word (its bitmask ob, first index o).
@@ -232,18 +261,49 @@ __device__ __forceinline__ void fp_load_words(const float *__restrict__ old_val,
     for (int u = 0; u < N; ++u) wv[u] = u < nc ? __ldg(old_val + o + u) : 0.f;
 }
 
+// Transposed copy of one staged 32 x 32 word (element (r, j) at r*32 + (j ^
+// ((r & 7) << 2))), lane = row: each column j's kept rows form one run in row
+// order starting at cb_j, the start of column j's run in this 32-row block
+// (cm: lane j's column mask, bit r = row r kept; cbl: lane j's cb_j).
+template <bool kCheck>
+__device__ __forceinline__ void fp_write_transposed(const float *xb, uint32_t cm, int32_t cbl, int64_t row0,
+                                                    float thr, int32_t cap32, int32_t *__restrict__ t_col,
+                                                    float *__restrict__ t_val) {
+    const int lane = threadIdx.x & 31;
+    const uint32_t lt = (1u << lane) - 1u;
+    const int sw = (lane & 7) << 2;
+#pragma unroll 4
+    for (int j = 0; j < 32; ++j) {
+        const uint32_t cmj = __shfl_sync(0xffffffffu, cm, j);
+        const int32_t cbj = __shfl_sync(0xffffffffu, cbl, j);
+        if ((cmj >> lane) & 1u) {
+            const int32_t pc = cbj + __popc(cmj & lt);
+            if (!kCheck || pc < cap32) {
+                const float z = xb[lane * 32 + (j ^ sw)];
+                t_col[pc] = (int32_t)(row0 + lane);
+                t_val[pc] = __fsub_rn(z, copysignf(thr, z));
+            }
+        }
+    }
+}
+
 // Write pass, column domain: lane = column within a word. Rows are taken in
 // groups of G (independent, so their loads overlap); each row's kept entries
 // of the W words of the span form one run of consecutive positions, written
 // word after word with no other store in between, so the 32-byte sector shared
 // by two words' runs is completed at once (a sector left half-written while
 // other rows' stores go by is fetched back from DRAM to be merged).
-template <bool kCheck, int G, int W>
+// With kT (W = 1) each kept entry's transposed position goes to t_pos: the
+// start of its column's run in the block (cbl) plus the kept rows above it.
+template <bool kCheck, int G, int W, bool kT = false>
 __device__ __forceinline__ void fp_write_span(const float *xb, const int (&lx)[8], uint32_t lt,
                                               const uint32_t (&kb)[W], int32_t pos, int32_t col0, float thr,
                                               int32_t cap32, int32_t *__restrict__ out_col,
-                                              float *__restrict__ out_val) {
+                                              float *__restrict__ out_val, int32_t cbl = 0,
+                                              int32_t *__restrict__ t_pos = nullptr) {
     const int lane = threadIdx.x & 31;
+    static_assert(!kT || W == 1, "the transposed positions are written one word at a time");
+    int32_t pc = cbl;   // kT: this column's next transposed position
 #pragma unroll
     for (int i0 = 0; i0 < 32; i0 += G) {
         uint32_t kw[G][W];
@@ -265,10 +325,13 @@ __device__ __forceinline__ void fp_write_span(const float *xb, const int (&lx)[8
             for (int c = 0; c < W; ++c) {
                 const uint32_t kwi = kw[u][c];
                 const int32_t q = pw + __popc(kwi & lt);
-                if (((kwi >> lane) & 1u) && (!kCheck || q < cap32)) {
+                const bool keep = (kwi >> lane) & 1u;
+                if (keep && (!kCheck || q < cap32)) {
                     out_col[q] = col0 + c * 32 + lane;
                     out_val[q] = __fsub_rn(z[u][c], copysignf(thr, z[u][c]));
+                    if (kT && (!kCheck || pc < cap32)) t_pos[q] = pc;
                 }
+                if (kT) pc += keep ? 1 : 0;
                 pw += __popc(kwi);
             }
         }
@@ -287,11 +350,22 @@ __device__ __forceinline__ void fp_write_span(const float *xb, const int (&lx)[8
 // contiguous runs.
 constexpr int kFpWalkMax = 96;
 
-template <bool kCheck>
+// With kT (cm, cbl, row0 as for fp_write_transposed): the word's transposed
+// runs first, from the staged block, then each kept entry's transposed
+// position to t_pos.
+template <bool kCheck, bool kT = false>
 __device__ __forceinline__ void fp_write_compact(const float *xb, uint8_t *cb, float *xr, int sw, uint32_t kw,
                                                  int32_t pos, int total, int32_t col0, float thr, int32_t cap32,
-                                                 int32_t *__restrict__ out_col, float *__restrict__ out_val) {
+                                                 int32_t *__restrict__ out_col, float *__restrict__ out_val,
+                                                 uint32_t cm = 0, int32_t cbl = 0, int64_t row0 = 0,
+                                                 int32_t *__restrict__ t_col = nullptr,
+                                                 float *__restrict__ t_val = nullptr,
+                                                 int32_t *__restrict__ t_pos = nullptr) {
     const int lane = threadIdx.x & 31;
+    if (kT) {
+        fp_write_transposed<kCheck>(xb, cm, cbl, row0, thr, cap32, t_col, t_val);
+        __syncwarp();   // the block's reads done before the rows are compacted in place
+    }
     const int cnt = __popc(kw);
     const int maxc = (int)__reduce_max_sync(0xffffffffu, (unsigned)cnt);
     uint32_t bits = kw;
@@ -323,9 +397,15 @@ __device__ __forceinline__ void fp_write_compact(const float *xb, uint8_t *cb, f
         }
         const int j = e - __shfl_sync(0xffffffffu, rpre, r);
         const int32_t q = __shfl_sync(0xffffffffu, pos, r) + j;
+        const int jb = e < total ? cb[r * 32 + j] : 0;   // the entry's column in the word
         if (e < total && (!kCheck || q < cap32)) {
             out_val[q] = xb[r * 32 + (j ^ ((r & 7) << 2))];
-            out_col[q] = col0 + cb[r * 32 + j];
+            out_col[q] = col0 + jb;
+        }
+        if (kT) {
+            const uint32_t cmj = __shfl_sync(0xffffffffu, cm, jb);
+            const int32_t pc = __shfl_sync(0xffffffffu, cbl, jb) + __popc(cmj & ((1u << r) - 1u));
+            if (e < total && (!kCheck || (q < cap32 && pc < cap32))) t_pos[q] = pc;
         }
     }
 }
@@ -342,10 +422,11 @@ __device__ __forceinline__ void fp_write_compact(const float *xb, uint8_t *cb, f
 // row. The write pass then switches to the column domain (lane = column): for
 // each row of the 32 the kept entries form one run of consecutive positions,
 // written with coalesced stores.
-template <bool kWrite>
+// kT (write pass only): the transposed copy is written too (FpTArgs).
+template <bool kWrite, bool kT>
 __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
     gemm_prox_tc_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
-                        FpArgs a, int32_t tiles_n, int32_t num_tiles) {
+                        FpArgs a, FpTArgs ta, int32_t tiles_n, int32_t num_tiles) {
     pdl_enter();
     constexpr int kEpi = FpShape<kWrite>::kEpi, kStages = FpShape<kWrite>::kStages;
     constexpr int kFpPre = FpShape<kWrite>::kPre, kGroup = FpShape<kWrite>::kGroup;
@@ -455,9 +536,9 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
         float tsum = 0.f;
         // software pipeline: the next tile's metadata one tile ahead, the
         // next word's stored weights one word ahead
-        FpMeta<kSpanWords> cur, nxt;
-        fp_load_meta<kWrite>(a, blockIdx.x, num_tiles, tiles_n, h, rowq, cur);
-        fp_load_meta<kWrite>(a, blockIdx.x + gridDim.x, num_tiles, tiles_n, h, rowq, nxt);
+        FpMeta<kSpanWords, kT> cur, nxt;
+        fp_load_meta<kWrite, kT>(a, ta, blockIdx.x, num_tiles, tiles_n, h, rowq, cur);
+        fp_load_meta<kWrite, kT>(a, ta, blockIdx.x + gridDim.x, num_tiles, tiles_n, h, rowq, nxt);
         float wv_n[kFpPre];
         int32_t ow_n = cur.o0;
         fp_load_words(a.old_val, cur.ob[0], ow_n, wv_n);
@@ -567,7 +648,7 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
                         cnt = 0;
                     }
                 } else {
-                    if (rv && word < a.wpr && a.wordpos) a.wordpos[row * a.wpr + word] = imin(pos, cap32);
+                    if (!kT && rv && word < a.wpr && a.wordpos) a.wordpos[row * a.wpr + word] = imin(pos, cap32);
                     pos += __popc(cur.kb[c]);
                     if (c % kSW == kSW - 1) {
                         // a group of words is staged: write it row by row. The
@@ -583,25 +664,52 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
                         }
                         const int total =
                             kSW == 1 ? (int)__reduce_add_sync(0xffffffffu, (unsigned)__popc(kbg[0])) : kFpWalkMax + 1;
-                        if (total <= kFpWalkMax) {
+                        if constexpr (kT && kSW == 1) {
+                            // the transposed copy too: lane j's column mask and run start in this 32-row block
+                            const uint32_t cm = warp_transpose32(kbg[0]);
+                            const int32_t cbl = cur.cb[c];
+                            const int64_t row0 = row - lane;
+                            if (total <= kFpWalkMax) {
+                                if (fits)
+                                    fp_write_compact<false, true>(xb, cb, xr, sw, kbg[0], pg, total, word * 32, a.thr,
+                                                                  cap32, a.out_col, a.out_val, cm, cbl, row0, ta.t_col,
+                                                                  ta.t_val, ta.t_pos);
+                                else
+                                    fp_write_compact<true, true>(xb, cb, xr, sw, kbg[0], pg, total, word * 32, a.thr,
+                                                                 cap32, a.out_col, a.out_val, cm, cbl, row0, ta.t_col,
+                                                                 ta.t_val, ta.t_pos);
+                            } else {
+                                if (fits) {
+                                    fp_write_span<false, kGroup, 1, true>(xb, lx, lt, kbg, pg, word * 32, a.thr, cap32,
+                                                                          a.out_col, a.out_val, cbl, ta.t_pos);
+                                    fp_write_transposed<false>(xb, cm, cbl, row0, a.thr, cap32, ta.t_col, ta.t_val);
+                                } else {
+                                    fp_write_span<true, kGroup, 1, true>(xb, lx, lt, kbg, pg, word * 32, a.thr, cap32,
+                                                                         a.out_col, a.out_val, cbl, ta.t_pos);
+                                    fp_write_transposed<true>(xb, cm, cbl, row0, a.thr, cap32, ta.t_col, ta.t_val);
+                                }
+                            }
+                        } else {
+                          if (total <= kFpWalkMax) {
                             if (fits)
                                 fp_write_compact<false>(xb, cb, xr, sw, kbg[0], pg, total, word * 32, a.thr, cap32,
                                                         a.out_col, a.out_val);
                             else
                                 fp_write_compact<true>(xb, cb, xr, sw, kbg[0], pg, total, word * 32, a.thr, cap32,
                                                        a.out_col, a.out_val);
-                        } else if (fits) {
+                          } else if (fits) {
                             fp_write_span<false, kGroup, kSW>(xb, lx, lt, kbg, pg, (word + 1 - kSW) * 32, a.thr, cap32,
                                                               a.out_col, a.out_val);
-                        } else {
+                          } else {
                             fp_write_span<true, kGroup, kSW>(xb, lx, lt, kbg, pg, (word + 1 - kSW) * 32, a.thr, cap32,
                                                              a.out_col, a.out_val);
+                          }
                         }
                     }
                 }
             }
             cur = nxt;
-            fp_load_meta<kWrite>(a, t + 2 * gridDim.x, num_tiles, tiles_n, h, rowq, nxt);
+            fp_load_meta<kWrite, kT>(a, ta, t + 2 * gridDim.x, num_tiles, tiles_n, h, rowq, nxt);
         }
         if (!kWrite && __any_sync(0xffffffffu, tsum != tsum) && lane == 0) s_nonfinite = 1;
     }
@@ -697,10 +805,12 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             fp_smem_bytes<false>()));
-        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             fp_smem_bytes<true>()));
+        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<false, false>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, fp_smem_bytes<false>()));
+        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<true, false>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, fp_smem_bytes<true>()));
+        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<true, true>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, fp_smem_bytes<true>()));
         attr_set[dev] = true;
     }
     launch_pdl(fp_oldbits_kernel, dim3((unsigned)ceil_div<int64_t>(m, 8)), dim3(256), 0, s, w_in->row_ptr,
@@ -722,13 +832,14 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     a.out_col = w_out->col_idx;
     a.out_val = w_out->val;
     a.wordpos = want_t ? wordpos : nullptr;
+    FpTArgs ta{};   // the transposed copy's arrays, for the write pass (set below)
     a.capacity = w_out->capacity;
     a.hdr = static_cast<WsHeader *>(ws);
     const int tiles_m = (int)ceil_div<int64_t>(m, kTcBM), tiles_n = (int)ceil_div<int64_t>(k, kTcBN);
     const int tiles = tiles_m * tiles_n;
     const unsigned grid = (unsigned)imin(tiles, num_sms());
-    launch_pdl(gemm_prox_tc_kernel<false>, dim3(grid), dim3(fp_threads<false>()), fp_smem_bytes<false>(), s, ma, mb, a,
-               tiles_n, tiles);
+    launch_pdl(gemm_prox_tc_kernel<false, false>, dim3(grid), dim3(fp_threads<false>()), fp_smem_bytes<false>(), s,
+               ma, mb, a, ta, tiles_n, tiles);
     launch_pdl(fp_rowscan_kernel, dim3((unsigned)ceil_div<int64_t>((int64_t)m * 32, 256)), dim3(256), 0, s, counts, m,
                L.nt, rowtot);
     count_launch(3);
@@ -736,11 +847,23 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     // pass and clamped to the capacity in w_out (overflow reported)
     int rc = scan_exclusive_i32_clamped(rowtot, m, rawptr, w_out->row_ptr, w_out->capacity, ws, s);
     if (rc) return rc;
-    launch_pdl(gemm_prox_tc_kernel<true>, dim3(grid), dim3(fp_threads<true>()), fp_smem_bytes<true>(), s, ma, mb, a,
-               tiles_n, tiles);
+    if (want_t) {
+        // the transposed copy's column pointers and per-block offsets from the keep bits; the write pass
+        // writes its arrays
+        rc = transpose_bits_prepare(w_out, kbits, base + L.off_tr, L.total - L.off_tr, s);
+        if (rc) return rc;
+        ta.t_rp = w_out->t_row_ptr;
+        ta.t_off = reinterpret_cast<const int32_t *>(base + L.off_tr);
+        ta.t_col = w_out->t_col_idx;
+        ta.t_val = w_out->t_val;
+        ta.t_pos = w_out->t_pos;
+    }
+    if (want_t)
+        launch_pdl(gemm_prox_tc_kernel<true, true>, dim3(grid), dim3(fp_threads<true>()), fp_smem_bytes<true>(), s,
+                   ma, mb, a, ta, tiles_n, tiles);
+    else
+        launch_pdl(gemm_prox_tc_kernel<true, false>, dim3(grid), dim3(fp_threads<true>()), fp_smem_bytes<true>(), s,
+                   ma, mb, a, ta, tiles_n, tiles);
     count_launch(1);
-    rc = check_launch("fused weight-gradient + prox kernels");
-    if (rc) return rc;
-    if (want_t) rc = transpose_from_bits_ext(w_out, kbits, wordpos, base + L.off_tr, L.total - L.off_tr, s);
-    return rc;
+    return check_launch("fused weight-gradient + prox kernels");
 }
