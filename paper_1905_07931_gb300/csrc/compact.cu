@@ -1857,9 +1857,10 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
 
 // Column pointers of the transposed copy (t_row_ptr) and, per 32-row block
 // and column, the block's offset in the column's run (in `scratch`, nb x cols
-// int32, followed by the column totals), from a keep bitmask (cols % 32 == 0).
+// int32, followed by the column totals), from a keep bitmask (cols % 32 == 0)
+// or, with have_counts, from the per-block column counts already in scratch.
 int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch, size_t scratch_bytes,
-                           cudaStream_t s) {
+                           cudaStream_t s, bool have_counts) {
     const int32_t rows = w->rows, cols = w->cols;
     const int32_t wpr = cols / 32;
     CSRT_ARG(scratch_bytes >= transpose_scratch_bytes(rows, cols), "scratch too small for the transposed copy");
@@ -1868,10 +1869,13 @@ int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch,
     int32_t *coltot = cnt + (int64_t)nb * cols;
     const int64_t warps = (int64_t)nb * wpr;
     const unsigned grid = (unsigned)ceil_div<int64_t>(warps * 32, 256);
-    launch_pdl(trb_count_kernel, dim3(grid), dim3(256), 0, s, keepbits, rows, wpr, cols, cnt);
+    if (!have_counts) {   // else the caller's kernel wrote them
+        launch_pdl(trb_count_kernel, dim3(grid), dim3(256), 0, s, keepbits, rows, wpr, cols, cnt);
+        count_launch(1);
+    }
     launch_pdl(tr_colscan_kernel, dim3(ceil_div(cols, 32)), dim3(256), 0, s, cnt, nb, cols, coltot);
     launch_pdl(scan_single_block_kernel, dim3(1), dim3(1024), 0, s, coltot, cols, w->t_row_ptr);
-    count_launch(3);
+    count_launch(2);
     return check_launch("transposed-copy count kernels");
 }
 
@@ -1879,7 +1883,7 @@ int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch,
 // `scratch` holds the per-block column counts and the column totals.
 int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t *wordpos, void *scratch,
                             size_t scratch_bytes, cudaStream_t s) {
-    int rc = transpose_bits_prepare(w, keepbits, scratch, scratch_bytes, s);
+    int rc = transpose_bits_prepare(w, keepbits, scratch, scratch_bytes, s, false);
     if (rc) return rc;
     const int32_t rows = w->rows, cols = w->cols;
     const int32_t wpr = cols / 32;

@@ -20,8 +20,9 @@
 //     the segment.
 //  3. fp_rowscan_kernel + scan_clamped_kernel: per-row offsets of the
 //     segments and the new row pointers (clamped to the capacity in w_out).
-//  4. With a transposed copy wanted: its column counts per 32-row block (from
-//     the keep bitmask), their scan down each column and the column pointers
+//  4. With a transposed copy wanted: the count pass also writes its column
+//     counts per 32-row block (a 32 x 32 bit transpose of the rows' keep
+//     words); their scan down each column and the column pointers follow
 //     (compact.cu, transpose_bits_prepare).
 //  5. gemm_prox_tc_kernel<write>: the same GEMM again; the epilogue recomputes
 //     z, passes each 32 x 32 block through shared memory and writes the kept
@@ -39,7 +40,7 @@ namespace csrt {
 int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t *wordpos, void *scratch,
                             size_t scratch_bytes, cudaStream_t s);
 int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch, size_t scratch_bytes,
-                           cudaStream_t s);
+                           cudaStream_t s, bool have_counts);
 size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
 
 // Segments (the unit of the per-row offsets) are 64 columns, two 32-column
@@ -209,6 +210,7 @@ struct FpTArgs {
     int32_t *t_col;
     float *t_val;
     int32_t *t_pos;
+    int32_t *t_cnt;   // count pass: kept rows per (32-row block, column)
 };
 
 
@@ -422,7 +424,8 @@ __device__ __forceinline__ void fp_write_compact(const float *xb, uint8_t *cb, f
 // row. The write pass then switches to the column domain (lane = column): for
 // each row of the 32 the kept entries form one run of consecutive positions,
 // written with coalesced stores.
-// kT (write pass only): the transposed copy is written too (FpTArgs).
+// kT: the transposed copy too (FpTArgs): its column counts per 32-row block
+// (count pass) or its arrays (write pass).
 template <bool kWrite, bool kT>
 __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
     gemm_prox_tc_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
@@ -641,6 +644,11 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
                 }
                 if (!kWrite) {
                     if (rv && word < a.wpr) a.kbits[row * a.wpr + word] = kw;
+                    if constexpr (kT) {   // lane j: kept rows of column 32 * word + j in this 32-row block
+                        const uint32_t cmc = warp_transpose32(kw);
+                        const int64_t brow = row - lane;
+                        if (brow < a.m && word < a.wpr) ta.t_cnt[(brow >> 5) * a.k + word * 32 + lane] = __popc(cmc);
+                    }
                     cnt += __popc(kw);
                     if (c % kFpTileWords == kFpTileWords - 1) {   // segment complete
                         const int seg = word / kFpTileWords;
@@ -811,6 +819,8 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, fp_smem_bytes<true>()));
         CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<true, true>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, fp_smem_bytes<true>()));
+        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<false, true>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, fp_smem_bytes<false>()));
         attr_set[dev] = true;
     }
     launch_pdl(fp_oldbits_kernel, dim3((unsigned)ceil_div<int64_t>(m, 8)), dim3(256), 0, s, w_in->row_ptr,
@@ -832,14 +842,19 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     a.out_col = w_out->col_idx;
     a.out_val = w_out->val;
     a.wordpos = want_t ? wordpos : nullptr;
-    FpTArgs ta{};   // the transposed copy's arrays, for the write pass (set below)
+    FpTArgs ta{};   // the transposed copy: the count pass's column counts here, the write pass's arrays below
+    if (want_t) ta.t_cnt = reinterpret_cast<int32_t *>(base + L.off_tr);
     a.capacity = w_out->capacity;
     a.hdr = static_cast<WsHeader *>(ws);
     const int tiles_m = (int)ceil_div<int64_t>(m, kTcBM), tiles_n = (int)ceil_div<int64_t>(k, kTcBN);
     const int tiles = tiles_m * tiles_n;
     const unsigned grid = (unsigned)imin(tiles, num_sms());
-    launch_pdl(gemm_prox_tc_kernel<false, false>, dim3(grid), dim3(fp_threads<false>()), fp_smem_bytes<false>(), s,
-               ma, mb, a, ta, tiles_n, tiles);
+    if (want_t)
+        launch_pdl(gemm_prox_tc_kernel<false, true>, dim3(grid), dim3(fp_threads<false>()), fp_smem_bytes<false>(), s,
+                   ma, mb, a, ta, tiles_n, tiles);
+    else
+        launch_pdl(gemm_prox_tc_kernel<false, false>, dim3(grid), dim3(fp_threads<false>()), fp_smem_bytes<false>(), s,
+                   ma, mb, a, ta, tiles_n, tiles);
     launch_pdl(fp_rowscan_kernel, dim3((unsigned)ceil_div<int64_t>((int64_t)m * 32, 256)), dim3(256), 0, s, counts, m,
                L.nt, rowtot);
     count_launch(3);
@@ -848,9 +863,9 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     int rc = scan_exclusive_i32_clamped(rowtot, m, rawptr, w_out->row_ptr, w_out->capacity, ws, s);
     if (rc) return rc;
     if (want_t) {
-        // the transposed copy's column pointers and per-block offsets from the keep bits; the write pass
-        // writes its arrays
-        rc = transpose_bits_prepare(w_out, kbits, base + L.off_tr, L.total - L.off_tr, s);
+        // the transposed copy's column pointers and per-block offsets from the count pass's column counts;
+        // the write pass writes its arrays
+        rc = transpose_bits_prepare(w_out, kbits, base + L.off_tr, L.total - L.off_tr, s, true);
         if (rc) return rc;
         ta.t_rp = w_out->t_row_ptr;
         ta.t_off = reinterpret_cast<const int32_t *>(base + L.off_tr);
