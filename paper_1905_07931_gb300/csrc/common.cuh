@@ -160,6 +160,76 @@ __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
     return x;
 }
 
+// Exclusive scan of n int32 values into out[0..n] (out[n] = the total) by one
+// block of 1024 threads, each taking a contiguous run; with out_clamped also
+// the same values clamped to `capacity`, a total above it reported in hdr
+// (CSRT_DEV_CAPACITY and the needed count).
+__device__ __forceinline__ void scan_block_1024(const int32_t *__restrict__ in, int32_t n, int32_t *__restrict__ out,
+                                                int32_t *__restrict__ out_clamped, int64_t capacity, WsHeader *hdr) {
+    __shared__ int32_t s_warp[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int per = (n + 1023) / 1024;
+    const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+    int32_t local = 0;
+    for (int i = i0; i < i1; ++i) local += in[i];
+    int32_t incl = local;
+    for (int off = 1; off < 32; off <<= 1) {
+        int32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    int32_t wp = 0, total = 0;
+    for (int w = 0; w < 32; ++w) {
+        if (w < warp) wp += s_warp[w];
+        total += s_warp[w];
+    }
+    int32_t run = incl - local + wp;
+    for (int i = i0; i < i1; ++i) {
+        out[i] = run;
+        if (out_clamped) out_clamped[i] = (int32_t)(run < capacity ? run : capacity);
+        run += in[i];
+    }
+    if (tid == 0) {
+        out[n] = total;
+        if (out_clamped) {
+            out_clamped[n] = (int32_t)(total < capacity ? total : capacity);
+            if (total > capacity) {
+                dev_flag(hdr, CSRT_DEV_CAPACITY);
+                atomicMax(&hdr->required, (unsigned long long)total);
+            }
+        }
+    }
+}
+
+// Block bx of a column scan over 32-row blocks, 256 threads (8 warps x 32
+// columns): for columns 32bx .. 32bx+31, the per-block counts cnt[b][j]
+// (nb x cols) become their exclusive prefix down the column, coltot[j] the
+// column's total.
+__device__ __forceinline__ void colscan_block(int32_t *__restrict__ cnt, int32_t nb, int32_t cols,
+                                              int32_t *__restrict__ coltot, int bx) {
+    __shared__ int32_t seg[8][32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int j = bx * 32 + lane;
+    const int b0 = (int)(((int64_t)nb * warp) / 8), b1 = (int)(((int64_t)nb * (warp + 1)) / 8);
+    int32_t sum = 0;
+    if (j < cols)
+        for (int b = b0; b < b1; ++b) sum += cnt[(int64_t)b * cols + j];
+    seg[warp][lane] = sum;
+    __syncthreads();
+    int32_t run = 0;
+    for (int w = 0; w < warp; ++w) run += seg[w][lane];
+    if (j < cols) {
+        for (int b = b0; b < b1; ++b) {
+            int32_t *p = cnt + (int64_t)b * cols + j;
+            const int32_t v = *p;
+            *p = run;
+            run += v;
+        }
+        if (warp == 7) coltot[j] = run;
+    }
+}
+
 // First index in [lo, hi) where the monotone predicate (true ... true,
 // false ... false) is false, or hi. All 32 lanes of a warp call it and get the
 // same answer after about log32(hi - lo) rounds of one probe per lane.

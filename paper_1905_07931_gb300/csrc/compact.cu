@@ -1510,56 +1510,14 @@ __global__ void __launch_bounds__(256) tr_count_kernel(const int32_t *__restrict
 __global__ void __launch_bounds__(256) tr_colscan_kernel(int32_t *__restrict__ cnt, int32_t nb,
                                                          int32_t cols, int32_t *__restrict__ coltot) {
     pdl_enter();
-    __shared__ int32_t seg[8][32];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int j = blockIdx.x * 32 + lane;
-    const int b0 = (int)(((int64_t)nb * warp) / 8), b1 = (int)(((int64_t)nb * (warp + 1)) / 8);
-    int32_t sum = 0;
-    if (j < cols)
-        for (int b = b0; b < b1; ++b) sum += cnt[(int64_t)b * cols + j];
-    seg[warp][lane] = sum;
-    __syncthreads();
-    int32_t run = 0;
-    for (int w = 0; w < warp; ++w) run += seg[w][lane];
-    if (j < cols) {
-        for (int b = b0; b < b1; ++b) {
-            int32_t *p = cnt + (int64_t)b * cols + j;
-            const int32_t v = *p;
-            *p = run;
-            run += v;
-        }
-        if (warp == 7) coltot[j] = run;
-    }
+    colscan_block(cnt, nb, cols, coltot, blockIdx.x);
 }
 
 // Exclusive scan of n values into out[0..n] (out[n] = total); one block.
 __global__ void __launch_bounds__(1024) scan_single_block_kernel(const int32_t *__restrict__ in, int32_t n,
                                                                  int32_t *__restrict__ out) {
     pdl_enter();
-    __shared__ int32_t s_warp[32];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int per = (n + 1023) / 1024;
-    const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
-    int32_t local = 0;
-    for (int i = i0; i < i1; ++i) local += in[i];
-    int32_t incl = local;
-    for (int off = 1; off < 32; off <<= 1) {
-        int32_t y = __shfl_up_sync(0xffffffffu, incl, off);
-        if (lane >= off) incl += y;
-    }
-    if (lane == 31) s_warp[warp] = incl;
-    __syncthreads();
-    int32_t wp = 0, total = 0;
-    for (int w = 0; w < 32; ++w) {
-        if (w < warp) wp += s_warp[w];
-        total += s_warp[w];
-    }
-    int32_t run = incl - local + wp;
-    for (int i = i0; i < i1; ++i) {
-        out[i] = run;
-        run += in[i];
-    }
-    if (tid == 0) out[n] = total;
+    scan_block_1024(in, n, out, nullptr, 0, nullptr);
 }
 
 // The same scan, also writing the row pointers clamped to a CSR's capacity
@@ -1571,38 +1529,7 @@ __global__ void __launch_bounds__(1024) scan_clamped_kernel(const int32_t *__res
                                                             int32_t *__restrict__ out_clamped, int64_t capacity,
                                                             WsHeader *hdr) {
     pdl_enter();
-    __shared__ int32_t s_warp[32];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int per = (n + 1023) / 1024;
-    const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
-    int32_t local = 0;
-    for (int i = i0; i < i1; ++i) local += in[i];
-    int32_t incl = local;
-    for (int off = 1; off < 32; off <<= 1) {
-        int32_t y = __shfl_up_sync(0xffffffffu, incl, off);
-        if (lane >= off) incl += y;
-    }
-    if (lane == 31) s_warp[warp] = incl;
-    __syncthreads();
-    int32_t wp = 0, total = 0;
-    for (int w = 0; w < 32; ++w) {
-        if (w < warp) wp += s_warp[w];
-        total += s_warp[w];
-    }
-    int32_t run = incl - local + wp;
-    for (int i = i0; i < i1; ++i) {
-        out[i] = run;
-        out_clamped[i] = (int32_t)imin<int64_t>(run, capacity);
-        run += in[i];
-    }
-    if (tid == 0) {
-        out[n] = total;
-        out_clamped[n] = (int32_t)imin<int64_t>(total, capacity);
-        if (total > capacity) {
-            dev_flag(hdr, CSRT_DEV_CAPACITY);
-            atomicMax(&hdr->required, (unsigned long long)total);
-        }
-    }
+    scan_block_1024(in, n, out, out_clamped, capacity, hdr);
 }
 
 int scan_exclusive_i32_clamped(const int32_t *in, int32_t n, int32_t *out, int32_t *out_clamped, int64_t capacity,
@@ -1857,10 +1784,9 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
 
 // Column pointers of the transposed copy (t_row_ptr) and, per 32-row block
 // and column, the block's offset in the column's run (in `scratch`, nb x cols
-// int32, followed by the column totals), from a keep bitmask (cols % 32 == 0)
-// or, with have_counts, from the per-block column counts already in scratch.
-int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch, size_t scratch_bytes,
-                           cudaStream_t s, bool have_counts) {
+// int32, followed by the column totals), from a keep bitmask (cols % 32 == 0).
+static int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch, size_t scratch_bytes,
+                                  cudaStream_t s) {
     const int32_t rows = w->rows, cols = w->cols;
     const int32_t wpr = cols / 32;
     CSRT_ARG(scratch_bytes >= transpose_scratch_bytes(rows, cols), "scratch too small for the transposed copy");
@@ -1869,13 +1795,10 @@ int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch,
     int32_t *coltot = cnt + (int64_t)nb * cols;
     const int64_t warps = (int64_t)nb * wpr;
     const unsigned grid = (unsigned)ceil_div<int64_t>(warps * 32, 256);
-    if (!have_counts) {   // else the caller's kernel wrote them
-        launch_pdl(trb_count_kernel, dim3(grid), dim3(256), 0, s, keepbits, rows, wpr, cols, cnt);
-        count_launch(1);
-    }
+    launch_pdl(trb_count_kernel, dim3(grid), dim3(256), 0, s, keepbits, rows, wpr, cols, cnt);
     launch_pdl(tr_colscan_kernel, dim3(ceil_div(cols, 32)), dim3(256), 0, s, cnt, nb, cols, coltot);
     launch_pdl(scan_single_block_kernel, dim3(1), dim3(1024), 0, s, coltot, cols, w->t_row_ptr);
-    count_launch(2);
+    count_launch(3);
     return check_launch("transposed-copy count kernels");
 }
 
@@ -1883,7 +1806,7 @@ int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch,
 // `scratch` holds the per-block column counts and the column totals.
 int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t *wordpos, void *scratch,
                             size_t scratch_bytes, cudaStream_t s) {
-    int rc = transpose_bits_prepare(w, keepbits, scratch, scratch_bytes, s, false);
+    int rc = transpose_bits_prepare(w, keepbits, scratch, scratch_bytes, s);
     if (rc) return rc;
     const int32_t rows = w->rows, cols = w->cols;
     const int32_t wpr = cols / 32;

@@ -22,8 +22,9 @@
 //     segments and the new row pointers (clamped to the capacity in w_out).
 //  4. With a transposed copy wanted: the count pass also writes its column
 //     counts per 32-row block (a 32 x 32 bit transpose of the rows' keep
-//     words); their scan down each column and the column pointers follow
-//     (compact.cu, transpose_bits_prepare).
+//     words); their scan down each column and the column pointers are taken
+//     in the same two launches as step 3 (fp_rows_cols_scan_kernel,
+//     fp_two_scans_kernel).
 //  5. gemm_prox_tc_kernel<write>: the same GEMM again; the epilogue recomputes
 //     z, passes each 32 x 32 block through shared memory and writes the kept
 //     entries of one row at a time at their final positions (a coalesced run
@@ -39,8 +40,6 @@ namespace csrt {
 
 int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t *wordpos, void *scratch,
                             size_t scratch_bytes, cudaStream_t s);
-int transpose_bits_prepare(csrt_csr *w, const uint32_t *keepbits, void *scratch, size_t scratch_bytes,
-                           cudaStream_t s, bool have_counts);
 size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
 
 // Segments (the unit of the per-row offsets) are 64 columns, two 32-column
@@ -737,12 +736,11 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
     }
 }
 
-// 3. Per row: exclusive offsets of the segments (in place) and the row total.
-__global__ void __launch_bounds__(256) fp_rowscan_kernel(int32_t *__restrict__ counts, int32_t m, int32_t nt,
-                                                         int32_t *__restrict__ rowtot) {
-    pdl_enter();
+// 3. Per row: exclusive offsets of the segments (in place) and the row total
+// (warp r of the grid takes row r).
+__device__ __forceinline__ void fp_rowscan_row(int32_t *__restrict__ counts, int32_t m, int32_t nt,
+                                               int32_t *__restrict__ rowtot, int64_t r) {
     const int lane = threadIdx.x & 31;
-    const int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     if (r >= m) return;
     int32_t *c = counts + r * nt;
     int32_t run = 0;
@@ -759,6 +757,40 @@ __global__ void __launch_bounds__(256) fp_rowscan_kernel(int32_t *__restrict__ c
         run += __shfl_sync(0xffffffffu, incl, 31);
     }
     if (lane == 0) rowtot[r] = run;
+}
+
+__global__ void __launch_bounds__(256) fp_rowscan_kernel(int32_t *__restrict__ counts, int32_t m, int32_t nt,
+                                                         int32_t *__restrict__ rowtot) {
+    pdl_enter();
+    fp_rowscan_row(counts, m, nt, rowtot, ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+}
+
+// With a transposed copy the two scans between the passes share launches:
+// blocks [0, rb) scan the rows' segment counts, the others the transposed
+// copy's column counts down each column; then block 0 of the second kernel
+// scans the row totals (the row pointers), block 1 the column totals (the
+// transposed copy's column pointers).
+__global__ void __launch_bounds__(256) fp_rows_cols_scan_kernel(int32_t *__restrict__ counts, int32_t m, int32_t nt,
+                                                                int32_t *__restrict__ rowtot, int32_t rb,
+                                                                int32_t *__restrict__ cnt, int32_t nb, int32_t cols,
+                                                                int32_t *__restrict__ coltot) {
+    pdl_enter();
+    if ((int)blockIdx.x < rb)   // block-uniform
+        fp_rowscan_row(counts, m, nt, rowtot, ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    else
+        colscan_block(cnt, nb, cols, coltot, (int)blockIdx.x - rb);
+}
+
+__global__ void __launch_bounds__(1024) fp_two_scans_kernel(const int32_t *__restrict__ rowtot, int32_t m,
+                                                            int32_t *__restrict__ rawptr,
+                                                            int32_t *__restrict__ row_ptr_out, int64_t capacity,
+                                                            WsHeader *hdr, const int32_t *__restrict__ coltot,
+                                                            int32_t cols, int32_t *__restrict__ t_row_ptr) {
+    pdl_enter();
+    if (blockIdx.x == 0)
+        scan_block_1024(rowtot, m, rawptr, row_ptr_out, capacity, hdr);
+    else
+        scan_block_1024(coltot, cols, t_row_ptr, nullptr, 0, nullptr);
 }
 
 int scan_exclusive_i32_clamped(const int32_t *in, int32_t n, int32_t *out, int32_t *out_clamped, int64_t capacity,
@@ -855,18 +887,27 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
     else
         launch_pdl(gemm_prox_tc_kernel<false, false>, dim3(grid), dim3(fp_threads<false>()), fp_smem_bytes<false>(), s,
                    ma, mb, a, ta, tiles_n, tiles);
-    launch_pdl(fp_rowscan_kernel, dim3((unsigned)ceil_div<int64_t>((int64_t)m * 32, 256)), dim3(256), 0, s, counts, m,
-               L.nt, rowtot);
-    count_launch(3);
-    // new row pointers: exclusive scan of the row totals (int32: nnz <= M*K < 2^31), unclamped for the write
-    // pass and clamped to the capacity in w_out (overflow reported)
-    int rc = scan_exclusive_i32_clamped(rowtot, m, rawptr, w_out->row_ptr, w_out->capacity, ws, s);
-    if (rc) return rc;
-    if (want_t) {
-        // the transposed copy's column pointers and per-block offsets from the count pass's column counts;
-        // the write pass writes its arrays
-        rc = transpose_bits_prepare(w_out, kbits, base + L.off_tr, L.total - L.off_tr, s, true);
+    count_launch(2);
+    const unsigned rb = (unsigned)ceil_div<int64_t>((int64_t)m * 32, 256);
+    int rc = 0;
+    if (!want_t) {
+        launch_pdl(fp_rowscan_kernel, dim3(rb), dim3(256), 0, s, counts, m, L.nt, rowtot);
+        count_launch(1);
+        // new row pointers: exclusive scan of the row totals (int32: nnz <= M*K < 2^31), unclamped for the
+        // write pass and clamped to the capacity in w_out (overflow reported)
+        rc = scan_exclusive_i32_clamped(rowtot, m, rawptr, w_out->row_ptr, w_out->capacity, ws, s);
         if (rc) return rc;
+    } else {
+        // the same, paired with the transposed copy's scans of the count pass's column counts (its per-block
+        // offsets down each column and its column pointers); the write pass writes its arrays
+        int32_t *tcnt = reinterpret_cast<int32_t *>(base + L.off_tr);
+        const int32_t nb = (int32_t)ceil_div<int64_t>(m, 32);
+        int32_t *coltot = tcnt + (int64_t)nb * k;
+        launch_pdl(fp_rows_cols_scan_kernel, dim3(rb + (unsigned)ceil_div(k, 32)), dim3(256), 0, s, counts, m, L.nt,
+                   rowtot, (int32_t)rb, tcnt, nb, k, coltot);
+        launch_pdl(fp_two_scans_kernel, dim3(2), dim3(1024), 0, s, rowtot, m, rawptr, w_out->row_ptr,
+                   w_out->capacity, static_cast<WsHeader *>(ws), coltot, k, w_out->t_row_ptr);
+        count_launch(2);
         ta.t_rp = w_out->t_row_ptr;
         ta.t_off = reinterpret_cast<const int32_t *>(base + L.off_tr);
         ta.t_col = w_out->t_col_idx;
