@@ -386,12 +386,13 @@ def op_bytes(name, info):
 # Kernels of one weight_grad_prox_update call: it starts with fp_oldbits_kernel
 # and runs on through these (the transposed copy included when built).
 FUSED_OP_KERNELS = ("fp_oldbits_kernel", "gemm_prox_tc_kernel", "fp_rowscan_kernel", "scan_clamped_kernel",
-                    "scan_single_block_kernel", "fp_finish_kernel", "trb_count_kernel", "tr_colscan_kernel",
-                    "trb_write_kernel")
+                    "fp_rows_cols_scan_kernel", "fp_two_scans_kernel", "scan_single_block_kernel",
+                    "trb_count_kernel", "tr_colscan_kernel", "trb_write_kernel")
 FUSED_OP_SOURCES = ["fused_prox.cu", "compact.cu", "tc_common.cuh", "common.cuh"]
 # the ncu command whose CSV record_traffic reads: the ops' kernels only
 TRAFFIC_NCU = ("ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum --clock-control none "
-               "-k regex:'fp_oldbits|gemm_prox|fp_rowscan|scan_clamped|scan_single|trb_|tr_colscan|spmm_merge' "
+               "-k regex:'fp_oldbits|gemm_prox|fp_rowscan|fp_rows_cols|fp_two_scans|scan_clamped|scan_single|trb_|"
+               "tr_colscan|spmm_merge' "
                "-c 60 --csv --log-file bench_dram.csv")
 
 
