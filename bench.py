@@ -471,7 +471,8 @@ def record_traffic(csv_path: str, out_path: str) -> dict:
 # ---------------------------------------------------------------------------
 
 KERNEL_OF_OP = {"spmm_fwd": "spmm_group_kernel", "spmm_bwd_t": "spmm_group_kernel", "sddmm": "sddmm_kernel",
-                "prox (lambda=1e-4)": "prox_rows_kernel", "prox (lambda*)": "prox_rows_kernel"}
+                "prox (lambda=1e-4)": "prox_count_kernel + prox_place_kernel",
+                "prox (lambda*)": "prox_count_kernel + prox_place_kernel"}
 
 
 def measure_kernels(hbm_peak: float, reps: int = 20):
@@ -708,7 +709,7 @@ def main():
         same_kernels = dom["name"] in ("spmm_fwd", "spmm_bwd_t", "spmm_fwd_bias_act", "spmm_bwd_t_relu") or (
             args.precision == "tf32" and args.prox_path == "fused" and args.optimizer == "sgd")
         if args.precision == "fp32" and dom["name"] == "weight_grad_prox_update":
-            kernel = "gemm_nt_f32_kernel + prox_rows_kernel (the op's unfused route at FP32)"
+            kernel = "gemm_nt_f32_kernel + prox_count_kernel + prox_place_kernel (the op's unfused route at FP32)"
         roof.update({"traffic": recorded_traffic(dom["label"]) if same_kernels else None, "kernel": kernel,
                      "op": dom["label"],
                      "algorithmic_bytes": int(bytes_) if bytes_ else None, "launch_ms": round(dom["ms"], 4)})
@@ -786,7 +787,7 @@ def profile_ops(net, C, torch, eta, lam, flush):
     kernel_of = {"spmm_fwd": "spmm_merge_kernel", "spmm_bwd_t": "spmm_merge_kernel",
                  "spmm_fwd_bias_act": "spmm_merge_kernel", "spmm_bwd_t_relu": "spmm_merge_kernel",
                  "weight_grad_dense": "gemm_tf32_tc_persistent_kernel", "weight_grad_sddmm": "sddmm_kernel",
-                 "prox_update_compact": "prox_rows_kernel", "prox_rmsprop_update_compact": "prox_rows_kernel",
+                 "prox_update_compact": "prox_count_kernel", "prox_rmsprop_update_compact": "prox_rows_kernel",
                  "prox_adam_update_compact": "prox_rows_kernel", "weight_grad_prox_update": "gemm_prox_tc_kernel",
                  "debias_update": "debias_kernel"}
     layer_of = {}
