@@ -1060,9 +1060,12 @@ __device__ __forceinline__ float prox_cp_value(float tv, bool stored, float eta,
 // pattern an entry is kept iff |fl(eta*G)| > thr, on it the fold's decision
 // counts, and, eta being positive, fl(eta*v) is NaN exactly where v (G, or z
 // at a stored position) is. Lanes 8q .. 8q+7 of a group hold its word q,
-// assembled by three shuffles. The keep words collect in shared memory and
-// leave afterwards as coalesced stores, with the kept count of every row
-// summed from them, and the tile's count is published at once. A tile keeping
+// assembled by three shuffles (measured against a ballot per word, lane =
+// column: 76 vs 96 us for the 4096 x 9216 prox at the density-preserving
+// lambda). The keep words collect in shared memory and, when the transposed
+// copy wants them, leave afterwards as coalesced stores; the kept count of
+// every row is summed from them (a one-row tile's is the tile's), and the
+// tile's count is published at once. A tile keeping
 // at most `stash` entries then writes them in CSR order to its stash (each
 // warp its segment's, lane = entry, the entry's word found by a search over
 // the words' exclusive counts), and is done without waiting on any other
@@ -1150,19 +1153,26 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_count_kernel(CompactArgs a,
         if (w < warp) wbase += t;
         tile_count += t;
     }
-    // keep words out (the tile's rows are contiguous in keepbits); rows' counts, a warp per row
-    uint32_t *kb_tile = keepbits + (int64_t)r0 * wpr;
-    for (int i = tid; i < nwt; i += kCThreads) kb_tile[i] = kwords[i];
-    for (int r = warp; r < nrows; r += kCThreads / 32) {
-        int32_t c = 0;
-        for (int i = lane; i < wpr; i += 32) c += __popc(kwords[r * wpr + i]);
+    // keep words out for the transposed copy (the tile's rows are contiguous
+    // in keepbits); rows' counts, a warp per row (a one-row tile's is the tile's)
+    if (kBits) {
+        uint32_t *kb_tile = keepbits + (int64_t)r0 * wpr;
+        for (int i = tid; i < nwt; i += kCThreads) kb_tile[i] = kwords[i];
+    }
+    if (nrows == 1) {
+        if (tid == 0) rowcnt[r0] = (int32_t)tile_count;
+    } else {
+        for (int r = warp; r < nrows; r += kCThreads / 32) {
+            int32_t c = 0;
+            for (int i = lane; i < wpr; i += 32) c += __popc(kwords[r * wpr + i]);
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) c += __shfl_xor_sync(0xffffffffu, c, off);
-        if (lane == 0) rowcnt[r0 + r] = c;
+            for (int off = 16; off > 0; off >>= 1) c += __shfl_xor_sync(0xffffffffu, c, off);
+            if (lane == 0) rowcnt[r0 + r] = c;
+        }
     }
     const bool stashed = tile_count <= (uint32_t)stash;
     if (tid == 0) {
-        tilecnt[tile] = stashed ? (int32_t)tile_count : -1;
+        tilecnt[tile] = stashed ? (int32_t)tile_count : -1 - (int32_t)tile_count;
         if (stashed)   // published without waiting (tile 0's count is its inclusive prefix)
             st_release_u64(a.status + tile, (tile == 0 ? kFlagInc : kFlagAgg) | tile_count);
     }
@@ -1191,7 +1201,7 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_count_kernel(CompactArgs a,
                 if (e < total) {
                     const int wi = i0 + src;
                     const int bit = nth_set_bit(word, k);
-                    const int row = wi / wpr;
+                    const int row = nrows == 1 ? 0 : wi / wpr;
                     sc[pos + e] = 32 * wi + bit - row * K;
                     sv[pos + e] = prox_cp_value(tile_v[32 * wi + bit], (onbits[wi] >> bit) & 1u, eta, thr);
                 }
@@ -1230,57 +1240,148 @@ __global__ void __launch_bounds__(kCThreads, 6) prox_count_kernel(CompactArgs a,
     prox_flags(a, nonfinite, s_fail);
 }
 
-// Place kernel: a stashed tile's run is copied to its final position (from
-// the scanned row counts, not clamped), and with kBits the word positions of
-// the transposed copy are written from the keep words. Tiles the count kernel
-// wrote itself (tilecnt -1) are skipped.
-template <bool kBits>
-__global__ void __launch_bounds__(kCThreads) prox_place_kernel(CompactArgs a, int32_t rows_per_tile,
-                                                               const uint32_t *__restrict__ keepbits,
-                                                               int32_t *__restrict__ wordpos, int32_t wpr,
-                                                               const int32_t *__restrict__ raw,
-                                                               const int32_t *__restrict__ tilecnt,
-                                                               const int32_t *__restrict__ st_col,
-                                                               const float *__restrict__ st_val, int32_t stash) {
+// Place kernel: a stashed tile's run is copied to its final position, and
+// with kBits the word positions of the transposed copy are written from the
+// keep words. Tiles the count kernel wrote itself (tilecnt -1 - count) are
+// skipped. A block takes kPlaceTiles consecutive tiles and loads, for each,
+// its count and the first two entries per thread of its stash together (a
+// stash holds at least 512 entries, so these reads stay inside it whatever
+// the count): one round of loads for the usual stash. With kPrefix the block
+// also finds where its rows start, the sum of the counts of every earlier
+// tile (a reduction; the launch takes this form up to kPlaceMaxTiles tiles),
+// and writes their row pointers (clamped to the capacity; the last block the
+// total and the overflow report), which otherwise the scan before it wrote,
+// with the unclamped starts in raw.
+constexpr int kPlaceTiles = 4;
+constexpr int64_t kPlaceMaxTiles = 4096;
+constexpr int kPlaceMaxRows = kPlaceTiles * (kRowBudget / 32);   // rows of a block (K >= 32)
+template <bool kBits, bool kPrefix>
+__global__ void __launch_bounds__(kCThreads, 4) prox_place_kernel(CompactArgs a, int32_t rows_per_tile,
+                                                                  const uint32_t *__restrict__ keepbits,
+                                                                  int32_t *__restrict__ wordpos, int32_t wpr,
+                                                                  const int32_t *__restrict__ rowcnt,
+                                                                  const int32_t *__restrict__ raw,
+                                                                  const int32_t *__restrict__ tilecnt,
+                                                                  const int32_t *__restrict__ st_col,
+                                                                  const float *__restrict__ st_val, int32_t stash) {
     pdl_enter();
+    __shared__ int32_t s_pre[kPrefix ? kPlaceMaxRows + 1 : 1];
+    __shared__ int32_t s_red[kCThreads / 32], s_part[kCThreads / 32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int64_t tile = blockIdx.x;
-    if (tile >= a.num_tiles) return;
-    const int r0 = (int)(tile * rows_per_tile);
-    const int nrows = imin(rows_per_tile, a.rows - r0);
-    const int32_t *sc = st_col + tile * (int64_t)stash;
-    const float *sv = st_val + tile * (int64_t)stash;
-    // the count, the position and the stash's first two entries per thread load together (a stash holds
-    // at least 512 entries, so these reads stay inside it whatever the count)
-    const int32_t count = __ldg(tilecnt + tile);
-    const uint32_t base = (uint32_t)__ldg(raw + r0);
-    const int32_t c0 = __ldg(sc + tid), c1 = __ldg(sc + tid + kCThreads);
-    const float v0 = __ldg(sv + tid), v1 = __ldg(sv + tid + kCThreads);
-    if (count < 0) return;
-    const uint32_t cap = (uint32_t)imin<int64_t>(a.capacity, 0x7fffffff);
-    for (int i = tid; i < count; i += kCThreads) {
-        const uint32_t p = base + (uint32_t)i;
-        const int32_t c = i < kCThreads ? c0 : i < 2 * kCThreads ? c1 : __ldg(sc + i);
-        const float v = i < kCThreads ? v0 : i < 2 * kCThreads ? v1 : __ldg(sv + i);
-        if (p < cap) {
-            a.out_col[p] = c;
-            a.out_val[p] = v;
+    const int64_t tile0 = (int64_t)blockIdx.x * kPlaceTiles;
+    int32_t count[kPlaceTiles], c0[kPlaceTiles], c1[kPlaceTiles];
+    float v0[kPlaceTiles], v1[kPlaceTiles];
+#pragma unroll
+    for (int j = 0; j < kPlaceTiles; ++j) {
+        const int64_t tile = tile0 + j;
+        count[j] = -1;
+        c0[j] = c1[j] = 0;
+        v0[j] = v1[j] = 0.f;
+        if (tile < a.num_tiles) {
+            const int32_t *sc = st_col + tile * (int64_t)stash;
+            const float *sv = st_val + tile * (int64_t)stash;
+            count[j] = __ldg(tilecnt + tile);
+            c0[j] = __ldg(sc + tid);
+            c1[j] = __ldg(sc + tid + kCThreads);
+            v0[j] = __ldg(sv + tid);
+            v1[j] = __ldg(sv + tid + kCThreads);
         }
     }
-    if (kBits) {   // word positions: a warp per row, a scan of the words' kept counts
-        for (int r = warp; r < nrows; r += kCThreads / 32) {
-            const int64_t wi0 = (int64_t)(r0 + r) * wpr;
-            int32_t run = __ldg(raw + r0 + r);
+    const int64_t r_begin = tile0 * rows_per_tile;
+    const int nr = (int)imin<int64_t>((int64_t)kPlaceTiles * rows_per_tile, a.rows - r_begin);
+    const uint32_t cap = (uint32_t)imin<int64_t>(a.capacity, 0x7fffffff);
+    int32_t block_base = 0;
+    if (kPrefix) {
+        // entries kept before the block: the counts of tiles 0 .. tile0-1, four loads in flight per thread
+        int32_t part = 0;
+        for (int64_t t0 = 0; t0 < tile0; t0 += 4 * kCThreads) {
+            int32_t c[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int64_t t = t0 + u * kCThreads + tid;
+                c[u] = t < tile0 ? __ldg(tilecnt + t) : 0;
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) part += c[u] >= 0 ? c[u] : -1 - c[u];
+        }
+        // the block's rows, four per thread: exclusive counts within the block
+        int32_t rc[4], own = 0;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int i = 4 * tid + u;
+            rc[u] = i < nr ? __ldg(rowcnt + r_begin + i) : 0;
+            own += rc[u];
+        }
+        int32_t incl = own;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int32_t y = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += y;
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
+        if (lane == 31) s_red[warp] = incl;
+        if (lane == 0) s_part[warp] = part;
+        __syncthreads();
+        int32_t wpre = 0;
+#pragma unroll
+        for (int w = 0; w < kCThreads / 32; ++w) {
+            if (w < warp) wpre += s_red[w];
+            block_base += s_part[w];
+        }
+        int32_t run = block_base + wpre + incl - own;   // the start of this thread's first row
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int i = 4 * tid + u;
+            if (i < nr) {
+                s_pre[i] = run;
+                a.out_row_ptr[r_begin + i] = (int32_t)imin<uint32_t>((uint32_t)run, cap);
+            }
+            run += rc[u];
+        }
+        if (r_begin + nr == a.rows && tid == kCThreads - 1) {   // the last block: the total
+            a.out_row_ptr[a.rows] = (int32_t)imin<uint32_t>((uint32_t)run, cap);
+            if ((int64_t)run > a.capacity) {
+                dev_flag(a.hdr, CSRT_DEV_CAPACITY);
+                atomicMax(&a.hdr->required, (unsigned long long)run);
+            }
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int j = 0; j < kPlaceTiles; ++j) {
+        const int64_t tile = tile0 + j;
+        if (count[j] <= 0) continue;
+        const int32_t *sc = st_col + tile * (int64_t)stash;
+        const float *sv = st_val + tile * (int64_t)stash;
+        const uint32_t base = kPrefix ? (uint32_t)s_pre[j * rows_per_tile] : (uint32_t)__ldg(raw + tile * rows_per_tile);
+        for (int i = tid; i < count[j]; i += kCThreads) {
+            const uint32_t p = base + (uint32_t)i;
+            const int32_t c = i < kCThreads ? c0[j] : i < 2 * kCThreads ? c1[j] : __ldg(sc + i);
+            const float v = i < kCThreads ? v0[j] : i < 2 * kCThreads ? v1[j] : __ldg(sv + i);
+            if (p < cap) {
+                a.out_col[p] = c;
+                a.out_val[p] = v;
+            }
+        }
+    }
+    if (kBits) {   // word positions: a warp per row of the stashed tiles, a scan of the words' kept counts
+        for (int i = warp; i < nr; i += kCThreads / 32) {
+            const int64_t tile = tile0 + i / rows_per_tile;
+            if (__ldg(tilecnt + tile) < 0) continue;
+            const int64_t r = r_begin + i;
+            const int64_t wi0 = r * wpr;
+            int32_t run = kPrefix ? s_pre[i] : __ldg(raw + r);
             for (int i0 = 0; i0 < wpr; i0 += 32) {
-                const int i = i0 + lane;
-                const int32_t c = i < wpr ? __popc(__ldg(keepbits + wi0 + i)) : 0;
+                const int w = i0 + lane;
+                const int32_t c = w < wpr ? __popc(__ldg(keepbits + wi0 + w)) : 0;
                 int32_t incl = c;
 #pragma unroll
                 for (int off = 1; off < 32; off <<= 1) {
                     const int32_t t = __shfl_up_sync(0xffffffffu, incl, off);
                     if (lane >= off) incl += t;
                 }
-                if (i < wpr) wordpos[wi0 + i] = run + incl - c;
+                if (w < wpr) wordpos[wi0 + w] = run + incl - c;
                 run += __shfl_sync(0xffffffffu, incl, 31);
             }
         }
@@ -1406,8 +1507,7 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
             const PlaceLayout P = place_layout(rows, cols);
             if (a.opt == kOptSgd && eta > 0.f && P.total > 0 && P.rows_per_tile == rows_per_tile &&
                 ws_bytes >= kWsReservedBytes + pre + P.total) {
-                // count, scan of the row counts (the new row pointers, clamped to the capacity, overflow
-                // reported), place
+                // count, the new row pointers (clamped to the capacity, overflow reported), place
                 char *pb = base + pre;
                 int32_t *rowcnt = reinterpret_cast<int32_t *>(pb + P.off_rowcnt);
                 int32_t *raw = reinterpret_cast<int32_t *>(pb + P.off_raw);
@@ -1425,14 +1525,28 @@ static int compact_launch(bool prox, const float *src, int32_t rows, int32_t col
                 count_launch();
                 int rc = check_launch("prox count kernel");
                 if (rc) return rc;
-                rc = scan_exclusive_i32_clamped(rowcnt, rows, raw, out->row_ptr, out->capacity, ws, s);
-                if (rc) return rc;
-                if (words)
-                    launch_pdl(prox_place_kernel<true>, dim3((unsigned)tiles), dim3(kCThreads), 0, s, a,
-                               rows_per_tile, keepbits, wordpos, cols / 32, raw, tilecnt, st_col, st_val, P.stash);
+                // the row pointers: in the place kernel (a reduction over the tiles' counts) up to
+                // kPlaceMaxTiles tiles, else a scan of the row counts first
+                const bool prefix = tiles <= kPlaceMaxTiles;
+                if (!prefix) {
+                    rc = scan_exclusive_i32_clamped(rowcnt, rows, raw, out->row_ptr, out->capacity, ws, s);
+                    if (rc) return rc;
+                }
+                const dim3 pgrid((unsigned)ceil_div<int64_t>(tiles, kPlaceTiles));
+                const uint32_t *kb = words ? keepbits : nullptr;
+                int32_t *wp = words ? wordpos : nullptr;
+                if (words && prefix)
+                    launch_pdl(prox_place_kernel<true, true>, pgrid, dim3(kCThreads), 0, s, a, rows_per_tile, kb, wp,
+                               cols / 32, rowcnt, raw, tilecnt, st_col, st_val, P.stash);
+                else if (words)
+                    launch_pdl(prox_place_kernel<true, false>, pgrid, dim3(kCThreads), 0, s, a, rows_per_tile, kb, wp,
+                               cols / 32, rowcnt, raw, tilecnt, st_col, st_val, P.stash);
+                else if (prefix)
+                    launch_pdl(prox_place_kernel<false, true>, pgrid, dim3(kCThreads), 0, s, a, rows_per_tile, kb, wp,
+                               cols / 32, rowcnt, raw, tilecnt, st_col, st_val, P.stash);
                 else
-                    launch_pdl(prox_place_kernel<false>, dim3((unsigned)tiles), dim3(kCThreads), 0, s, a,
-                               rows_per_tile, keepbits, nullptr, cols / 32, raw, tilecnt, st_col, st_val, P.stash);
+                    launch_pdl(prox_place_kernel<false, false>, pgrid, dim3(kCThreads), 0, s, a, rows_per_tile, kb,
+                               wp, cols / 32, rowcnt, raw, tilecnt, st_col, st_val, P.stash);
                 if (bits_done) *bits_done = words;
                 count_launch();
                 return check_launch("prox place kernel");

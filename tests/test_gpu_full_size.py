@@ -170,6 +170,34 @@ def test_prox_on_the_sweep_layer(C, density, zipf):
             torch.cuda.empty_cache()
 
 
+def test_prox_beyond_the_place_kernels_prefix(C):
+    """prox_update_compact on a layer of 4100 x 8192 (one row per tile, 4100
+    tiles: more than the place kernel sums counts over itself, so the row
+    pointers come from a scan of the row counts), bit for bit at lambda =
+    1e-4 and at lambda*, with and without the transposed copy."""
+    from paper_1905_07931_gb300 import synth
+    m, k, density = 4100, 8192, 0.05
+    rng = synth.rng_for(7)
+    w = synth.masked_weights(rng, m, k, density, zipf=False)
+    g = synth.std_normal(rng, m, k)
+    eta, lam = synth.ETA, synth.LAMBDA
+    ref_in = O.csr_from_dense(w)
+    ws = C.Workspace(m, k, 1)
+    W = C.CSR(m, k, capacity=max(ref_in.nnz, 1), transposed=False)
+    C.csr_from_dense(_dev(w), W, ws)
+    gd = _dev(g)
+    for lam_v in (lam, _lambda_star(w, g, eta, density)):
+        ref = O.prox_update_compact(ref_in, g, eta, lam_v)
+        t_ref = O.csr_transpose(ref)
+        for transposed in (True, False):
+            out = C.CSR(m, k, transposed=transposed)
+            C.prox_update_compact(W, gd, eta, lam_v, out, ws)
+            assert ws.status()[0] == 0
+            _assert_same_csr(out, ref, t_ref, transposed)
+            del out
+            torch.cuda.empty_cache()
+
+
 # ---------------------------------------------------------------------------
 # The classifier-head step (9216-4096-4096-1000, batch 256): the fused
 # gradient + prox op against the unfused calls at the bench's own shapes

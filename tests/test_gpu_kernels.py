@@ -404,6 +404,51 @@ def test_prox_bit_exact(C, m, k, density, gscale, eta, lam):
     assert ws.status()[0] == 0
 
 
+def _largest_below(eta, thr):
+    """The largest float32 x >= 0 with fl(eta*x) <= thr (None if none), by
+    walking float32 bit patterns from fl(thr/eta): the decision boundary of
+    |fl(eta*G)| > thr in G, found with numpy's float32 products."""
+    eta, thr = np.float32(eta), np.float32(thr)
+    ok = lambda u: np.float32(eta * np.array([u], np.uint32).view(np.float32)[0]) <= thr
+    if not ok(0):
+        return None
+    u = int(min(np.array([thr / eta], np.float32).view(np.uint32)[0], 0x7F800000))
+    while u > 0 and not ok(u):
+        u -= 1
+    while u < 0x7F800000 and ok(u + 1):
+        u += 1
+    return np.array([u], np.uint32).view(np.float32)[0]
+
+
+@pytest.mark.parametrize("eta,lam", [(0.01, 1e-4), (0.013, 7.7e-5), (1e-3, 1e-38), (3.0, 1e-7), (0.01, 0.0)])
+@pytest.mark.parametrize("m,k", [(64, 256), (3, 9216)])
+def test_prox_keep_boundary(C, eta, lam, m, k):
+    """Gradients on both sides of the keep boundary: off the pattern an entry
+    is kept iff |fl(eta*G)| > fl(eta*lambda) (Section 2.2's soft threshold
+    applied to 0 - eta*G). G takes the largest magnitude that is dropped, the
+    next float up, their negatives and a few patterns around them, on stored
+    and unstored positions; bit-exact against the oracle."""
+    thr = np.float32(np.float32(eta) * np.float32(lam))
+    b = _largest_below(eta, thr)
+    assert b is not None and np.float32(np.float32(eta) * np.nextafter(b, np.float32(np.inf))) > thr
+    near = np.array([b], np.float32).view(np.uint32)[0].astype(np.int64) + np.arange(-3, 4)
+    near = near[(near >= 0) & (near < 0x7F800000)].astype(np.uint32).view(np.float32)
+    rng = np.random.default_rng(int(eta * 1e4) + m)
+    vals = np.concatenate([near, -near])
+    g = rng.choice(vals, size=(m, k)).astype(F32)
+    g[:, ::7] = (rng.standard_normal((m, (k + 6) // 7)) * 4 * max(b, 1e-30)).astype(F32)
+    a = _sparse(rng, m, k, 0.1)
+    ws = _ws(C, m, k, 1)
+    w = _gpu_csr(C, a, ws)
+    out = C.CSR(m, k)
+    C.prox_update_compact(w, _dev(g), eta, lam, out, ws)
+    ref = O.prox_update_compact(O.csr_from_dense(a), g, eta, lam)
+    _check_csr_equal(out, ref)
+    kept = int(ref.row_ptr[-1])
+    assert 0 < kept < m * k   # both decisions occur
+    assert ws.status()[0] == 0
+
+
 @pytest.mark.parametrize("eta,lam", [(0.0, 1e-4), (0.01, 0.0), (1e-3, 1e-38), (0.5, 1e30), (1e20, 1e20),
                                      (3.0, 1e-7)])
 def test_prox_threshold_edges(C, eta, lam):
