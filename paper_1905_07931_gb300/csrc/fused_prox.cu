@@ -70,7 +70,11 @@ constexpr int kFpMaxK = 16384;
 // of a word handled together in the write pass's column domain.
 template <bool kWrite> struct FpShape;
 template <> struct FpShape<false> {
-    static constexpr int kEpi = CSRT_FP_COUNT_EPI, kStages = CSRT_FP_COUNT_EPI > 8 ? 3 : 4, kPre = 8, kGroup = 8;
+    // kPre 4 rather than 8: 15% fewer instructions, the count pass of the
+    // 4096 x 9216 layer 45.4 -> 44.4 us (at 5% density 2% of the rows' words
+    // hold more than four stored weights, half the warps' words one such row;
+    // the loop after the prefetched ones takes them)
+    static constexpr int kEpi = CSRT_FP_COUNT_EPI, kStages = CSRT_FP_COUNT_EPI > 8 ? 3 : 4, kPre = 4, kGroup = 8;
 };
 #ifndef CSRT_FP_WRITE_STAGE_WORDS
 #define CSRT_FP_WRITE_STAGE_WORDS 1
