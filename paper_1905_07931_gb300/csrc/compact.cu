@@ -1838,15 +1838,23 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
         // a dense block: walk its rows (lane = column) and then its columns
         // (lane = row); a step per row or column costs less than the search
         // of the enumeration once most lanes hold an entry
+        // The 32 rows' values are loaded first, all in flight at once, then
+        // staged (loading and staging row by row waited once per row).
         const unsigned lt = (1u << lane) - 1u;
-        int64_t pc = cb_mine;
+        float v[32];
+#pragma unroll
         for (int r = 0; r < 32; ++r) {
             const uint32_t rw = __shfl_sync(0xffffffffu, rw_mine, r);
-            if (rw == 0u) continue;
-            const int32_t rp = __shfl_sync(0xffffffffu, rp_mine, r);
+            const int64_t pr = (int64_t)__shfl_sync(0xffffffffu, rp_mine, r) + __popc(rw & lt);
+            v[r] = ((rw >> lane) & 1u) && pr < capacity ? __ldg(val + pr) : 0.f;
+        }
+        int64_t pc = cb_mine;
+#pragma unroll
+        for (int r = 0; r < 32; ++r) {
+            const uint32_t rw = __shfl_sync(0xffffffffu, rw_mine, r);
+            const int64_t pr = (int64_t)__shfl_sync(0xffffffffu, rp_mine, r) + __popc(rw & lt);
             if ((rw >> lane) & 1u) {
-                const int64_t pr = (int64_t)rp + __popc(rw & lt);
-                tl[r * 32 + (lane ^ r)] = pr < capacity ? __ldg(val + pr) : 0.f;
+                tl[r * 32 + (lane ^ r)] = v[r];
                 if (pc < capacity && pr < capacity) t_pos[pr] = (int32_t)pc;
                 ++pc;
             }
@@ -1866,20 +1874,34 @@ __global__ void __launch_bounds__(256) trb_write_kernel(const uint32_t *__restri
         }
         return;
     }
-    for (int e0 = 0; e0 < total; e0 += 32) {   // row-major (CSR) order
-        const int e = e0 + lane;
-        const int r = warp_last_le(rpre, e);
-        const uint32_t rw = __shfl_sync(0xffffffffu, rw_mine, r);
-        const int k = e - __shfl_sync(0xffffffffu, rpre, r);
-        const int32_t rp = __shfl_sync(0xffffffffu, rp_mine, r);
-        const int j = nth_set_bit(rw, k);
-        const uint32_t cm = __shfl_sync(0xffffffffu, cm_mine, j);
-        const int64_t cb = __shfl_sync(0xffffffffu, cb_mine, j);
-        if (e < total) {
-            const int64_t pr = (int64_t)rp + k;
-            const int64_t pc = cb + __popc(cm & ((1u << r) - 1u));
-            tl[r * 32 + (j ^ r)] = pr < capacity ? __ldg(val + pr) : 0.f;
-            if (pc < capacity && pr < capacity) t_pos[pr] = (int32_t)pc;
+    constexpr int kRounds = 4;   // 32-entry rounds whose value loads are in flight together
+    for (int e00 = 0; e00 < total; e00 += 32 * kRounds) {   // row-major (CSR) order
+        float v[kRounds];
+        int64_t pr[kRounds], pc[kRounds];
+        int at[kRounds];
+#pragma unroll
+        for (int q = 0; q < kRounds; ++q) {
+            at[q] = -1;
+            if (e00 + 32 * q >= total) continue;   // the same for every lane
+            const int e = e00 + 32 * q + lane;
+            const int r = warp_last_le(rpre, e);
+            const uint32_t rw = __shfl_sync(0xffffffffu, rw_mine, r);
+            const int k = e - __shfl_sync(0xffffffffu, rpre, r);
+            const int32_t rp = __shfl_sync(0xffffffffu, rp_mine, r);
+            const int j = nth_set_bit(rw, k);
+            const uint32_t cm = __shfl_sync(0xffffffffu, cm_mine, j);
+            const int64_t cb = __shfl_sync(0xffffffffu, cb_mine, j);
+            pr[q] = (int64_t)rp + k;
+            pc[q] = cb + __popc(cm & ((1u << r) - 1u));
+            at[q] = e < total ? r * 32 + (j ^ r) : -1;
+            v[q] = e < total && pr[q] < capacity ? __ldg(val + pr[q]) : 0.f;
+        }
+#pragma unroll
+        for (int q = 0; q < kRounds; ++q) {
+            if (e00 + 32 * q < total && at[q] >= 0) {
+                tl[at[q]] = v[q];
+                if (pc[q] < capacity && pr[q] < capacity) t_pos[pr[q]] = (int32_t)pc[q];
+            }
         }
     }
     __syncwarp();

@@ -153,19 +153,16 @@ __global__ void __launch_bounds__(256) fp_oldbits_kernel(const int32_t *__restri
     const int32_t s = row_ptr[r], e = row_ptr[r + 1];
     for (int i = lane; i < wpr; i += 32) w[i] = 0u;
     __syncwarp();
-    // four independent column loads in flight per lane (the kernel is bound by
-    // their latency: one warp per row, few rows per SM)
-    int32_t k = s + lane;
-    for (; k + 96 < e; k += 128) {
-        int c[4];
+    // sixteen independent column loads in flight per lane: a row of up to 512
+    // stored entries in one round (the kernel is bound by their latency: one
+    // warp per row, few rows per SM)
+    for (int32_t k = s + lane; k < e; k += 512) {
+        int c[16];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) c[u] = __ldg(col + k + 32 * u);
+        for (int u = 0; u < 16; ++u) c[u] = k + 32 * u < e ? __ldg(col + k + 32 * u) : -1;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) atomicOr(&w[c[u] >> 5], 1u << (c[u] & 31));
-    }
-    for (; k < e; k += 32) {
-        const int c = __ldg(col + k);
-        atomicOr(&w[c >> 5], 1u << (c & 31));
+        for (int u = 0; u < 16; ++u)
+            if (c[u] >= 0) atomicOr(&w[c[u] >> 5], 1u << (c[u] & 31));
     }
     __syncwarp();
     for (int i = lane; i < wpr; i += 32) obits[r * wpr + i] = w[i];
