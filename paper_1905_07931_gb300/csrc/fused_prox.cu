@@ -38,8 +38,6 @@
 
 namespace csrt {
 
-int transpose_from_bits_ext(csrt_csr *w, const uint32_t *keepbits, const int32_t *wordpos, void *scratch,
-                            size_t scratch_bytes, cudaStream_t s);
 size_t transpose_scratch_bytes(int32_t rows, int32_t cols);
 
 // Segments (the unit of the per-row offsets) are 64 columns, two 32-column
