@@ -87,7 +87,22 @@ template <> struct FpShape<true> {
     static constexpr int kEpi = CSRT_FP_WRITE_EPI, kPre = CSRT_FP_WRITE_PRE, kGroup = CSRT_FP_WRITE_GROUP,
                          kStageWords = CSRT_FP_WRITE_STAGE_WORDS, kStages = kStageWords > 2 ? 2 : 3;
 };
-template <bool kWrite> constexpr int fp_threads() { return 64 + FpShape<kWrite>::kEpi * 32; }
+// Threads of a pass: the producer warps (TMA, MMA; with kSplit a whole
+// warpgroup of four, two of them idle) and the epilogue warps.
+template <bool kWrite, bool kSplit = false> constexpr int fp_threads() {
+    return (kSplit ? 128 : 64) + FpShape<kWrite>::kEpi * 32;
+}
+// kSplit (write pass): the producer warpgroup gives up registers, the four
+// epilogue warpgroups take them (setmaxnreg), within the launch's allocation
+// of 640 threads x 96 registers: 128 x 32 + 512 x 112 = 61,440. The 18-warp
+// launch caps every thread at 96 registers, where the write pass spills
+// (48-60 bytes); split, it does not (4096 x 9216 layer 136.2 -> 132.4 us,
+// 4096 x 4096 with the transposed copy 114.5 -> 109.6 us). A cap of 112 for
+// all 18 warps does not launch: registers are allocated for whole groups of
+// four warps.
+constexpr int kFpProdRegs = 32, kFpEpiRegs = 112;
+static_assert(128 * kFpProdRegs + FpShape<true>::kEpi * 32 * kFpEpiRegs <= fp_threads<true, true>() * 96,
+              "register split above the launch's allocation");
 // Per epilogue warp: 32 x 32 float buffers, row r's 16-byte chunk c at float
 // offset r*32 + ((c ^ (r & 7)) << 2), so that a row written as eight 16-byte
 // stores and a column read one element per lane are both free of bank
@@ -424,12 +439,13 @@ __device__ __forceinline__ void fp_write_compact(const float *xb, uint8_t *cb, f
 // written with coalesced stores.
 // kT: the transposed copy too (FpTArgs): its column counts per 32-row block
 // (count pass) or its arrays (write pass).
-template <bool kWrite, bool kT>
-__global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
+template <bool kWrite, bool kT, bool kSplit = false>
+__global__ void __launch_bounds__(fp_threads<kWrite, kSplit>(), 1)
     gemm_prox_tc_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                         FpArgs a, FpTArgs ta, int32_t tiles_n, int32_t num_tiles) {
     pdl_enter();
     constexpr int kEpi = FpShape<kWrite>::kEpi, kStages = FpShape<kWrite>::kStages;
+    constexpr int kProd = kSplit ? 4 : 2;   // warps before the epilogue warps
     constexpr int kFpPre = FpShape<kWrite>::kPre, kGroup = FpShape<kWrite>::kGroup;
     constexpr int kSpanCols = kTcBN / (kEpi / 4);   // columns per epilogue warp
     constexpr int kSpanWords = kSpanCols / 32;
@@ -478,7 +494,9 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = *tmem_slot;
-
+    if (warp < kProd) {
+    // every warp of a warpgroup runs the same setmaxnreg
+    if constexpr (kSplit) asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kFpProdRegs));
     if (warp == 0) {
         if (lane == 0) {
             int it = 0;
@@ -519,8 +537,10 @@ __global__ void __launch_bounds__(fp_threads<kWrite>(), 1)
             mma_commit(fin);
             mbar_wait(fin, 0);
         }
+    }
     } else {
-        const int e = warp - 2;
+        if constexpr (kSplit) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kFpEpiRegs));
+        const int e = warp - kProd;
         const int q = warp & 3;   // the TMEM lane quarter this warp may read
         const int h = e >> 2;     // column span within the tile
         const int64_t rowq = q * 32 + lane;
@@ -840,7 +860,7 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
 
     CUtensorMap ma, mb;
     CSRT_ARG(make_map(&ma, dy, m, n, kTcBM) && make_map(&mb, x, k, n, kTcBN), "tensor map encoding failed");
-    static bool attr_set[64] = {false};
+    static bool attr_set[64] = {false}, split_ok[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
@@ -852,8 +872,21 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, fp_smem_bytes<true>()));
         CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<false, true>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, fp_smem_bytes<false>()));
+        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<true, false, true>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, fp_smem_bytes<true>()));
+        CSRT_CHECK_CUDA(cudaFuncSetAttribute(gemm_prox_tc_kernel<true, true, true>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, fp_smem_bytes<true>()));
+        // the register split needs the launch to hold what it hands out (ptxas gives 96 per thread at
+        // 640 threads; the 18-warp write pass otherwise)
+        cudaFuncAttributes fa0{}, fa1{};
+        CSRT_CHECK_CUDA(cudaFuncGetAttributes(&fa0, gemm_prox_tc_kernel<true, false, true>));
+        CSRT_CHECK_CUDA(cudaFuncGetAttributes(&fa1, gemm_prox_tc_kernel<true, true, true>));
+        const int need = 128 * kFpProdRegs + FpShape<true>::kEpi * 32 * kFpEpiRegs;
+        split_ok[dev] = fa0.numRegs * fp_threads<true, true>() >= need &&
+                        fa1.numRegs * fp_threads<true, true>() >= need;
         attr_set[dev] = true;
     }
+    const bool split = dev >= 0 && dev < 64 && split_ok[dev];
     launch_pdl(fp_oldbits_kernel, dim3((unsigned)ceil_div<int64_t>(m, 8)), dim3(256), 0, s, w_in->row_ptr,
                w_in->col_idx, m, L.wpr, L.nt, obits, ostart);
     FpArgs a;
@@ -913,9 +946,15 @@ extern "C" int weight_grad_prox_update(const csrt_csr *w_in, const float *dy, co
         ta.t_val = w_out->t_val;
         ta.t_pos = w_out->t_pos;
     }
-    if (want_t)
+    if (want_t && split)
+        launch_pdl(gemm_prox_tc_kernel<true, true, true>, dim3(grid), dim3(fp_threads<true, true>()),
+                   fp_smem_bytes<true>(), s, ma, mb, a, ta, tiles_n, tiles);
+    else if (want_t)
         launch_pdl(gemm_prox_tc_kernel<true, true>, dim3(grid), dim3(fp_threads<true>()), fp_smem_bytes<true>(), s,
                    ma, mb, a, ta, tiles_n, tiles);
+    else if (split)
+        launch_pdl(gemm_prox_tc_kernel<true, false, true>, dim3(grid), dim3(fp_threads<true, true>()),
+                   fp_smem_bytes<true>(), s, ma, mb, a, ta, tiles_n, tiles);
     else
         launch_pdl(gemm_prox_tc_kernel<true, false>, dim3(grid), dim3(fp_threads<true>()), fp_smem_bytes<true>(), s,
                    ma, mb, a, ta, tiles_n, tiles);
